@@ -1,0 +1,193 @@
+"""Seeded synthetic workloads for the block-verify hot path.
+
+This module only draws random inputs of the right shapes and distributions; it holds
+none of the method's arithmetic (no softmax, no acceptance test, no attention).  Both
+the CUDA path and the CPU oracle are fed from it.
+
+The five workloads stand in for the paper's evaluation data (GSM8K ... MT-Bench,
+Section 3.1), which needs trained Qwen3 / DFlash models; they reproduce the shapes of
+those models instead:
+
+  tiny           1 seq, context 256, B=8, 4/2 heads, D=64, fp32, vocab 1024,
+                 policy hidden 256 over 9 candidates
+  qwen3_4b       1 seq, context 2048, B=16, 32/8 heads, D=128, bf16, vocab 151936
+  ragged         32 seqs, B_s in {8..24} (60% on 14-18), context U[512, 8192],
+                 Qwen3-4B heads, bf16, vocab 151936, policy N=32 over 2560-d states
+  drafter_bidir  16 seqs, context 4096, B=16 mask-token queries, bidirectional
+  long_context   8 seqs, context 32768, B=16, 32/8 heads, D=128, bf16, vocab 151936
+
+Block of B query positions = the anchor token plus gamma = B - 1 drafted tokens; the
+verify pass yields B target rows.  Draft tokens at T > 0 are drawn from the draft
+distribution with the Gumbel-max trick (a sampler of the drafter, not of the
+acceptance rule); at T = 0 they are the draft rows' argmax.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass, field
+
+import numpy as np
+
+CANDIDATES = np.arange(8, 25, 2, dtype=np.int32)  # {8, 10, ..., 24}
+
+
+@dataclass(frozen=True)
+class Workload:
+    name: str
+    seed: int
+    num_seqs: int
+    ctx: tuple  # per-sequence context length L_s (or a single value, repeated)
+    block: tuple  # per-sequence block size B_s
+    num_q_heads: int
+    num_kv_heads: int
+    head_dim: int
+    dtype: str  # "f32" or "bf16"
+    vocab: int
+    logit_std: float
+    temperatures: tuple
+    mask: str = "causal"
+    has_accept: bool = True
+    policy: dict = field(default_factory=dict)
+
+
+def _rng(seed: int, stream: int) -> np.random.Generator:
+    return np.random.default_rng([seed, stream])
+
+
+def f32_to_bf16_bits(x: np.ndarray) -> np.ndarray:
+    """Round float32 values to bfloat16 (nearest, ties to even); returns the uint16 bits."""
+    u = np.ascontiguousarray(x, dtype=np.float32).view(np.uint32).astype(np.uint64)
+    u = u + 0x7FFF + ((u >> 16) & 1)
+    return (u >> 16).astype(np.uint16)
+
+
+def bf16_bits_to_f32(b: np.ndarray) -> np.ndarray:
+    return (np.ascontiguousarray(b, dtype=np.uint16).astype(np.uint32) << 16).view(np.float32)
+
+
+def _ragged_blocks(seed: int, n: int) -> tuple:
+    sizes = np.array([8, 10, 12, 14, 16, 18, 20, 24])
+    probs = np.array([0.08, 0.08, 0.08, 0.2, 0.2, 0.2, 0.08, 0.08])
+    return tuple(int(b) for b in _rng(seed, 90).choice(sizes, size=n, p=probs))
+
+
+def _ragged_ctx(seed: int, n: int) -> tuple:
+    return tuple(int(c) for c in _rng(seed, 91).integers(512, 8192, size=n, endpoint=True))
+
+
+def get(name: str) -> Workload:
+    """The named workload (shapes and seeds fixed)."""
+    if name == "tiny":
+        return Workload("tiny", 0, 1, (256,), (8,), 4, 2, 64, "f32", 1024, 2.0, (1.0,),
+                        policy=dict(num_reqs=1, d_in=1024, hidden=256, wdtype="f32", feat_std=2.0))
+    if name == "qwen3_4b":
+        return Workload("qwen3_4b", 2, 1, (2048,), (16,), 32, 8, 128, "bf16", 151936, 3.0, (1.0, 0.0))
+    if name == "ragged":
+        return Workload("ragged", 3, 32, _ragged_ctx(3, 32), _ragged_blocks(3, 32), 32, 8, 128, "bf16",
+                        151936, 3.0, (1.0,),
+                        policy=dict(num_reqs=32, d_in=2560, hidden=2048, wdtype="bf16", feat_std=1.0))
+    if name == "drafter_bidir":
+        return Workload("drafter_bidir", 4, 16, (4096,) * 16, (16,) * 16, 32, 8, 128, "bf16", 151936, 3.0,
+                        (), mask="bidir", has_accept=False)
+    if name == "long_context":
+        return Workload("long_context", 5, 8, (32768,) * 8, (16,) * 8, 32, 8, 128, "bf16", 151936, 3.0,
+                        (0.0, 1.0))
+    raise KeyError(name)
+
+
+NAMES = ("tiny", "qwen3_4b", "ragged", "drafter_bidir", "long_context")
+
+
+def custom(name="custom", seed=0, ctx=(64,), block=(8,), num_q_heads=4, num_kv_heads=2, head_dim=128,
+           dtype="bf16", vocab=1000, logit_std=3.0, temperatures=(1.0,), mask="causal", policy=None) -> Workload:
+    """A workload of arbitrary shape (used for small parity cases and edge cases)."""
+    ctx = tuple(int(c) for c in ctx)
+    block = tuple(int(b) for b in block)
+    assert len(ctx) == len(block)
+    return Workload(name, seed, len(ctx), ctx, block, num_q_heads, num_kv_heads, head_dim, dtype, vocab,
+                    logit_std, tuple(temperatures), mask=mask, policy=policy or {})
+
+
+def offsets(lengths) -> np.ndarray:
+    out = np.zeros(len(lengths) + 1, dtype=np.int32)
+    out[1:] = np.cumsum(np.asarray(lengths, dtype=np.int64))
+    return out
+
+
+def attention_inputs(w: Workload) -> dict:
+    """Q [sum B_s, Hq, D], K/V [sum (L_s + B_s), Hkv, D] ~ N(0,1) and the ragged offsets.
+
+    For bf16 workloads the arrays are uint16 bf16 bits; for f32 they are float32.
+    """
+    blocks = np.asarray(w.block, dtype=np.int64)
+    kv_lens = np.asarray(w.ctx, dtype=np.int64) + blocks
+    cu_q = offsets(blocks)
+    cu_kv = offsets(kv_lens)
+    tq, tkv = int(cu_q[-1]), int(cu_kv[-1])
+    out = dict(cu_q=cu_q, cu_kv=cu_kv, num_q_heads=w.num_q_heads, num_kv_heads=w.num_kv_heads,
+               head_dim=w.head_dim, dtype=w.dtype, mask=w.mask, max_q_len=int(blocks.max(initial=0)),
+               max_kv_len=int(kv_lens.max(initial=0)))
+    shapes = dict(q=(tq, w.num_q_heads, w.head_dim), k=(tkv, w.num_kv_heads, w.head_dim),
+                  v=(tkv, w.num_kv_heads, w.head_dim))
+    for i, key in enumerate(("q", "k", "v")):
+        x = _rng(w.seed, 10 + i).standard_normal(shapes[key], dtype=np.float32)
+        out[key] = f32_to_bf16_bits(x) if w.dtype == "bf16" else x
+    return out
+
+
+def accept_inputs(w: Workload, temperature: float, planted_match: float = 0.0) -> dict:
+    """Target / draft logits, draft tokens and uniforms for one acceptance step.
+
+    target rows ~ N(0, logit_std^2) [sum (gamma_s + 1), V]; draft rows = matching target
+    row + N(0, 1) [sum gamma_s, V]; gamma_s = B_s - 1.  With planted_match > 0 each draft
+    row is, with that probability, an exact copy of its target row (full agreement).
+    """
+    gammas = np.asarray(w.block, dtype=np.int64) - 1
+    cu_draft = offsets(gammas)
+    s = w.num_seqs
+    td = int(cu_draft[-1])
+    V = w.vocab
+    target = _rng(w.seed, 20).standard_normal((td + s, V), dtype=np.float32) * np.float32(w.logit_std)
+    noise = _rng(w.seed, 21).standard_normal((td, V), dtype=np.float32)
+    # target row index of drafted position i of sequence s is cu_draft[s] + s + i
+    seq_of_draft = np.repeat(np.arange(s), gammas)
+    trow = np.arange(td) + seq_of_draft
+    draft = target[trow] + noise
+    if planted_match > 0.0:
+        copy = _rng(w.seed, 22).random(td) < planted_match
+        draft[copy] = target[trow[copy]]
+    if temperature > 0.0:
+        g = _rng(w.seed, 23).gumbel(size=(td, V)).astype(np.float32)
+        tokens = np.argmax(draft / np.float32(temperature) + g, axis=1).astype(np.int32)
+    else:
+        tokens = np.argmax(draft, axis=1).astype(np.int32)
+    u_accept = _rng(w.seed, 24).random(td, dtype=np.float32)
+    u_sample = _rng(w.seed, 25).random(s, dtype=np.float32)
+    return dict(target_logits=target, draft_logits=draft, draft_tokens=tokens, cu_draft=cu_draft,
+                u_accept=u_accept, u_sample=u_sample, vocab=V, temperature=float(temperature))
+
+
+def policy_inputs(w: Workload) -> dict:
+    """Pooled-feature matrix (4 prefill rows per request, the last one pooled) and MLP weights."""
+    p = w.policy
+    n, d_in, hidden = p["num_reqs"], p["d_in"], p["hidden"]
+    c = len(CANDIDATES)
+    rows_per_req = 4
+    feats = _rng(w.seed, 30).standard_normal((n * rows_per_req, d_in), dtype=np.float32) * np.float32(p["feat_std"])
+    row_index = (np.arange(n, dtype=np.int32) * rows_per_req + rows_per_req - 1).astype(np.int32)
+    w1 = _rng(w.seed, 31).standard_normal((hidden, d_in), dtype=np.float32) * np.float32(1.0 / np.sqrt(d_in))
+    b1 = _rng(w.seed, 32).standard_normal(hidden, dtype=np.float32) * np.float32(0.1)
+    w2 = _rng(w.seed, 33).standard_normal((c, hidden), dtype=np.float32) * np.float32(1.0 / np.sqrt(hidden))
+    b2 = _rng(w.seed, 34).standard_normal(c, dtype=np.float32) * np.float32(0.1)
+    out = dict(row_index=row_index, b1=b1, b2=b2, candidates=CANDIDATES.copy(), wdtype=p["wdtype"])
+    if p["wdtype"] == "bf16":
+        out.update(feats=f32_to_bf16_bits(feats), w1=f32_to_bf16_bits(w1), w2=f32_to_bf16_bits(w2))
+    else:
+        out.update(feats=feats, w1=w1, w2=w2)
+    return out
+
+
+def as_f64(x: np.ndarray, dtype: str) -> np.ndarray:
+    """The exact fp64 values of an f32 array or of bf16 bits."""
+    if dtype == "bf16":
+        return bf16_bits_to_f32(x).astype(np.float64)
+    return np.asarray(x, dtype=np.float32).astype(np.float64)
