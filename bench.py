@@ -1,0 +1,458 @@
+"""Benchmark of the block-verify hot path on GB300.
+
+One step = one block-verify pass of the Qwen3-4B-shaped workload (1 sequence, context 2048,
+block B = 16, 32/8 heads, head_dim 128, bf16 KV; acceptance over a 151936-token vocabulary at
+T = 1): bp_block_attention (causal within the block) followed by bp_spec_accept.  Inputs are
+seeded synthetic data already resident in HBM; eight copies (8 x 27.6 MB > 129 MB L2) are
+rotated so that no step finds its inputs in L2.  Steps are replayed from a CUDA graph and timed
+with CUDA events on the launching stream.
+
+The JSON line also carries: the roofline of the dominant kernel (timed alone, live), every
+hot-path row timed on its own (drafter bidirectional attention, greedy acceptance, the policy
+head), an end-to-end figure through the public API from pinned host buffers, the CPU oracle's
+throughput on the host cores, and the SM clocks sampled during the timed region.
+
+  python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+Under torchrun each rank runs an independent replica on its own GPU (no data-path collective).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "verified tokens/sec and % of HBM roofline for block-verify attention+accept, 1 GB300"
+WORKLOAD = "qwen3_4b"
+COPIES = 8
+L2_BYTES = 129e6
+
+
+def peaks():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        return float(d["hbm_gbs"]), "measured"
+    return 6800.0, "fallback"
+
+
+def dist_env():
+    return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
+
+
+# ----------------------------------------------------------------------------- byte counts
+def attention_bytes(w) -> float:
+    """K and V read once, Q read and O written once (bf16)."""
+    e = 2
+    blocks = np.asarray(w.block)
+    kv = (np.asarray(w.ctx) + blocks).sum() * w.num_kv_heads * w.head_dim * 2 * e
+    qo = 2 * blocks.sum() * w.num_q_heads * w.head_dim * e
+    return float(kv + qo)
+
+
+def accept_bytes(w, temperature: float) -> float:
+    """Target rows (gamma+1 per sequence) and, at T > 0, draft rows (gamma), fp32, read once."""
+    g = np.asarray(w.block) - 1
+    rows = (g + 1).sum() + (g.sum() if temperature > 0 else 0)
+    return float(rows * w.vocab * 4)
+
+
+def policy_bytes(pin) -> float:
+    return float(pin["w1"].nbytes + pin["w2"].nbytes)
+
+
+# ----------------------------------------------------------------------------- clocks
+class ClockSampler:
+    QUERY = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,clocks_event_reasons.hw_slowdown,"
+             "clocks_event_reasons.hw_thermal_slowdown,clocks_event_reasons.sw_thermal_slowdown,"
+             "clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, gpu_index: int):
+        self.gpu = gpu_index
+        self.proc = None
+
+    def __enter__(self):
+        try:
+            self.proc = subprocess.Popen(["nvidia-smi", "-i", str(self.gpu), f"--query-gpu={self.QUERY}",
+                                          "--format=csv,noheader,nounits", "-lms", "50"],
+                                         stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except OSError:
+            self.proc = None
+        time.sleep(0.15)
+        return self
+
+    def __exit__(self, *exc):
+        self.out = ""
+        if self.proc is not None:
+            time.sleep(0.1)
+            self.proc.terminate()
+            try:
+                self.out, _ = self.proc.communicate(timeout=5)
+            except subprocess.TimeoutExpired:
+                self.proc.kill()
+                self.out, _ = self.proc.communicate()
+
+    def summary(self):
+        sm, mx, reasons = [], None, set()
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in (self.out or "").strip().splitlines():
+            parts = [x.strip() for x in line.split(",")]
+            if len(parts) < 8:
+                continue
+            try:
+                sm.append(float(parts[0]))
+                mx = float(parts[1])
+            except ValueError:
+                continue
+            for name, flag in zip(names, parts[4:8]):
+                if flag.lower() == "active":
+                    reasons.add(name)
+        loaded = [x for x in sm if mx and x > 0.5 * mx] or sm
+        return {"sm_mhz": statistics.median(loaded) if loaded else None, "sm_max_mhz": mx,
+                "reasons": sorted(reasons), "samples": len(sm)}
+
+
+# ----------------------------------------------------------------------------- our arm
+def run_ours(args):
+    import torch
+
+    import paper_2606_31315_gb300 as bp
+    from paper_2606_31315_gb300 import workloads as wl
+
+    rank, world, local = dist_env()
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.init_process_group("nccl")
+    torch.cuda.set_device(local)
+    dev = torch.device("cuda", local)
+    bp.build()
+    bp.load()
+    w = wl.get(WORKLOAD)
+    a = wl.attention_inputs(w)
+    acc = wl.accept_inputs(w, 1.0)
+    acc0 = wl.accept_inputs(w, 0.0)
+
+    def bf(x):
+        return torch.from_numpy(x.view(np.int16)).to(dev).view(torch.bfloat16)
+
+    def t(x):
+        return torch.from_numpy(np.ascontiguousarray(x)).to(dev)
+
+    copies = []
+    for _ in range(COPIES):
+        copies.append(dict(q=bf(a["q"]), k=bf(a["k"]), v=bf(a["v"]), o=torch.empty(a["q"].shape, dtype=torch.bfloat16,
+                                                                                     device=dev),
+                           target=t(acc["target_logits"]), draft=t(acc["draft_logits"]), tok=t(acc["draft_tokens"]),
+                           ua=t(acc["u_accept"]), us=t(acc["u_sample"]), tok0=t(acc0["draft_tokens"])))
+    cu_q, cu_kv, cu_d = t(a["cu_q"]), t(a["cu_kv"]), t(acc["cu_draft"])
+    S, TD, V = w.num_seqs, int(acc["cu_draft"][-1]), w.vocab
+    n_acc = torch.empty(S, dtype=torch.int32, device=dev)
+    out_tok = torch.empty(TD + S, dtype=torch.int32, device=dev)
+    ws_a = bp.workspace(bp.block_attention_workspace_size(S, a["max_q_len"], 32, 8, 128), dev)
+    ws_s = bp.workspace(bp.spec_accept_workspace_size(S, TD, V), dev)
+    stream = torch.cuda.Stream(device=dev)
+
+    def attn(c, mask=bp.MASK_CAUSAL):
+        bp.block_attention(c["q"], c["k"], c["v"], cu_q, cu_kv, a["max_q_len"], a["max_kv_len"], mask=mask,
+                           out=c["o"], ws=ws_a, stream=stream)
+
+    def accept(c, temp=1.0):
+        if temp > 0:
+            bp.spec_accept(c["target"], c["draft"], c["tok"], cu_d, temp, c["ua"], c["us"], n_accepted=n_acc,
+                           out_tokens=out_tok, want_accept_prob=False, ws=ws_s, stream=stream)
+        else:
+            bp.spec_accept(c["target"], None, c["tok0"], cu_d, 0.0, None, None, n_accepted=n_acc, out_tokens=out_tok,
+                           want_accept_prob=False, ws=ws_s, stream=stream)
+
+    def step(c):
+        attn(c)
+        accept(c)
+
+    def graph_of(fn):
+        """One CUDA graph running fn once on each input copy."""
+        with torch.cuda.stream(stream):
+            for c in copies:  # warm the code paths outside capture
+                fn(c)
+        stream.synchronize()
+        g = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(g, stream=stream):
+            for c in copies:
+                fn(c)
+        stream.synchronize()
+        return g
+
+    def time_graph(g, reps):
+        """Seconds per replay (events on the launching stream)."""
+        e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+        torch.cuda.synchronize(dev)
+        e0.record(stream)
+        for _ in range(reps):
+            g.replay()
+        e1.record(stream)
+        e1.synchronize()
+        return e0.elapsed_time(e1) / 1e3 / reps
+
+    def barrier():
+        if world > 1:
+            import torch.distributed as dist
+
+            dist.barrier()
+
+    # ---------------- the timed region: exactly K steps
+    g_step = graph_of(step)
+    reps_w = max(1, -(-args.warmup // COPIES))
+    with torch.cuda.stream(stream):
+        for _ in range(reps_w):
+            g_step.replay()
+    stream.synchronize()
+    full, rem = divmod(args.steps, COPIES)
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    barrier()
+    torch.cuda.synchronize(dev)
+    with ClockSampler(local) as clk:
+        with torch.cuda.stream(stream):
+            e0.record(stream)
+            for _ in range(full):
+                g_step.replay()
+            for i in range(rem):
+                step(copies[i])
+            e1.record(stream)
+        e1.synchronize()
+    torch.cuda.synchronize(dev)
+    barrier()
+    elapsed = e0.elapsed_time(e1) / 1e3
+    if world > 1:
+        import torch.distributed as dist
+
+        tt = torch.tensor([elapsed], device=dev, dtype=torch.float64)
+        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
+        elapsed = float(tt.item())
+    tokens_per_step = int(np.sum(w.block))
+    value = world * tokens_per_step * args.steps / elapsed
+    ms_per_step = elapsed / args.steps * 1e3
+    step_bytes = attention_bytes(w) + accept_bytes(w, 1.0)
+    peak, peak_kind = peaks()
+
+    # ---------------- each hot-path row timed alone (same rotation, graph replays)
+    reps = max(20, min(2000, args.steps // COPIES))
+    t_attn = time_graph(graph_of(attn), reps) / COPIES
+    t_acc = time_graph(graph_of(accept), reps) / COPIES
+    t_bidir = time_graph(graph_of(lambda c: attn(c, bp.MASK_BIDIR)), reps) / COPIES
+    t_acc0 = time_graph(graph_of(lambda c: accept(c, 0.0)), reps) / COPIES
+    pw = wl.get("ragged")
+    pin = wl.policy_inputs(pw)
+    pf = {k: (bf(pin[k]) if k in ("feats", "w1", "w2") else t(pin[k])) for k in
+          ("feats", "w1", "w2", "b1", "b2", "candidates", "row_index")}
+    ws_p = bp.workspace(bp.policy_select_workspace_size(32, 2048, 9), dev)
+    bsz = torch.empty(32, dtype=torch.int32, device=dev)
+
+    def policy(_c):
+        bp.policy_select(pf["feats"], pf["w1"], pf["b1"], pf["w2"], pf["b2"], pf["candidates"],
+                         row_index=pf["row_index"], block_size=bsz, want_logits=False, ws=ws_p, stream=stream)
+
+    t_pol = time_graph(graph_of(policy), reps) / COPIES
+
+    def row(tsec, nbytes, kernels):
+        gbs = nbytes / tsec / 1e9
+        return {"us": round(tsec * 1e6, 3), "bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
+                "kernels": kernels}
+
+    rows = {
+        "a2_a4_verify_attention_causal": row(t_attn, attention_bytes(w), ["attn_bf16_tc_kernel"]),
+        "a3_drafter_attention_bidir": row(t_bidir, attention_bytes(w), ["attn_bf16_tc_kernel"]),
+        "a5_a6_accept_t1": row(t_acc, accept_bytes(w, 1.0), ["accept_rows_kernel<10,false,true>"]),
+        "a7_accept_greedy_t0": row(t_acc0, accept_bytes(w, 0.0), ["accept_rows_kernel<10,true,true>"]),
+        "a1_policy_head_32req_2560x2048": row(t_pol, policy_bytes(pin), ["policy_hidden_kernel", "policy_out_kernel"]),
+    }
+    dom_name, dom_t, dom_bytes = ("accept_rows_kernel", t_acc, accept_bytes(w, 1.0))
+    traffic = committed_traffic(dom_name)
+    roofline = {"bound": "hbm", "kernel": dom_name, "achieved": round(dom_bytes / dom_t / 1e9, 1), "peak": peak,
+                "peak_kind": f"{peak_kind} hbm_gbs (burst copy)", "unit": "GB/s",
+                "frac": round(dom_bytes / dom_t / 1e9 / peak, 4), "traffic": traffic,
+                "algorithmic_bytes": dom_bytes, "avg_launch_us": round(dom_t * 1e6, 3)}
+
+    # ---------------- end to end through the public API from pinned host buffers
+    e2e = run_e2e(bp, torch, dev, stream, a, acc, w, min(args.steps, 200))
+
+    result = {
+        "metric": METRIC, "value": round(value, 1), "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+        "warmup": args.warmup, "ms_per_step": round(ms_per_step, 6), "higher_is_better": True, "scaling": "weak",
+        "vs_baseline": None, "dtype": "bf16", "data": "synthetic",
+        "config": {"workload": "qwen3_4b: 1 seq, context 2048, block 16, 32/8 heads, head_dim 128, bf16 KV; "
+                               "acceptance over vocab 151936 fp32 logits at T=1",
+                   "global_batch": world, "seq_len": 2064, "parallelism": f"replicas x{world}",
+                   "l2": f"{COPIES} rotating input copies ({COPIES * step_bytes / 1e6:.0f} MB) > 129 MB L2",
+                   "graph": f"CUDA graph of {COPIES} steps"},
+        "hbm_roofline": {"step_bytes": step_bytes, "achieved_gbs": round(step_bytes / (elapsed / args.steps) / 1e9, 1),
+                         "peak": peak, "frac": round(step_bytes / (elapsed / args.steps) / 1e9 / peak, 4),
+                         "roofline_tokens_per_s": round(tokens_per_step / (step_bytes / (peak * 1e9)), 1)},
+        "roofline": roofline,
+        "rows": rows,
+        "e2e": e2e,
+        "gpu_launches": 2 * args.steps,
+        "clocks": clk.summary(),
+    }
+    if rank == 0:
+        result["cpu_baseline"] = cpu_baseline(seconds=args.cpu_seconds)
+        print(json.dumps(result), flush=True)
+    if world > 1:
+        import torch.distributed as dist
+
+        dist.destroy_process_group()
+
+
+def committed_traffic(kernel: str):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken on the current source."""
+    path = os.path.join(ROOT, "profiles", "traffic.json")
+    if not os.path.exists(path):
+        return None
+    with open(path) as f:
+        d = json.load(f).get(kernel)
+    if not d:
+        return None
+    src = os.path.join(ROOT, "paper_2606_31315_gb300", "csrc", d["source"])
+    with open(src, "rb") as f:
+        digest = hashlib.sha256(f.read()).hexdigest()[:16]
+    return d["dram_bytes_per_launch"] if digest == d["source_sha256_16"] else None
+
+
+def run_e2e(bp, torch, dev, stream, a, acc, w, steps):
+    """Same metric through the public API with inputs in pinned host memory: every step copies
+    its inputs host->device, runs both calls and copies the emitted tokens back."""
+    def pin(x, dtype=None):
+        tt = torch.from_numpy(np.ascontiguousarray(x.view(np.int16) if dtype == "bf16" else x))
+        return tt.pin_memory()
+
+    host = dict(q=pin(a["q"], "bf16"), k=pin(a["k"], "bf16"), v=pin(a["v"], "bf16"), cu_q=pin(a["cu_q"]),
+                cu_kv=pin(a["cu_kv"]), target=pin(acc["target_logits"]), draft=pin(acc["draft_logits"]),
+                tok=pin(acc["draft_tokens"]), cu_d=pin(acc["cu_draft"]), ua=pin(acc["u_accept"]),
+                us=pin(acc["u_sample"]))
+    devb = {k: torch.empty(v.shape, dtype=v.dtype, device=dev) for k, v in host.items()}
+    S, TD = w.num_seqs, int(acc["cu_draft"][-1])
+    out_h = torch.empty(TD + S, dtype=torch.int32).pin_memory()
+    nacc_h = torch.empty(S, dtype=torch.int32).pin_memory()
+    n_acc = torch.empty(S, dtype=torch.int32, device=dev)
+    out_tok = torch.empty(TD + S, dtype=torch.int32, device=dev)
+    o = torch.empty(a["q"].shape, dtype=torch.bfloat16, device=dev)
+    ws_a = bp.workspace(bp.block_attention_workspace_size(S, a["max_q_len"], 32, 8, 128), dev)
+    ws_s = bp.workspace(bp.spec_accept_workspace_size(S, TD, w.vocab), dev)
+    h2d = sum(v.numel() * v.element_size() for v in host.values())
+    d2h = out_h.numel() * 4 + nacc_h.numel() * 4
+
+    def one():
+        with torch.cuda.stream(stream):
+            for k, v in host.items():
+                devb[k].copy_(v, non_blocking=True)
+            q = devb["q"].view(torch.bfloat16)
+            k_ = devb["k"].view(torch.bfloat16)
+            v_ = devb["v"].view(torch.bfloat16)
+            bp.block_attention(q, k_, v_, devb["cu_q"], devb["cu_kv"], a["max_q_len"], a["max_kv_len"], out=o,
+                               ws=ws_a, stream=stream)
+            bp.spec_accept(devb["target"], devb["draft"], devb["tok"], devb["cu_d"], 1.0, devb["ua"], devb["us"],
+                           n_accepted=n_acc, out_tokens=out_tok, want_accept_prob=False, ws=ws_s, stream=stream)
+            out_h.copy_(out_tok, non_blocking=True)
+            nacc_h.copy_(n_acc, non_blocking=True)
+
+    for _ in range(5):
+        one()
+    stream.synchronize()
+    e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+    e0.record(stream)
+    for _ in range(steps):
+        one()
+    e1.record(stream)
+    e1.synchronize()
+    sec = e0.elapsed_time(e1) / 1e3 / steps
+    return {"value": round(int(np.sum(w.block)) / sec, 1), "unit": "tokens/s", "h2d_bytes_per_step": int(h2d),
+            "d2h_bytes_per_step": int(d2h), "steps": steps, "ms_per_step": round(sec * 1e3, 4)}
+
+
+# ----------------------------------------------------------------------------- CPU oracle
+def oracle_step_fn():
+    import oracle
+    from paper_2606_31315_gb300 import workloads as wl
+
+    oracle.build()
+    w = wl.get(WORKLOAD)
+    a = wl.attention_inputs(w)
+    acc = wl.accept_inputs(w, 1.0)
+    q, k, v = (wl.as_f64(a[x], "bf16") for x in ("q", "k", "v"))
+
+    def step():
+        oracle.block_attention(q, k, v, a["cu_q"], a["cu_kv"], w.num_kv_heads, oracle.MASK_CAUSAL)
+        oracle.spec_accept(acc["target_logits"], acc["draft_logits"], acc["draft_tokens"], acc["cu_draft"], 1.0,
+                           acc["u_accept"], acc["u_sample"])
+
+    return step, int(np.sum(w.block)), oracle.num_threads()
+
+
+def cpu_baseline(seconds: float = 10.0, max_steps: int | None = None):
+    """The fp64 oracle, as it stands, on the host cores: full qwen3_4b steps for a bounded time."""
+    step, tokens, cores = oracle_step_fn()
+    step()  # first call pays for page faults
+    n, t0 = 0, time.perf_counter()
+    while True:
+        step()
+        n += 1
+        el = time.perf_counter() - t0
+        if el >= seconds or (max_steps is not None and n >= max_steps):
+            break
+    return {"value": round(tokens * n / el, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+            "sample": f"{n} full qwen3_4b steps (causal attention + T=1 acceptance) in {el:.1f} s"}
+
+
+def run_reference(args):
+    rank, world, _ = dist_env()
+    if rank != 0:
+        return
+    step, tokens, cores = oracle_step_fn()
+    for _ in range(args.warmup):
+        step()
+    t0 = time.perf_counter()
+    for _ in range(args.steps):
+        step()
+    el = time.perf_counter() - t0
+    value = tokens * args.steps / el
+    res = {"impl": "reference", "metric": METRIC, "value": round(value, 2), "unit": "tokens/s", "n_gpus": world,
+           "steps": args.steps, "warmup": args.warmup, "ms_per_step": round(el / args.steps * 1e3, 3),
+           "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic",
+           "config": {"workload": "qwen3_4b: 1 seq, context 2048, block 16, 32/8 heads, head_dim 128, bf16 KV; "
+                                  "acceptance over vocab 151936 fp32 logits at T=1", "global_batch": 1,
+                      "seq_len": 2064},
+           "cpu_baseline": {"value": round(value, 2), "unit": "tokens/s", "cores": cores, "kind": "oracle",
+                            "sample": f"{args.steps} full qwen3_4b steps on the host cores"},
+           "e2e": {"value": round(value, 2), "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(res), flush=True)
+
+
+def main():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=None)
+    ap.add_argument("--warmup", type=int, default=None)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--cpu-seconds", type=float, default=10.0)
+    args = ap.parse_args()
+    if args.impl == "reference":
+        args.steps = 20 if args.steps is None else args.steps
+        args.warmup = 3 if args.warmup is None else args.warmup
+        run_reference(args)
+    else:
+        args.steps = 100_000 if args.steps is None else args.steps
+        args.warmup = 800 if args.warmup is None else max(3, args.warmup)
+        run_ours(args)
+
+
+if __name__ == "__main__":
+    main()

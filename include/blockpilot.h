@@ -1,0 +1,173 @@
+/*
+ * blockpilot.h -- C ABI of the GB300 (sm_103a) block-verify hot path of BlockPilot
+ * (instance-adaptive block sizes for diffusion-based speculative decoding,
+ * arxiv 2606.31315).
+ *
+ * Three operations, one per stage of the per-request pipeline of Section 2.4:
+ *
+ *   bp_policy_select    once per request: the block-size predictor (Sections 2.3, 2.4)
+ *   bp_block_attention  every step: block attention of the drafter (bidirectional within
+ *                       the block) and of the target's verify pass (causal within the block)
+ *                       over the KV cache (Section 2.1, Figure 1)
+ *   bp_spec_accept      every step: lossless acceptance of the drafted block over the full
+ *                       vocabulary -- the longest accepted prefix plus one corrected or bonus
+ *                       token (Figure 1; Section 1)
+ *
+ * Conventions shared by every entry point
+ *   - Pointers to tensors are DEVICE pointers (cudaMalloc / torch allocations), owned by
+ *     the caller; the library never allocates, frees or retains them after the call.
+ *   - `stream` is a cudaStream_t (NULL = legacy default stream).  Calls only enqueue work:
+ *     they return before the GPU has run it and never synchronize, except bp_get_status.
+ *   - `workspace` is caller-owned device scratch of at least the size the matching
+ *     *_workspace_size function returns, 256-byte aligned, ZERO-FILLED BEFORE ITS FIRST
+ *     USE.  Every call leaves it in a state the next call can use (counters back at zero);
+ *     its first 16 bytes hold a sticky device error word read by bp_get_status.  Two calls
+ *     that may run concurrently need distinct workspaces.
+ *   - Host-checkable problems (NULL pointers, unsupported shapes, a workspace that is too
+ *     small) return an error code immediately and enqueue nothing.  Problems only the GPU
+ *     sees (a draft token id outside [0, V), a bounded wait that timed out) set the
+ *     workspace error word; the outputs of that call are then undefined.
+ *   - There is no CPU fallback: without a usable sm_103a device the calls return
+ *     BP_ERR_CUDA.
+ */
+#ifndef BLOCKPILOT_H
+#define BLOCKPILOT_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+#define BP_ABI_VERSION 1
+
+/* Symbols of the ABI are exported; everything else in the library is hidden. */
+#if defined(__GNUC__)
+#define BP_API __attribute__((visibility("default")))
+#else
+#define BP_API
+#endif
+
+typedef enum {
+    BP_OK = 0,
+    BP_ERR_INVALID_ARG = 1, /* NULL pointer, negative size, inconsistent shape */
+    BP_ERR_UNSUPPORTED = 2, /* valid but not implemented (e.g. bf16 attention with head_dim != 128) */
+    BP_ERR_CUDA = 3,        /* a CUDA runtime/driver call failed (no device, launch failure) */
+    BP_ERR_WORKSPACE = 4,   /* workspace NULL, misaligned or smaller than required */
+    BP_ERR_TIMEOUT = 5,     /* a device-side bounded wait expired (from bp_get_status) */
+    BP_ERR_DEVICE_FLAG = 6  /* a device-side argument check failed (from bp_get_status) */
+} bp_status;
+
+typedef enum {
+    BP_MASK_CAUSAL_BLOCK = 0, /* target verify: block query i sees context + block keys 0..i */
+    BP_MASK_BIDIR_BLOCK = 1   /* dLLM drafter: every block query sees context + whole block */
+} bp_mask;
+
+typedef enum { BP_F32 = 0, BP_BF16 = 1 } bp_dtype;
+
+/* ---------------------------------------------------------------------------------
+ * Block attention.  Section 2.1 (the drafter proposes B tokens in one forward pass and
+ * the target verifies them in one parallel pass) and the Figure 1 caption.
+ *
+ * For every sequence s, query head h and block position i:
+ *   O[i,h] = sum_j softmax_j(scale * <q_{i,h}, k_{j,h/g}> + M_ij) v_{j,h/g},  g = Hq/Hkv
+ * Sequence s owns query rows [cu_q[s], cu_q[s+1]) -- its block, B_s = cu_q[s+1]-cu_q[s]
+ * rows -- and key/value rows [cu_kv[s], cu_kv[s+1]): its L_s context rows followed by the
+ * block's own B_s rows (so cu_kv[s+1]-cu_kv[s] = L_s + B_s >= B_s).
+ * Mask: BP_MASK_CAUSAL_BLOCK lets block query i see keys 0 .. L_s+i; BP_MASK_BIDIR_BLOCK
+ * lets every block query see all L_s+B_s keys.
+ *
+ *   q, o     [total_q][num_q_heads][head_dim]   dtype (o written in dtype)
+ *   k, v     [total_kv][num_kv_heads][head_dim] dtype; 16-byte aligned base addresses
+ *   lse      [total_q][num_q_heads] float32, natural-log log-sum-exp of the scaled masked
+ *            scores of each output row; may be NULL
+ *   cu_q, cu_kv  [num_seqs+1] int32 device arrays, non-decreasing, cu_*[0] = 0,
+ *            cu_q[num_seqs] = total_q, cu_kv[num_seqs] = total_kv
+ *   max_q_len, max_kv_len  host-side upper bounds of B_s and L_s+B_s
+ *   dtype    BP_BF16 (tensor-core path, head_dim 128) or BP_F32 (head_dim <= 128)
+ *   softmax_scale  0 selects 1/sqrt(head_dim)
+ * Limits: 1 <= num_kv_heads, num_q_heads % num_kv_heads == 0, max_q_len <= 64,
+ * max_q_len <= max_kv_len.  Every key row must be finite (bf16 or fp32 values).
+ * ------------------------------------------------------------------------------- */
+BP_API size_t bp_block_attention_workspace_size(int num_seqs, int max_q_len, int num_q_heads, int num_kv_heads,
+                                         int head_dim);
+BP_API int bp_block_attention(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
+                       const int32_t* cu_kv, int num_seqs, int total_q, int total_kv, int max_q_len,
+                       int max_kv_len, int num_q_heads, int num_kv_heads, int head_dim, int dtype, int mask,
+                       float softmax_scale, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------
+ * Lossless speculative acceptance over the full vocabulary.  Figure 1 caption (the
+ * target accepts the longest consistent prefix of the drafted block), Section 1 and
+ * Section 3.1 Metrics (the target's output distribution is preserved exactly).  The
+ * paper leaves the rule to standard speculative sampling; this library implements:
+ *
+ *   p_i = softmax(target_row_i / T), q_i = softmax(draft_row_i / T)
+ *   a_i = min(1, p_i(x_i) / q_i(x_i))         (q=0<p gives 1; p=q=0 gives 0)
+ *   k   = first i < gamma_s with u_accept_i >= a_i, else gamma_s
+ *   emitted token at slot k: the smallest t with C_t > u_sample_s * Z, C_t = sum_{j<=t} w_j,
+ *   Z = sum_j w_j, where w = max(0, p_k - q_k) when k < gamma_s (w = p_k if that residual
+ *   is identically zero) and w = p_gamma (the bonus row) when every draft was accepted.
+ * temperature == 0 is greedy: accept iff x_i == argmax(target_row_i) (lowest index on
+ * ties), emit argmax(target_row_k); draft_logits, u_accept and u_sample are not read.
+ *
+ *   Sequence s has gamma_s = cu_draft[s+1] - cu_draft[s] >= 0 drafted tokens.
+ *   target_logits  [total_draft + num_seqs][vocab] fp32; the gamma_s + 1 target rows of s
+ *                  start at row cu_draft[s] + s
+ *   draft_logits   [total_draft][vocab] fp32; NULL allowed iff temperature == 0
+ *   draft_tokens   [total_draft] int32, each in [0, vocab) (else BP_ERR_DEVICE_FLAG)
+ *   cu_draft       [num_seqs+1] int32 device array, non-decreasing, cu_draft[0] = 0
+ *   u_accept       [total_draft] fp32 uniforms in [0,1); u_sample [num_seqs] in [0,1)
+ *   n_accepted     [num_seqs] int32 out: k
+ *   out_tokens     [total_draft + num_seqs] int32 out: slots cu_draft[s]+s .. +gamma_s hold
+ *                  x_0..x_{k-1}, the emitted token, then -1
+ *   accept_prob    [total_draft] fp32 out: a_i for every drafted position; may be NULL
+ * Row addresses must be 16-byte aligned for the vectorised path (vocab % 4 == 0 and
+ * 16-byte aligned bases); other vocabularies take a scalar path.
+ * ------------------------------------------------------------------------------- */
+BP_API size_t bp_spec_accept_workspace_size(int num_seqs, int total_draft, int vocab);
+BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
+                   const int32_t* cu_draft, int num_seqs, int total_draft, int vocab, float temperature,
+                   const float* u_accept, const float* u_sample, int32_t* n_accepted, int32_t* out_tokens,
+                   float* accept_prob, void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------
+ * Block-size policy head, run once per request after prefill.  Sections 2.3 and 2.4:
+ * an MLP maps the request's prefill representation to one logit per candidate block
+ * size and B_hat = argmax over the candidates, fixed for the whole request; Section 3.1
+ * fixes two layers (hidden width 2048 by default).  With ReLU as the activation:
+ *
+ *   h = max(0, W1 x + b1),  o = W2 h + b2,  block_size_out[n] = candidates[argmax o]
+ *
+ * (lowest index on ties).  Pooling: request n reads feature row row_index[n] (e.g. its
+ * last prefill token), or row n when row_index is NULL.  No preprocessing of x (Table 5).
+ *
+ *   feats       rows of d_in values of type wdtype, row_stride elements apart (>= d_in)
+ *   w1 [hidden][d_in], w2 [num_cand][hidden] of type wdtype; b1 [hidden], b2 [num_cand] fp32
+ *   candidates  [num_cand] int32 device array of block sizes
+ *   logits_out  [num_reqs][num_cand] fp32 out, may be NULL; block_size_out [num_reqs] int32 out
+ * Limits: d_in % 8 == 0 and 16-byte aligned rows for bf16 (d_in % 4 == 0 for fp32),
+ * num_cand <= 64.
+ * ------------------------------------------------------------------------------- */
+BP_API size_t bp_policy_select_workspace_size(int num_reqs, int hidden, int num_cand);
+BP_API int bp_policy_select(const void* feats, int64_t feat_row_stride, const int32_t* row_index, int num_reqs, int d_in,
+                     const void* w1, const float* b1, int hidden, const void* w2, const float* b2, int num_cand,
+                     const int32_t* candidates, int wdtype, float* logits_out, int32_t* block_size_out,
+                     void* workspace, size_t workspace_bytes, void* stream);
+
+/* Reads and clears the sticky device error word of `workspace` (synchronizes `stream`).
+ * Returns BP_OK, BP_ERR_TIMEOUT or BP_ERR_DEVICE_FLAG (or BP_ERR_CUDA if the read fails). */
+BP_API int bp_get_status(void* workspace, void* stream);
+
+/* Human-readable name of a bp_status value (static string, never NULL). */
+BP_API const char* bp_error_string(int status);
+
+/* BP_ABI_VERSION of the loaded library. */
+BP_API int bp_abi_version(void);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* BLOCKPILOT_H */

@@ -1,0 +1,198 @@
+"""ctypes binding of libblockpilot (argument marshalling only).
+
+Every function takes CUDA tensors, passes their device pointers and the current torch
+stream to the C ABI and returns the output tensors.  No step of the computation happens
+here; if the library is missing or the call fails the binding raises -- there is no
+fallback path.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+
+import torch
+
+from . import _build
+
+BP_OK = 0
+BP_ERR_INVALID_ARG = 1
+BP_ERR_UNSUPPORTED = 2
+BP_ERR_CUDA = 3
+BP_ERR_WORKSPACE = 4
+BP_ERR_TIMEOUT = 5
+BP_ERR_DEVICE_FLAG = 6
+
+MASK_CAUSAL = 0
+MASK_BIDIR = 1
+F32 = 0
+BF16 = 1
+
+_lib = None
+
+
+class BlockPilotError(RuntimeError):
+    def __init__(self, status: int, where: str):
+        self.status = status
+        msg = _lib.bp_error_string(status).decode() if _lib is not None else str(status)
+        super().__init__(f"{where}: {msg}")
+
+
+def library_path() -> str:
+    return _build.LIB
+
+
+def load():
+    """Load libblockpilot.so (built by ``__graft_entry__.build()`` / ``_build.build()``)."""
+    global _lib
+    if _lib is not None:
+        return _lib
+    if not os.path.exists(_build.LIB):
+        raise RuntimeError(f"libblockpilot.so is not built ({_build.LIB}); run __graft_entry__.build() first")
+    lib = ctypes.CDLL(_build.LIB)
+    vp, i32, i64, f32, sz = ctypes.c_void_p, ctypes.c_int, ctypes.c_int64, ctypes.c_float, ctypes.c_size_t
+    lib.bp_abi_version.argtypes = []
+    lib.bp_abi_version.restype = i32
+    lib.bp_error_string.argtypes = [i32]
+    lib.bp_error_string.restype = ctypes.c_char_p
+    lib.bp_block_attention_workspace_size.argtypes = [i32, i32, i32, i32, i32]
+    lib.bp_block_attention_workspace_size.restype = sz
+    lib.bp_block_attention.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, i32, i32, i32,
+                                       f32, vp, sz, vp]
+    lib.bp_block_attention.restype = i32
+    lib.bp_spec_accept_workspace_size.argtypes = [i32, i32, i32]
+    lib.bp_spec_accept_workspace_size.restype = sz
+    lib.bp_spec_accept.argtypes = [vp, vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bp_spec_accept.restype = i32
+    lib.bp_policy_select_workspace_size.argtypes = [i32, i32, i32]
+    lib.bp_policy_select_workspace_size.restype = sz
+    lib.bp_policy_select.argtypes = [vp, i64, vp, i32, i32, vp, vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, sz, vp]
+    lib.bp_policy_select.restype = i32
+    lib.bp_get_status.argtypes = [vp, vp]
+    lib.bp_get_status.restype = i32
+    _lib = lib
+    return lib
+
+
+def _ptr(t) -> ctypes.c_void_p | None:
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _stream(stream) -> ctypes.c_void_p:
+    if stream is None:
+        stream = torch.cuda.current_stream()
+    return ctypes.c_void_p(stream.cuda_stream)
+
+
+def _check(rc: int, where: str):
+    if rc != BP_OK:
+        raise BlockPilotError(rc, where)
+
+
+def _cuda(t, name):
+    if t is not None and (not t.is_cuda or not t.is_contiguous()):
+        raise ValueError(f"{name} must be a contiguous CUDA tensor")
+
+
+def workspace(nbytes: int, device) -> torch.Tensor:
+    """Zero-filled device workspace (the library itself never allocates)."""
+    return torch.zeros(max(int(nbytes), 256), dtype=torch.uint8, device=device)
+
+
+# --------------------------------------------------------------------------- attention
+def block_attention_workspace_size(num_seqs, max_q_len, num_q_heads, num_kv_heads, head_dim) -> int:
+    return int(load().bp_block_attention_workspace_size(num_seqs, max_q_len, num_q_heads, num_kv_heads, head_dim))
+
+
+def block_attention(q, k, v, cu_q, cu_kv, max_q_len: int, max_kv_len: int, mask: int = MASK_CAUSAL,
+                    softmax_scale: float = 0.0, out=None, lse=None, ws=None, stream=None):
+    """O = block attention of q over (k, v); see ``bp_block_attention`` in include/blockpilot.h.
+
+    q [total_q, Hq, D], k/v [total_kv, Hkv, D] (bf16 or fp32), cu_q/cu_kv int32 [S+1] on the device.
+    Returns (o, lse_or_None)."""
+    lib = load()
+    for t, n in ((q, "q"), (k, "k"), (v, "v"), (cu_q, "cu_q"), (cu_kv, "cu_kv"), (out, "out"), (lse, "lse")):
+        _cuda(t, n)
+    dtype = {torch.bfloat16: BF16, torch.float32: F32}.get(q.dtype)
+    if dtype is None or k.dtype != q.dtype or v.dtype != q.dtype:
+        raise ValueError("q, k, v must all be bf16 or all fp32")
+    total_q, hq, d = q.shape
+    total_kv, hkv, _ = k.shape
+    s = cu_q.numel() - 1
+    if out is None:
+        out = torch.empty_like(q)
+    if ws is None:
+        ws = workspace(lib.bp_block_attention_workspace_size(s, max_q_len, hq, hkv, d), q.device)
+    rc = lib.bp_block_attention(_ptr(q), _ptr(k), _ptr(v), _ptr(out), _ptr(lse), _ptr(cu_q), _ptr(cu_kv), s, total_q,
+                                total_kv, int(max_q_len), int(max_kv_len), hq, hkv, d, dtype, int(mask),
+                                float(softmax_scale), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "bp_block_attention")
+    return out, lse
+
+
+# --------------------------------------------------------------------------- acceptance
+def spec_accept_workspace_size(num_seqs, total_draft, vocab) -> int:
+    return int(load().bp_spec_accept_workspace_size(num_seqs, total_draft, vocab))
+
+
+def spec_accept(target_logits, draft_logits, draft_tokens, cu_draft, temperature: float, u_accept=None,
+                u_sample=None, n_accepted=None, out_tokens=None, accept_prob=None, want_accept_prob=True, ws=None,
+                stream=None):
+    """Lossless acceptance; see ``bp_spec_accept``.  Returns (n_accepted, out_tokens, accept_prob)."""
+    lib = load()
+    for t, n in ((target_logits, "target_logits"), (draft_logits, "draft_logits"), (draft_tokens, "draft_tokens"),
+                 (cu_draft, "cu_draft"), (u_accept, "u_accept"), (u_sample, "u_sample")):
+        _cuda(t, n)
+    s = cu_draft.numel() - 1
+    total_draft = draft_tokens.numel()
+    vocab = target_logits.shape[1]
+    dev = target_logits.device
+    if n_accepted is None:
+        n_accepted = torch.empty(s, dtype=torch.int32, device=dev)
+    if out_tokens is None:
+        out_tokens = torch.empty(total_draft + s, dtype=torch.int32, device=dev)
+    if accept_prob is None and want_accept_prob:
+        accept_prob = torch.empty(total_draft, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(lib.bp_spec_accept_workspace_size(s, total_draft, vocab), dev)
+    rc = lib.bp_spec_accept(_ptr(target_logits), _ptr(draft_logits), _ptr(draft_tokens), _ptr(cu_draft), s,
+                            total_draft, vocab, float(temperature), _ptr(u_accept), _ptr(u_sample), _ptr(n_accepted),
+                            _ptr(out_tokens), _ptr(accept_prob), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "bp_spec_accept")
+    return n_accepted, out_tokens, accept_prob
+
+
+# --------------------------------------------------------------------------- policy head
+def policy_select_workspace_size(num_reqs, hidden, num_cand) -> int:
+    return int(load().bp_policy_select_workspace_size(num_reqs, hidden, num_cand))
+
+
+def policy_select(feats, w1, b1, w2, b2, candidates, row_index=None, num_reqs=None, block_size=None, logits=None,
+                  want_logits=True, ws=None, stream=None):
+    """Block-size policy head; see ``bp_policy_select``.  Returns (block_size, logits)."""
+    lib = load()
+    for t, n in ((feats, "feats"), (w1, "w1"), (b1, "b1"), (w2, "w2"), (b2, "b2"), (candidates, "candidates"),
+                 (row_index, "row_index")):
+        _cuda(t, n)
+    wdtype = {torch.bfloat16: BF16, torch.float32: F32}.get(w1.dtype)
+    if wdtype is None or feats.dtype != w1.dtype or w2.dtype != w1.dtype:
+        raise ValueError("feats, w1, w2 must share one dtype (bf16 or fp32)")
+    hidden, d_in = w1.shape
+    c = w2.shape[0]
+    n = num_reqs if num_reqs is not None else (row_index.numel() if row_index is not None else feats.shape[0])
+    dev = feats.device
+    if block_size is None:
+        block_size = torch.empty(n, dtype=torch.int32, device=dev)
+    if logits is None and want_logits:
+        logits = torch.empty((n, c), dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(lib.bp_policy_select_workspace_size(n, hidden, c), dev)
+    rc = lib.bp_policy_select(_ptr(feats), feats.stride(0), _ptr(row_index), n, d_in, _ptr(w1), _ptr(b1), hidden,
+                              _ptr(w2), _ptr(b2), c, _ptr(candidates), wdtype, _ptr(logits), _ptr(block_size),
+                              _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "bp_policy_select")
+    return block_size, logits
+
+
+def get_status(ws, stream=None) -> int:
+    """Reads and clears the device error word of a workspace (synchronizes the stream)."""
+    return int(load().bp_get_status(_ptr(ws), _stream(stream)))

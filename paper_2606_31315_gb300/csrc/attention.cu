@@ -1,0 +1,611 @@
+// Block attention for the verify (causal-within-block) and drafter (bidirectional-
+// within-block) passes of block-diffusion speculative decoding (Section 2.1,
+// Figure 1 of the BlockPilot paper).
+//
+// bf16 tensor-core path (sm_103a):
+//   * One work unit = (sequence, KV head, 128-row query tile).  The B_s block
+//     queries of the g = Hq/Hkv query heads that share a KV head are packed as the
+//     rows of one M=128 tile (row r = i*g + j: block position i, head j of the
+//     group), so QK^T and PV are M=128 tcgen05 MMAs that read each K/V tile once.
+//   * A thread-block cluster of CS CTAs splits the unit's keys; each CTA streams its
+//     share of 128-key K/V tiles through a 3-stage TMA ring (SWIZZLE_128B), computes
+//     S = Q K^T into tensor memory, runs an online softmax (fp32, exp2 domain, lazy
+//     rescale of the TMEM accumulator when the row max grows by more than 2^8),
+//     writes P (bf16) back into tensor memory and accumulates O += P V with P as the
+//     TMEM A operand.  The CS partial results are merged through distributed shared
+//     memory -- no global scratch, one launch.
+//   * Units are issued longest-first so that ragged batches finish together.
+//   Warp roles: warp 0 = TMA producer + TMEM allocator, warp 1 = MMA issuer,
+//   warps 2..5 = softmax / epilogue (one query row per thread, TMEM lane = row).
+//
+// fp32 path: a plain SIMT kernel (one warp per output row, online softmax).
+#include <cooperative_groups.h>
+#include <cuda_bf16.h>
+
+#include "common.cuh"
+#include "ptx_sm103.cuh"
+
+namespace cg = cooperative_groups;
+
+namespace bp {
+namespace {
+
+constexpr int kD = 128;       // head_dim of the tensor-core path
+constexpr int kTileN = 128;   // keys per K/V tile
+constexpr int kM = 128;       // query rows per tile
+constexpr int kStages = 3;    // K/V ring depth
+constexpr int kHalf = kTileN * 64 * 2;          // one 64-column SW128 half of a 128-row tile: 16 KB
+constexpr int kQBytes = kM * kD * 2;            // 32 KB
+constexpr int kKVBytes = kTileN * kD * 2;       // 32 KB for K, 32 KB for V
+constexpr int kStageBytes = 2 * kKVBytes;       // 64 KB
+constexpr int kDynSmem = kQBytes + kStages * kStageBytes + 1024;
+constexpr int kThreads = 192;
+constexpr uint32_t kTmemCols = 512;
+constexpr uint32_t kColO = 256;
+constexpr int kMaxOrderedSeqs = 256;  // longest-first ordering for batches up to this size
+
+struct AttnParams {
+    const __nv_bfloat16* q;
+    __nv_bfloat16* o;
+    float* lse;
+    const int32_t* cu_q;
+    const int32_t* cu_kv;
+    int num_seqs, num_q_heads, num_kv_heads, group, m_tiles;
+    int causal;
+    float scale_log2;  // softmax scale * log2(e)
+    unsigned int* err;
+};
+
+__device__ __forceinline__ uint32_t col_s(int sb) { return sb ? 128u : 0u; }  // TMEM column of S buffer sb
+
+__device__ __forceinline__ float fast_exp2(float x) {
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+__device__ __forceinline__ uint32_t cluster_rank() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_ctarank;" : "=r"(r));
+    return r;
+}
+__device__ __forceinline__ uint32_t cluster_size() {
+    uint32_t r;
+    asm volatile("mov.u32 %0, %%cluster_nctarank;" : "=r"(r));
+    return r;
+}
+
+__global__ void __launch_bounds__(kThreads, 1)
+    attn_bf16_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
+                        const AttnParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sQ = smem;
+    uint8_t* sKV = smem + kQBytes;  // stage s: K at s*64KB, V at s*64KB + 32KB
+
+    __shared__ uint64_t bar_kv_full[kStages], bar_kv_empty[kStages];
+    __shared__ uint64_t bar_s_full[2], bar_p_full[2], bar_pv_done[2], bar_o_done;
+    __shared__ uint32_t tmem_base_sh;
+    __shared__ int unit_seq_sh;
+    __shared__ int32_t cu_kv_sh[kMaxOrderedSeqs + 1];
+
+    const int tid = threadIdx.x;
+    const int warp = tid >> 5, lane = tid & 31;
+    const uint32_t CS = cluster_size();
+    const uint32_t crank = cluster_rank();
+    const int unit_rank = blockIdx.x / CS;
+    const int G = p.group;
+    const int units_per_seq = p.num_kv_heads * p.m_tiles;
+    const int seq_rank = unit_rank / units_per_seq;
+    const int h = (unit_rank / p.m_tiles) % p.num_kv_heads;
+    const int mt = unit_rank % p.m_tiles;
+
+    // ---- which sequence: the seq_rank-th longest (ties by index) for small batches
+    if (p.num_seqs <= kMaxOrderedSeqs) {
+        for (int s = tid; s <= p.num_seqs; s += kThreads) cu_kv_sh[s] = p.cu_kv[s];
+        __syncthreads();
+        for (int s = tid; s < p.num_seqs; s += kThreads) {
+            const int len = cu_kv_sh[s + 1] - cu_kv_sh[s];
+            int rank = 0;
+            for (int t = 0; t < p.num_seqs; ++t) {
+                const int lt = cu_kv_sh[t + 1] - cu_kv_sh[t];
+                rank += (lt > len) || (lt == len && t < s);
+            }
+            if (rank == seq_rank) unit_seq_sh = s;
+        }
+        __syncthreads();
+    } else {
+        if (tid == 0) unit_seq_sh = seq_rank;
+        __syncthreads();
+    }
+    const int s = unit_seq_sh;
+    const int q0 = p.cu_q[s];
+    const int B = p.cu_q[s + 1] - q0;
+    const int kv0 = p.cu_kv[s];
+    const int n = p.cu_kv[s + 1] - kv0;
+    const int L = n - B;
+    const int rows = B * G;
+    const int row0 = mt * kM;
+    const int m_valid = min(kM, rows - row0);
+    if (m_valid <= 0) return;  // uniform across the cluster: every CTA decodes the same unit
+
+    const int tiles = (n + kTileN - 1) / kTileN;
+    const int t_begin = (int)((long long)crank * tiles / CS);
+    const int t_end = (int)((long long)(crank + 1) * tiles / CS);
+    const int nt = t_end - t_begin;
+
+    // ---- Q tile -> shared memory, SWIZZLE_128B K-major (two 64-column halves)
+    for (int idx = tid; idx < kM * 16; idx += kThreads) {
+        const int r = idx >> 4, ch = idx & 15;
+        uint4 val = make_uint4(0, 0, 0, 0);
+        if (r < m_valid) {
+            const int lr = row0 + r;
+            const int i = lr / G, j = lr % G;
+            val = *reinterpret_cast<const uint4*>(p.q + ((size_t)(q0 + i) * p.num_q_heads + h * G + j) * kD + ch * 8);
+        }
+        const int half = ch >> 3, c8 = ch & 7;
+        *reinterpret_cast<uint4*>(sQ + half * kHalf + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
+    }
+    fence_proxy_async_smem();
+    if (tid == 0) {
+        for (int i = 0; i < kStages; ++i) {
+            mbar_init(&bar_kv_full[i], 1);
+            mbar_init(&bar_kv_empty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
+            mbar_init(&bar_s_full[i], 1);
+            mbar_init(&bar_p_full[i], 128);
+            mbar_init(&bar_pv_done[i], 1);
+        }
+        mbar_init(&bar_o_done, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(&tmem_base_sh, kTmemCols);
+        tmem_relinquish();
+    }
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_base_sh;
+
+    if (warp == 0) {
+        // ================= TMA producer
+        if (lane == 0 && nt > 0) {
+            prefetch_tensormap(&kmap);
+            prefetch_tensormap(&vmap);
+            int issued = 0;
+            for (int j = 0; j < nt; ++j) {
+                const int st = j % kStages;
+                if (j >= kStages && !mbar_wait(&bar_kv_empty[st], ((j / kStages) - 1) & 1, kWaitBudget)) {
+                    raise_error(p.err, kErrTimeout);
+                    break;
+                }
+                uint8_t* sK = sKV + st * kStageBytes;
+                uint8_t* sV = sK + kKVBytes;
+                const int key = kv0 + (t_begin + j) * kTileN;
+                mbar_arrive_expect_tx(&bar_kv_full[st], kStageBytes);
+                tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, h, key);
+                tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, h, key);
+                tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, h, key);
+                tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, h, key);
+                ++issued;
+            }
+            // no copy may still be in flight when the CTA leaves
+            for (int j = max(0, issued - kStages); j < issued; ++j)
+                if (!mbar_wait(&bar_kv_full[j % kStages], (j / kStages) & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
+        }
+    } else if (warp == 1) {
+        // ================= MMA issuer
+        if (lane == 0 && nt > 0) {
+            const uint32_t id_s = idesc_bf16_f32(kM, kTileN, false, false);
+            const uint32_t id_o = idesc_bf16_f32(kM, kD, false, true);
+            const uint32_t q_addr = smem_addr(sQ);
+            bool ok = true;
+            auto issue_pv = [&](int j) {
+                const int sb = j & 1, st = j % kStages;
+                if (!mbar_wait(&bar_p_full[sb], (j >> 1) & 1, kWaitBudget)) return false;
+                tc_fence_after();
+                const uint32_t v_addr = smem_addr(sKV + st * kStageBytes + kKVBytes);
+                for (int kk = 0; kk < kTileN / 16; ++kk) {
+                    const uint64_t bdesc = smem_desc(v_addr + kk * 2048, kHalf, 1024, kSwizzle128B);
+                    umma_ts(tmem + kColO, tmem + col_s(sb) + kk * 8, bdesc, id_o, (j > 0 || kk > 0) ? 1u : 0u);
+                }
+                umma_commit(&bar_pv_done[sb]);
+                umma_commit(&bar_kv_empty[st]);
+                return true;
+            };
+            for (int j = 0; j < nt && ok; ++j) {
+                const int sb = j & 1, st = j % kStages;
+                if (!mbar_wait(&bar_kv_full[st], (j / kStages) & 1, kWaitBudget)) { ok = false; break; }
+                if (j >= 2 && !mbar_wait(&bar_pv_done[sb], ((j - 2) >> 1) & 1, kWaitBudget)) { ok = false; break; }
+                tc_fence_after();
+                const uint32_t k_addr = smem_addr(sKV + st * kStageBytes);
+                for (int kk = 0; kk < kD / 16; ++kk) {
+                    const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+                    const uint64_t adesc = smem_desc(q_addr + off, 16, 1024, kSwizzle128B);
+                    const uint64_t bdesc = smem_desc(k_addr + off, 16, 1024, kSwizzle128B);
+                    umma_ss(tmem + col_s(sb), adesc, bdesc, id_s, kk > 0 ? 1u : 0u);
+                }
+                umma_commit(&bar_s_full[sb]);
+                if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+            }
+            if (ok && !issue_pv(nt - 1)) ok = false;
+            if (!ok) raise_error(p.err, kErrTimeout);
+            umma_commit(&bar_o_done);
+            // no MMA may still be writing tensor memory when it is released
+            if (!mbar_wait(&bar_o_done, 0, kWaitBudget)) raise_error(p.err, kErrTimeout);
+        }
+    }
+
+    // ================= softmax / epilogue warps (2..5); row = TMEM lane
+    const int quad = warp & 3;
+    const int r = quad * 32 + lane;
+    const bool is_softmax = warp >= 2;
+    const bool row_active = is_softmax && r < m_valid;
+    const bool warp_active = is_softmax && (quad * 32 < m_valid);
+    const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
+    const int limit = row_active ? (p.causal ? L + (row0 + r) / G + 1 : n) : 0;
+    float m_run = -INFINITY, l_run = 0.f;
+    float o_acc[kD];
+    bool failed = false;
+
+    if (is_softmax) {
+        for (int j = 0; j < nt; ++j) {
+            const int sb = j & 1;
+            if (!__all_sync(0xffffffffu, mbar_wait(&bar_s_full[sb], (j >> 1) & 1, kWaitBudget))) {
+                failed = true;
+                break;
+            }
+            tc_fence_after();
+            if (warp_active) {
+                const int nvalid = limit - (t_begin + j) * kTileN;
+                float x[kTileN];
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t v[32];
+                    tmem_ld32(tmem + lane_base + col_s(sb) + c * 32, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        const int kidx = c * 32 + e;
+                        x[kidx] = (kidx < nvalid) ? __uint_as_float(v[e]) * p.scale_log2 : -INFINITY;
+                    }
+                }
+                float mt_ = -INFINITY;
+#pragma unroll
+                for (int e = 0; e < kTileN; ++e) mt_ = fmaxf(mt_, x[e]);
+                const float m_new = fmaxf(m_run, mt_);
+                const bool need = m_new > m_run + 8.f;
+                const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
+                // rescale the TMEM accumulator of rows whose max grew (warp-uniform TMEM access)
+                if (__any_sync(0xffffffffu, need && j > 0 && m_run != -INFINITY)) {
+                    if (!__all_sync(0xffffffffu,
+                                    mbar_wait(&bar_pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, kWaitBudget))) {
+                        failed = true;
+                    } else {
+                        tc_fence_after();
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            uint32_t v[32];
+                            tmem_ld32(tmem + lane_base + kColO + c * 32, v);
+                            tmem_ld_wait();
+                            uint32_t w0[16], w1[16];
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                w0[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+                                w1[e] = __float_as_uint(__uint_as_float(v[16 + e]) * alpha);
+                            }
+                            tmem_st16(tmem + lane_base + kColO + c * 32, w0);
+                            tmem_st16(tmem + lane_base + kColO + c * 32 + 16, w1);
+                        }
+                    }
+                }
+                if (need) {
+                    l_run *= alpha;
+                    m_run = m_new;
+                }
+                float lsum = 0.f;
+                const bool any = m_run != -INFINITY;
+#pragma unroll
+                for (int c = 0; c < 4; ++c) {
+                    uint32_t pk[16];
+#pragma unroll
+                    for (int e = 0; e < 16; ++e) {
+                        const float a = any ? fast_exp2(x[c * 32 + 2 * e] - m_run) : 0.f;
+                        const float b = any ? fast_exp2(x[c * 32 + 2 * e + 1] - m_run) : 0.f;
+                        lsum += a + b;
+                        pk[e] = pack_bf16x2(a, b);
+                    }
+                    tmem_st16(tmem + lane_base + col_s(sb) + c * 16, pk);
+                }
+                l_run += lsum;
+                tmem_st_wait();
+            }
+            tc_fence_before();
+            mbar_arrive(&bar_p_full[sb]);
+            if (failed) break;
+        }
+        // final accumulator
+        if (nt > 0 && !failed && !__all_sync(0xffffffffu, mbar_wait(&bar_o_done, 0, kWaitBudget))) failed = true;
+        failed = __any_sync(0xffffffffu, failed);
+        if (failed) raise_error(p.err, kErrTimeout);
+        tc_fence_after();
+        if (warp_active && nt > 0 && !failed) {
+#pragma unroll
+            for (int c = 0; c < 4; ++c) {
+                uint32_t v[32];
+                tmem_ld32(tmem + lane_base + kColO + c * 32, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 32; ++e) o_acc[c * 32 + e] = __uint_as_float(v[e]);
+            }
+        } else {
+#pragma unroll
+            for (int e = 0; e < kD; ++e) o_acc[e] = 0.f;
+            if (nt == 0 || failed) {
+                m_run = -INFINITY;
+                l_run = 0.f;
+            }
+        }
+    }
+
+    const float kLn2 = 0.6931471805599453f;
+    if (CS == 1) {
+        if (row_active) {
+            const int lr = row0 + r;
+            const int i = lr / G, jh = lr % G;
+            const size_t orow = (size_t)(q0 + i) * p.num_q_heads + h * G + jh;
+            const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+            __nv_bfloat16* dst = p.o + orow * kD;
+#pragma unroll
+            for (int c = 0; c < kD / 8; ++c) {
+                uint4 w;
+                w.x = pack_bf16x2(o_acc[c * 8 + 0] * inv, o_acc[c * 8 + 1] * inv);
+                w.y = pack_bf16x2(o_acc[c * 8 + 2] * inv, o_acc[c * 8 + 3] * inv);
+                w.z = pack_bf16x2(o_acc[c * 8 + 4] * inv, o_acc[c * 8 + 5] * inv);
+                w.w = pack_bf16x2(o_acc[c * 8 + 6] * inv, o_acc[c * 8 + 7] * inv);
+                *reinterpret_cast<uint4*>(dst + c * 8) = w;
+            }
+            if (p.lse) p.lse[orow] = (m_run + __log2f(l_run)) * kLn2;
+        }
+    } else {
+        // ---- cluster merge of the CS partial (m, l, O) triples through distributed shared memory
+        cg::cluster_group cluster = cg::this_cluster();
+        // all TMA loads of this CTA were consumed, so the K/V ring is free:
+        //   opart  [kM rows][kD] fp32 partial O (16-byte chunks swizzled by row)
+        //   row_ml [kM] (m, l) of each row's partial
+        float* opart = reinterpret_cast<float*>(sKV);
+        float2* row_ml = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float));
+        if (is_softmax) {
+            if (row_active) {
+#pragma unroll
+                for (int c = 0; c < kD / 4; ++c) {
+                    const int pc = c ^ (r & 31);
+                    *reinterpret_cast<float4*>(opart + r * kD + pc * 4) =
+                        make_float4(o_acc[c * 4], o_acc[c * 4 + 1], o_acc[c * 4 + 2], o_acc[c * 4 + 3]);
+                }
+            }
+            row_ml[r] = make_float2(m_run, l_run);
+        }
+        cluster.sync();
+        const int per = (m_valid + (int)CS - 1) / (int)CS;
+        const int rbeg = (int)crank * per;
+        const int rend = min(m_valid, rbeg + per);
+        for (int item = tid; item < (rend - rbeg) * (kD / 4); item += kThreads) {
+            const int rr = rbeg + item / (kD / 4);
+            const int c = item % (kD / 4);
+            float M = -INFINITY;
+            for (uint32_t pr = 0; pr < CS; ++pr) {
+                const float2 ml = *cluster.map_shared_rank(&row_ml[rr], pr);
+                M = fmaxf(M, ml.x);
+            }
+            float Lsum = 0.f;
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+            for (uint32_t pr = 0; pr < CS; ++pr) {
+                const float2 ml = *cluster.map_shared_rank(&row_ml[rr], pr);
+                if (ml.x == -INFINITY) continue;
+                const float w = fast_exp2(ml.x - M);
+                Lsum += w * ml.y;
+                const float4 v = *cluster.map_shared_rank(
+                    reinterpret_cast<float4*>(opart + rr * kD + ((c ^ (rr & 31)) * 4)), pr);
+                acc.x += w * v.x;
+                acc.y += w * v.y;
+                acc.z += w * v.z;
+                acc.w += w * v.w;
+            }
+            const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+            const int lr = row0 + rr;
+            const int i = lr / G, jh = lr % G;
+            const size_t orow = (size_t)(q0 + i) * p.num_q_heads + h * G + jh;
+            uint2 w2;
+            w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+            w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+            *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
+            if (c == 0 && p.lse) p.lse[orow] = (M + __log2f(Lsum)) * kLn2;
+        }
+        cluster.sync();
+    }
+
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, kTmemCols);
+}
+
+// --------------------------------------------------------------------------- fp32 SIMT path
+// One warp per (query row, query head): online softmax over the row's visible keys in
+// chunks of 32 (lane = key), lane d-slices of the output.
+constexpr int kF32MaxD = 128;
+
+__global__ void __launch_bounds__(128) attn_f32_simt_kernel(const float* __restrict__ q, const float* __restrict__ k,
+                                                            const float* __restrict__ v, float* __restrict__ o,
+                                                            float* __restrict__ lse, const int32_t* __restrict__ cu_q,
+                                                            const int32_t* __restrict__ cu_kv, int num_seqs,
+                                                            int total_q, int hq, int hkv, int D, int causal,
+                                                            float scale) {
+    __shared__ float qs[4][kF32MaxD];
+    const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const long long row = (long long)blockIdx.x * 4 + wib;
+    if (row >= (long long)total_q * hq) return;
+    const int t = (int)(row / hq), h = (int)(row % hq);
+    const int g = hq / hkv, kvh = h / g;
+    int lo = 0, hi = num_seqs;  // sequence containing query t: cu_q[s] <= t < cu_q[s+1]
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (cu_q[mid] <= t) lo = mid; else hi = mid;
+    }
+    const int s = lo;
+    const int B = cu_q[s + 1] - cu_q[s];
+    const int i = t - cu_q[s];
+    const int kv0 = cu_kv[s];
+    const int n = cu_kv[s + 1] - kv0;
+    const int L = n - B;
+    const int nk = causal ? L + i + 1 : n;
+    for (int d = lane; d < D; d += 32) qs[wib][d] = q[((size_t)t * hq + h) * D + d];
+    __syncwarp();
+    float m = -INFINITY, l = 0.f;
+    float acc[kF32MaxD / 32];
+#pragma unroll
+    for (int e = 0; e < kF32MaxD / 32; ++e) acc[e] = 0.f;
+    for (int j0 = 0; j0 < nk; j0 += 32) {
+        const int j = j0 + lane;
+        float sc = -INFINITY;
+        if (j < nk) {
+            const float* kr = k + ((size_t)(kv0 + j) * hkv + kvh) * D;
+            float dot = 0.f;
+            for (int d = 0; d < D; ++d) dot = fmaf(qs[wib][d], kr[d], dot);
+            sc = dot * scale;
+        }
+        float cm = sc;
+        for (int off = 16; off; off >>= 1) cm = fmaxf(cm, __shfl_xor_sync(0xffffffffu, cm, off));
+        const float m_new = fmaxf(m, cm);
+        const float alpha = (m == -INFINITY) ? 0.f : expf(m - m_new);
+        const float pj = (j < nk) ? expf(sc - m_new) : 0.f;
+        float ps = pj;
+        for (int off = 16; off; off >>= 1) ps += __shfl_xor_sync(0xffffffffu, ps, off);
+        l = l * alpha + ps;
+#pragma unroll
+        for (int e = 0; e < kF32MaxD / 32; ++e) acc[e] *= alpha;
+        const int cnt = min(32, nk - j0);
+        for (int jj = 0; jj < cnt; ++jj) {
+            const float pjj = __shfl_sync(0xffffffffu, pj, jj);
+            const float* vr = v + ((size_t)(kv0 + j0 + jj) * hkv + kvh) * D;
+#pragma unroll
+            for (int e = 0; e < kF32MaxD / 32; ++e) {
+                const int d = lane + e * 32;
+                if (d < D) acc[e] = fmaf(pjj, vr[d], acc[e]);
+            }
+        }
+        m = m_new;
+    }
+#pragma unroll
+    for (int e = 0; e < kF32MaxD / 32; ++e) {
+        const int d = lane + e * 32;
+        if (d < D) o[((size_t)t * hq + h) * D + d] = acc[e] / l;
+    }
+    if (lse && lane == 0) lse[(size_t)t * hq + h] = m + logf(l);
+}
+
+}  // namespace
+
+int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
+    if (a.head_dim != kD) return BP_ERR_UNSUPPORTED;
+    const int G = a.num_q_heads / a.num_kv_heads;
+    const int m_tiles = (a.max_q_len * G + kM - 1) / kM;
+    const long long units = (long long)a.num_seqs * a.num_kv_heads * m_tiles;
+    if (units == 0 || a.total_q == 0) return BP_OK;
+
+    CUtensorMap kmap, vmap;
+    const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)a.num_kv_heads, (cuuint64_t)a.total_kv};
+    const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.num_kv_heads * kD * 2};
+    const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileN};
+    int rc = encode_tensor_map(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.k), dims, strides,
+                               box, CU_TENSOR_MAP_SWIZZLE_128B);
+    if (rc != BP_OK) return rc;
+    rc = encode_tensor_map(&vmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.v), dims, strides, box,
+                           CU_TENSOR_MAP_SWIZZLE_128B);
+    if (rc != BP_OK) return rc;
+
+    AttnParams p;
+    p.q = static_cast<const __nv_bfloat16*>(a.q);
+    p.o = static_cast<__nv_bfloat16*>(a.o);
+    p.lse = a.lse;
+    p.cu_q = a.cu_q;
+    p.cu_kv = a.cu_kv;
+    p.num_seqs = a.num_seqs;
+    p.num_q_heads = a.num_q_heads;
+    p.num_kv_heads = a.num_kv_heads;
+    p.group = G;
+    p.m_tiles = m_tiles;
+    p.causal = a.mask == BP_MASK_CAUSAL_BLOCK;
+    p.scale_log2 = a.scale * 1.4426950408889634f;
+    p.err = a.err_word;
+
+    // once per device: opt in to the shared-memory size and non-portable clusters, and find the
+    // largest cluster of these CTAs the GPU can co-schedule (queried outside any graph capture)
+    static int configured_device = -1;
+    static int max_cluster = 1;
+    if (configured_device != dev.device) {
+        if (cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                cudaSuccess)
+            return BP_ERR_CUDA;
+        max_cluster = 1;
+        for (int cs = 16; cs >= 2; cs /= 2) {
+            cudaLaunchConfig_t probe = {};
+            cudaLaunchAttribute pa[1];
+            probe.gridDim = dim3(cs, 1, 1);
+            probe.blockDim = dim3(kThreads, 1, 1);
+            probe.dynamicSmemBytes = kDynSmem;
+            pa[0].id = cudaLaunchAttributeClusterDimension;
+            pa[0].val.clusterDim.x = cs;
+            pa[0].val.clusterDim.y = 1;
+            pa[0].val.clusterDim.z = 1;
+            probe.attrs = pa;
+            probe.numAttrs = 1;
+            int n_clusters = 0;
+            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel, &probe) == cudaSuccess &&
+                n_clusters > 0) {
+                max_cluster = cs;
+                break;
+            }
+            cudaGetLastError();
+        }
+        configured_device = dev.device;
+    }
+    // cluster size: split each unit's keys so that about one wave of CTAs covers the GPU
+    const int max_tiles = (a.max_kv_len + kTileN - 1) / kTileN;
+    int cs = 1;
+    while (cs * 2 <= max_cluster && units * cs * 2 <= dev.sm_count && cs * 2 <= max_tiles) cs *= 2;
+
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.gridDim = dim3((unsigned)(units * cs), 1, 1);
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kDynSmem;
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = cs;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel, kmap, vmap, p) != cudaSuccess) return BP_ERR_CUDA;
+    return BP_OK;
+}
+
+int launch_attention_f32(const AttentionArgs& a, cudaStream_t stream) {
+    if (a.head_dim > kF32MaxD) return BP_ERR_UNSUPPORTED;
+    const long long rows = (long long)a.total_q * a.num_q_heads;
+    if (rows == 0) return BP_OK;
+    const unsigned blocks = (unsigned)((rows + 3) / 4);
+    attn_f32_simt_kernel<<<blocks, 128, 0, stream>>>(
+        static_cast<const float*>(a.q), static_cast<const float*>(a.k), static_cast<const float*>(a.v),
+        static_cast<float*>(a.o), a.lse, a.cu_q, a.cu_kv, a.num_seqs, a.total_q, a.num_q_heads, a.num_kv_heads,
+        a.head_dim, a.mask == BP_MASK_CAUSAL_BLOCK, a.scale);
+    return cudaGetLastError() == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+}
+
+}  // namespace bp

@@ -1,0 +1,102 @@
+// Internal declarations shared by the translation units of libblockpilot.
+#pragma once
+
+#include <cuda.h>
+#include <cuda_runtime.h>
+#include <stddef.h>
+#include <stdint.h>
+
+#include "../../include/blockpilot.h"
+
+namespace bp {
+
+// Workspace header: the first 256 bytes of every workspace.
+//   word 0: sticky error bits (kErrTimeout | kErrDeviceArg), cleared by bp_get_status
+struct WorkspaceHeader {
+    unsigned int error_bits;
+    unsigned int pad[63];
+};
+static_assert(sizeof(WorkspaceHeader) == 256, "workspace header is 256 bytes");
+
+enum : unsigned int { kErrTimeout = 1u, kErrDeviceArg = 2u };
+
+// Cycle budget of every bounded device-side wait (about one second at 2 GHz).
+constexpr long long kWaitBudget = 2000000000LL;
+
+__device__ __forceinline__ void raise_error(unsigned int* err_word, unsigned int bits) {
+    if (err_word) atomicOr(err_word, bits);
+}
+
+inline size_t align_up(size_t x, size_t a) { return (x + a - 1) / a * a; }
+
+// Properties of the current device, cached once per device.
+struct DeviceInfo {
+    int device = -1;
+    int sm_count = 0;
+    int cc_major = 0, cc_minor = 0;
+    int max_smem_optin = 0;
+};
+int device_info(DeviceInfo* out);  // BP_OK or BP_ERR_CUDA
+
+// Encodes a tiled TMA descriptor (driver entry point resolved once).
+int encode_tensor_map(CUtensorMap* map, CUtensorMapDataType dt, cuuint32_t rank, void* base, const cuuint64_t* dims,
+                      const cuuint64_t* strides_bytes, const cuuint32_t* box, CUtensorMapSwizzle swizzle);
+
+// Launchers (host side).  They assume the arguments were validated by the API layer.
+struct AttentionArgs {
+    const void* q;
+    const void* k;
+    const void* v;
+    void* o;
+    float* lse;
+    const int32_t* cu_q;
+    const int32_t* cu_kv;
+    int num_seqs, total_q, total_kv, max_q_len, max_kv_len;
+    int num_q_heads, num_kv_heads, head_dim;
+    int mask;
+    float scale;
+    unsigned int* err_word;
+};
+int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+int launch_attention_f32(const AttentionArgs& a, cudaStream_t stream);
+
+struct AcceptArgs {
+    const float* target;
+    const float* draft;
+    const int32_t* tokens;
+    const int32_t* cu_draft;
+    int num_seqs, total_draft, vocab;
+    float temperature;
+    const float* u_accept;
+    const float* u_sample;
+    int32_t* n_accepted;
+    int32_t* out_tokens;
+    float* accept_prob;
+    void* scratch;  // workspace past the header
+    unsigned int* err_word;
+};
+size_t accept_scratch_bytes(int num_seqs, int total_draft, int vocab);
+int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+
+struct PolicyArgs {
+    const void* feats;
+    int64_t row_stride;
+    const int32_t* row_index;
+    int num_reqs, d_in;
+    const void* w1;
+    const float* b1;
+    int hidden;
+    const void* w2;
+    const float* b2;
+    int num_cand;
+    const int32_t* candidates;
+    int wdtype;
+    float* logits_out;
+    int32_t* block_size_out;
+    void* scratch;
+    unsigned int* err_word;
+};
+size_t policy_scratch_bytes(int num_reqs, int hidden, int num_cand);
+int launch_policy(const PolicyArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+
+}  // namespace bp

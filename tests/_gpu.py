@@ -1,0 +1,143 @@
+"""Helpers for the GPU parity tests: move seeded workloads to the device, run the CUDA path
+through the C ABI, run the oracle on the same inputs (whole or sampled) and compare."""
+from __future__ import annotations
+
+import numpy as np
+import torch
+
+import oracle
+import paper_2606_31315_gb300 as bp
+from paper_2606_31315_gb300 import workloads as wl
+
+ATTN_TOL = 2e-2      # max |O - O_ref| / max |O_ref| per (sequence, query head) slice
+LSE_TOL = 2e-3       # absolute, natural-log units
+PROB_TOL = 1e-5      # accept_prob absolute
+FLAG = 1e-5          # near-tie flag for ratio test and inverse-CDF draws
+
+
+def dev():
+    return torch.device("cuda:0")
+
+
+def to_dev(x: np.ndarray, dtype: str | None = None) -> torch.Tensor:
+    if dtype == "bf16":
+        return torch.from_numpy(np.ascontiguousarray(x).view(np.int16)).to(dev()).view(torch.bfloat16)
+    return torch.from_numpy(np.ascontiguousarray(x)).to(dev())
+
+
+def run_attention(a: dict, mask: int):
+    """CUDA path on the whole workload; returns (o fp32 numpy, lse numpy)."""
+    q, k, v = to_dev(a["q"], a["dtype"]), to_dev(a["k"], a["dtype"]), to_dev(a["v"], a["dtype"])
+    cu_q, cu_kv = to_dev(a["cu_q"]), to_dev(a["cu_kv"])
+    lse = torch.empty(q.shape[0], q.shape[1], dtype=torch.float32, device=dev())
+    ws = bp.workspace(bp.block_attention_workspace_size(len(a["cu_q"]) - 1, a["max_q_len"], q.shape[1], k.shape[1],
+                                                        q.shape[2]), dev())
+    o, _ = bp.block_attention(q, k, v, cu_q, cu_kv, a["max_q_len"], a["max_kv_len"], mask=mask, lse=lse, ws=ws)
+    assert bp.get_status(ws) == 0
+    return o.float().cpu().numpy(), lse.cpu().numpy()
+
+
+def oracle_attention_slice(a: dict, s: int, kv_head: int | None, mask: int):
+    """Oracle on sequence s (all heads, or the query heads of one KV head); returns the
+    (o, lse) rows of that sequence and the q-head indices covered."""
+    cq, ck = a["cu_q"], a["cu_kv"]
+    hq, hkv = a["num_q_heads"], a["num_kv_heads"]
+    g = hq // hkv
+    heads = np.arange(hq) if kv_head is None else np.arange(kv_head * g, (kv_head + 1) * g)
+    kvh = np.arange(hkv) if kv_head is None else np.array([kv_head])
+    q = wl.as_f64(a["q"][cq[s]:cq[s + 1]][:, heads], a["dtype"])
+    k = wl.as_f64(a["k"][ck[s]:ck[s + 1]][:, kvh], a["dtype"])
+    v = wl.as_f64(a["v"][ck[s]:ck[s + 1]][:, kvh], a["dtype"])
+    o, lse = oracle.block_attention(q, k, v, [0, q.shape[0]], [0, k.shape[0]], len(kvh), mask)
+    return o, lse, heads
+
+
+def attention_errors(o_gpu, lse_gpu, a: dict, mask: int, seqs, kv_head: int | None = None):
+    """Worst per-(sequence, head) relative error and worst lse error over the sampled sequences."""
+    worst, worst_lse = 0.0, 0.0
+    for s in seqs:
+        cq = a["cu_q"]
+        if cq[s + 1] == cq[s]:
+            continue
+        o_ref, lse_ref, heads = oracle_attention_slice(a, s, kv_head, mask)
+        got = o_gpu[cq[s]:cq[s + 1]][:, heads]
+        for hi in range(len(heads)):
+            denom = np.abs(o_ref[:, hi]).max()
+            worst = max(worst, np.abs(got[:, hi] - o_ref[:, hi]).max() / max(denom, 1e-30))
+        worst_lse = max(worst_lse, np.abs(lse_gpu[cq[s]:cq[s + 1]][:, heads] - lse_ref).max())
+    return worst, worst_lse
+
+
+def run_accept(inp: dict, temperature: float, ws=None):
+    g = {key: to_dev(inp[key]) for key in ("target_logits", "draft_tokens", "cu_draft", "u_accept", "u_sample")}
+    draft = to_dev(inp["draft_logits"]) if temperature > 0 else None
+    s = len(inp["cu_draft"]) - 1
+    if ws is None:
+        ws = bp.workspace(bp.spec_accept_workspace_size(s, int(inp["cu_draft"][-1]), inp["target_logits"].shape[1]),
+                          dev())
+    n_acc, out, ap = bp.spec_accept(g["target_logits"], draft, g["draft_tokens"], g["cu_draft"], temperature,
+                                    g["u_accept"], g["u_sample"], ws=ws)
+    status = bp.get_status(ws)
+    return n_acc.cpu().numpy(), out.cpu().numpy(), ap.cpu().numpy(), status
+
+
+def run_oracle_accept(inp: dict, temperature: float):
+    return oracle.spec_accept(inp["target_logits"], inp["draft_logits"] if temperature > 0 else None,
+                              inp["draft_tokens"], inp["cu_draft"], temperature, inp["u_accept"], inp["u_sample"])
+
+
+def _near_tie_tokens(inp: dict, s: int, k: int, temperature: float) -> np.ndarray:
+    """Tokens whose fp64 inverse-CDF interval lies within FLAG of the draw's threshold (sequence s,
+    emitting at slot k).  Used only for sequences the oracle flags as near-ties."""
+    from scipy import special
+
+    cu = inp["cu_draft"]
+    gamma = cu[s + 1] - cu[s]
+    p = special.softmax(inp["target_logits"][cu[s] + s + k].astype(np.float64) / temperature)
+    w = p
+    if k < gamma:
+        q = special.softmax(inp["draft_logits"][cu[s] + k].astype(np.float64) / temperature)
+        r = np.maximum(p - q, 0.0)
+        if r.sum() > 0:
+            w = r
+    c = np.cumsum(w)
+    thr = float(inp["u_sample"][s]) * c[-1]
+    prev = np.concatenate([[0.0], c[:-1]])
+    return np.nonzero((w > 0) & (prev - FLAG <= thr) & (thr < c + FLAG))[0]
+
+
+def compare_accept(inp: dict, temperature: float, gpu=None, ref=None):
+    """Asserts parity.  Unflagged sequences: n_accepted and out_tokens bit-exact.  Flagged sequences
+    (near-ties): the GPU's prefix must follow from its own accept_prob (which is within 1e-5 of
+    the oracle's), the positions where it departs from the oracle must be near-ties, and its
+    emitted token must lie in the fp64 near-tie set.  Returns (flagged, sequences)."""
+    n_acc, out, ap, status = gpu if gpu is not None else run_accept(inp, temperature)
+    ref = ref if ref is not None else run_oracle_accept(inp, temperature)
+    assert status == 0, f"device error status {status}"
+    cu = inp["cu_draft"]
+    s = len(cu) - 1
+    assert np.abs(ap - ref["accept_prob"]).max(initial=0.0) <= PROB_TOL, np.abs(ap - ref["accept_prob"]).max()
+    flagged = (ref["ratio_margin"] < FLAG) | (ref["cdf_margin"] < FLAG)
+    if temperature == 0:
+        assert not flagged.any()
+    for i in range(s):
+        lo, hi = cu[i] + i, cu[i + 1] + i + 1
+        gamma = cu[i + 1] - cu[i]
+        k = int(n_acc[i])
+        if temperature > 0:
+            # the GPU's prefix is the ratio test applied to its own a_i
+            ua = inp["u_accept"][cu[i]:cu[i + 1]]
+            rej = np.nonzero(~(ua < ap[cu[i]:cu[i + 1]]))[0]
+            assert k == (rej[0] if len(rej) else gamma), (i, k, rej)
+        if not flagged[i]:
+            assert k == ref["n_accepted"][i], (i, k, ref["n_accepted"][i])
+            np.testing.assert_array_equal(out[lo:hi], ref["out_tokens"][lo:hi], err_msg=f"sequence {i}")
+            continue
+        kr = int(ref["n_accepted"][i])
+        if k != kr:  # a departure of the prefix is allowed only at a ratio-test near-tie
+            j = min(k, kr)
+            assert abs(float(inp["u_accept"][cu[i] + j]) - ref["accept_prob"][cu[i] + j]) < FLAG, (i, k, kr)
+        np.testing.assert_array_equal(out[lo:lo + k], inp["draft_tokens"][cu[i]:cu[i] + k])
+        assert np.all(out[lo + k + 1:hi] == -1)
+        assert out[lo + k] in _near_tie_tokens(inp, i, k, temperature), (i, k, out[lo + k])
+    return int(flagged.sum()), s

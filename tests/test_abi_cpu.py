@@ -1,0 +1,122 @@
+"""Host-side checks of the C-ABI library (no GPU needed): it builds for sm_103a, loads,
+exports exactly the symbols include/blockpilot.h declares, validates arguments on the host
+before touching CUDA, and has no CPU fallback.  Also checks that the product package never
+reaches the oracle."""
+import ast
+import ctypes
+import os
+import re
+
+import pytest
+
+import paper_2606_31315_gb300 as bp
+from paper_2606_31315_gb300 import _build
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+HEADER = os.path.join(ROOT, "include", "blockpilot.h")
+
+
+@pytest.fixture(scope="module")
+def lib():
+    _build.build()
+    return bp.load()
+
+
+def _declared():
+    text = open(HEADER).read()
+    return sorted(set(re.findall(r"BP_API\s+[\w\s\*]*?\b(bp_\w+)\s*\(", text)))
+
+
+def _exported():
+    import subprocess
+
+    out = subprocess.run(["nm", "-D", "--defined-only", _build.LIB], capture_output=True, text=True, check=True).stdout
+    return sorted({line.split()[-1] for line in out.splitlines() if " T " in line and line.split()[-1].startswith("bp_")})
+
+
+def test_exports_match_header(lib):
+    declared = _declared()
+    assert len(declared) >= 9
+    assert _exported() == declared
+    for name in declared:
+        assert hasattr(lib, name)
+
+
+def test_version_and_error_strings(lib):
+    assert lib.bp_abi_version() == 1
+    for code in range(7):
+        assert lib.bp_error_string(code).startswith(b"BP_")
+    assert lib.bp_error_string(99) == b"unknown bp_status"
+
+
+def test_workspace_sizes(lib):
+    assert bp.block_attention_workspace_size(1, 16, 32, 8, 128) >= 256
+    w = bp.spec_accept_workspace_size(1, 15, 151936)
+    assert w > 256 and w % 256 == 0
+    assert bp.spec_accept_workspace_size(32, 500, 151936) > w
+    assert bp.policy_select_workspace_size(32, 2048, 9) >= 256 + 32 * 2048 * 4
+    assert lib.bp_spec_accept_workspace_size(-1, 0, 10) == 0
+
+
+def test_host_validation_needs_no_gpu(lib):
+    vp = ctypes.c_void_p
+    fake = vp(0x10000)
+    ws = vp(0x20000)
+    # NULL q
+    rc = lib.bp_block_attention(None, fake, fake, fake, None, fake, fake, 1, 16, 2064, 16, 2064, 32, 8, 128, 1, 0,
+                                0.0, ws, 4096, None)
+    assert rc == 1
+    # head ratio
+    rc = lib.bp_block_attention(fake, fake, fake, fake, None, fake, fake, 1, 16, 2064, 16, 2064, 30, 8, 128, 1, 0,
+                                0.0, ws, 4096, None)
+    assert rc == 1
+    # bf16 head_dim 64 is not implemented
+    rc = lib.bp_block_attention(fake, fake, fake, fake, None, fake, fake, 1, 16, 2064, 16, 2064, 32, 8, 64, 1, 0,
+                                0.0, ws, 4096, None)
+    assert rc == 2
+    # workspace too small / misaligned
+    rc = lib.bp_block_attention(fake, fake, fake, fake, None, fake, fake, 1, 16, 2064, 16, 2064, 32, 8, 128, 1, 0,
+                                0.0, ws, 16, None)
+    assert rc == 4
+    rc = lib.bp_block_attention(fake, fake, fake, fake, None, fake, fake, 1, 16, 2064, 16, 2064, 32, 8, 128, 1, 0,
+                                0.0, vp(0x20010), 4096, None)
+    assert rc == 4
+    # acceptance: T > 0 without draft logits; negative temperature
+    rc = lib.bp_spec_accept(fake, None, fake, fake, 1, 15, 1000, ctypes.c_float(1.0), fake, fake, fake, fake, None,
+                            ws, 1 << 20, None)
+    assert rc == 1
+    rc = lib.bp_spec_accept(fake, fake, fake, fake, 1, 15, 1000, ctypes.c_float(-1.0), fake, fake, fake, fake, None,
+                            ws, 1 << 20, None)
+    assert rc == 1
+    # policy: too many candidates
+    rc = lib.bp_policy_select(fake, 64, None, 1, 64, fake, fake, 32, fake, fake, 65, fake, 1, None, fake, ws,
+                              1 << 20, None)
+    assert rc == 2
+
+
+def test_no_cpu_fallback_without_gpu(lib):
+    import torch
+
+    if torch.cuda.is_available():
+        pytest.skip("a GPU is present; this checks the GPU-less failure mode")
+    vp = ctypes.c_void_p
+    fake = vp(0x10000)
+    rc = lib.bp_block_attention(fake, fake, fake, fake, None, fake, fake, 1, 16, 2064, 16, 2064, 32, 8, 128, 1, 0,
+                                0.0, vp(0x20000), 4096, None)
+    assert rc == 3  # BP_ERR_CUDA: there is nothing to fall back to
+
+
+def test_product_package_never_imports_the_oracle():
+    pkg = os.path.join(ROOT, "paper_2606_31315_gb300")
+    for dirpath, _, files in os.walk(pkg):
+        for f in files:
+            path = os.path.join(dirpath, f)
+            if f.endswith(".py"):
+                tree = ast.parse(open(path).read())
+                for node in ast.walk(tree):
+                    if isinstance(node, ast.Import):
+                        assert all(not a.name.startswith("oracle") for a in node.names), path
+                    if isinstance(node, ast.ImportFrom):
+                        assert not (node.module or "").startswith("oracle"), path
+            if f.endswith((".cu", ".cuh", ".h")):
+                assert "bpo_" not in open(path).read(), path

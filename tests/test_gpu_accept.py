@@ -1,0 +1,139 @@
+"""GPU parity of bp_spec_accept against the fp64 oracle.
+
+Bars: accept_prob within 1e-5 absolute at every drafted position; n_accepted and the emitted
+tokens bit-exact for every sequence not flagged as a near-tie (|u_i - a_i| < 1e-5 at a tested
+position, or an inverse-CDF threshold within 1e-5 of a cumulative boundary); greedy (T = 0)
+bit-exact with no flags.  Full-size workloads run exactly as the benchmark launches them.
+"""
+import numpy as np
+import pytest
+import torch
+from scipy import stats
+
+import paper_2606_31315_gb300 as bp
+from paper_2606_31315_gb300 import workloads as wl
+
+from _gpu import compare_accept, run_accept, run_oracle_accept, to_dev
+
+pytestmark = pytest.mark.gpu
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    bp.build()
+    bp.load()
+
+
+def test_tiny():
+    w = wl.get("tiny")
+    compare_accept(wl.accept_inputs(w, 1.0), 1.0)
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_qwen3_4b_full(temp):
+    w = wl.get("qwen3_4b")
+    compare_accept(wl.accept_inputs(w, temp), temp)
+
+
+def test_ragged_batch_full():
+    w = wl.get("ragged")
+    flagged, s = compare_accept(wl.accept_inputs(w, 1.0), 1.0)
+    # about a quarter of the draws over a 151936-token vocabulary land within 1e-5 of a CDF
+    # boundary (most tokens carry less mass than that); those are checked for validity instead
+    assert flagged < s // 2
+
+
+@pytest.mark.parametrize("temp", [0.0, 1.0])
+def test_long_context_full(temp):
+    w = wl.get("long_context")
+    compare_accept(wl.accept_inputs(w, temp), temp)
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_planted_long_prefixes(temp):
+    """Draft rows copied from target rows with probability 0.9: long accepted prefixes and bonus draws."""
+    w = wl.custom(seed=44, ctx=(0,) * 12, block=(16, 16, 8, 24, 1, 16, 16, 12, 16, 20, 16, 2), vocab=151936)
+    inp = wl.accept_inputs(w, temp, planted_match=0.9)
+    compare_accept(inp, temp)
+    n_acc, _, _, _ = run_accept(inp, temp)
+    assert n_acc.max() >= 10
+
+
+@pytest.mark.parametrize("vocab", [5, 1001, 4099, 32000])
+def test_vocab_sizes_and_scalar_path(vocab):
+    w = wl.custom(seed=vocab, ctx=(0,) * 6, block=(16, 1, 3, 9, 24, 16), vocab=vocab)
+    for temp in (1.0, 0.0):
+        compare_accept(wl.accept_inputs(w, temp), temp)
+
+
+@pytest.mark.parametrize("temp", [0.05, 0.7, 3.0])
+def test_temperatures(temp):
+    w = wl.custom(seed=int(temp * 100), ctx=(0,) * 10, block=(16,) * 10, vocab=20000)
+    compare_accept(wl.accept_inputs(w, temp), temp)
+
+
+def test_workspace_reuse_gives_identical_results():
+    w = wl.custom(seed=9, ctx=(0,) * 5, block=(16, 4, 1, 16, 8), vocab=50000)
+    inp = wl.accept_inputs(w, 1.0)
+    ws = bp.workspace(bp.spec_accept_workspace_size(5, int(inp["cu_draft"][-1]), 50000), torch.device("cuda"))
+    r1 = run_accept(inp, 1.0, ws=ws)
+    r2 = run_accept(inp, 1.0, ws=ws)
+    for x, y in zip(r1[:3], r2[:3]):
+        np.testing.assert_array_equal(x, y)
+    compare_accept(inp, 1.0, gpu=r2)
+
+
+def test_lossless_chi_square_on_gpu():
+    """V = 16, gamma = 3, drafts sampled from q: the first emitted token follows p_0 (chi-square at
+    alpha = 1e-3 over 2e5 seeded trials), and the GPU agrees with the oracle trial by trial."""
+    V, gamma, n = 16, 3, 200_000
+    rng = np.random.default_rng(77)
+    p_rows = rng.dirichlet(np.full(V, 2.0), size=gamma + 1)
+    q_rows = rng.dirichlet(np.full(V, 2.0), size=gamma)
+    tl, dl = np.log(p_rows).astype(np.float32), np.log(q_rows).astype(np.float32)
+    cdf = np.cumsum(q_rows, axis=1)
+    uu = rng.random((n, gamma))
+    toks = np.stack([np.minimum(np.searchsorted(cdf[i], uu[:, i], side="right"), V - 1) for i in range(gamma)],
+                    axis=1).astype(np.int32)
+    inp = dict(target_logits=np.tile(tl, (n, 1)), draft_logits=np.tile(dl, (n, 1)), draft_tokens=toks.reshape(-1),
+               cu_draft=(np.arange(n + 1) * gamma).astype(np.int32),
+               u_accept=rng.random(n * gamma, dtype=np.float32), u_sample=rng.random(n, dtype=np.float32))
+    gpu = run_accept(inp, 1.0)
+    n_acc, out = gpu[0], gpu[1].reshape(n, gamma + 1)
+    counts = np.bincount(out[:, 0], minlength=V)
+    p0 = np.exp(tl[0].astype(np.float64))
+    p0 /= p0.sum()
+    stat = ((counts - n * p0) ** 2 / (n * p0)).sum()
+    assert stat < stats.chi2.ppf(1 - 1e-3, V - 1), stat
+    # prefix survival (Appendix A.1): E[n_acc] = sum_i prod_{j<=i} alpha_j
+    q = np.exp(dl.astype(np.float64))
+    q /= q.sum(axis=1, keepdims=True)
+    p = np.exp(tl.astype(np.float64))
+    p /= p.sum(axis=1, keepdims=True)
+    expect = np.cumprod(np.minimum(p[:gamma], q).sum(axis=1)).sum()
+    assert abs(n_acc.mean() - expect) < 5 * n_acc.std() / np.sqrt(n)
+    m = 20_000  # trial-by-trial agreement with the oracle on the first m trials
+    small = dict(target_logits=inp["target_logits"][: m * (gamma + 1)], draft_logits=inp["draft_logits"][: m * gamma],
+                 draft_tokens=inp["draft_tokens"][: m * gamma], cu_draft=inp["cu_draft"][: m + 1],
+                 u_accept=inp["u_accept"][: m * gamma], u_sample=inp["u_sample"][:m])
+    compare_accept(small, 1.0, gpu=(gpu[0][:m], gpu[1][: m * (gamma + 1)], gpu[2][: m * gamma], 0),
+                   ref=run_oracle_accept(small, 1.0))
+
+
+def test_out_of_range_draft_token_sets_device_flag():
+    w = wl.custom(seed=3, ctx=(0, 0), block=(4, 4), vocab=1000)
+    inp = wl.accept_inputs(w, 1.0)
+    inp["draft_tokens"][2] = 1000  # caught by the kernel's own bounds check, never dereferenced
+    status = run_accept(inp, 1.0)[3]
+    assert status == 6  # BP_ERR_DEVICE_FLAG
+
+
+def test_host_side_validation():
+    t = torch.zeros((2, 100), device="cuda")
+    tok = torch.zeros(1, dtype=torch.int32, device="cuda")
+    cu = torch.tensor([0, 1], dtype=torch.int32, device="cuda")
+    with pytest.raises(bp.BlockPilotError) as e:
+        bp.spec_accept(t, None, tok, cu, 1.0, torch.zeros(1, device="cuda"), torch.zeros(1, device="cuda"))
+    assert e.value.status == 1  # T > 0 needs draft logits

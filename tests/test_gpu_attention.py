@@ -1,0 +1,123 @@
+"""GPU parity of bp_block_attention against the fp64 oracle (bf16 tensor-core path and fp32 path).
+
+Tolerance: max |O - O_ref| / max |O_ref| <= 2e-2 per (sequence, query head) slice (bf16 inputs,
+fp32 accumulation); log-sum-exp within 2e-3.  Small ragged cases are compared in full; the
+full-size workloads run exactly as the benchmark launches them and are compared on sampled
+sequences (and KV heads for the 32K-context case).
+"""
+import numpy as np
+import pytest
+import torch
+
+import paper_2606_31315_gb300 as bp
+from paper_2606_31315_gb300 import workloads as wl
+
+from _gpu import ATTN_TOL, LSE_TOL, attention_errors, run_attention, to_dev
+
+pytestmark = pytest.mark.gpu
+
+CAUSAL, BIDIR = bp.MASK_CAUSAL, bp.MASK_BIDIR
+
+
+@pytest.fixture(scope="module", autouse=True)
+def _lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    bp.build()
+    bp.load()
+
+
+def _check(a, mask, seqs=None, kv_head=None):
+    o, lse = run_attention(a, mask)
+    seqs = range(len(a["cu_q"]) - 1) if seqs is None else seqs
+    err, lerr = attention_errors(o, lse, a, mask, seqs, kv_head)
+    assert err <= ATTN_TOL, err
+    assert lerr <= LSE_TOL, lerr
+    return o, lse
+
+
+@pytest.mark.parametrize("mask", [CAUSAL, BIDIR])
+@pytest.mark.parametrize("ctx,block", [
+    ((0, 1, 127, 300, 1000), (1, 8, 16, 24, 13)),   # ragged, tile-crossing contexts, B=1 decode
+    ((129, 0, 5), (64, 2, 33)),                     # B=64: two 128-row query tiles; L=0
+    ((2048,), (16,)),                                # Qwen3-4B verify shape, one sequence
+    ((4000, 10, 255, 256, 257), (16, 16, 16, 16, 16)),
+])
+def test_ragged_small(ctx, block, mask):
+    w = wl.custom(seed=sum(ctx) + len(block), ctx=ctx, block=block, num_q_heads=32, num_kv_heads=8)
+    _check(wl.attention_inputs(w), mask)
+
+
+@pytest.mark.parametrize("hq,hkv", [(8, 8), (64, 8), (16, 2), (4, 1)])
+def test_group_sizes(hq, hkv):
+    w = wl.custom(seed=hq * 10 + hkv, ctx=(300, 77), block=(12, 31), num_q_heads=hq, num_kv_heads=hkv)
+    for mask in (CAUSAL, BIDIR):
+        _check(wl.attention_inputs(w), mask)
+
+
+def test_qwen3_4b_full():
+    a = wl.attention_inputs(wl.get("qwen3_4b"))
+    _check(a, CAUSAL)
+    _check(a, BIDIR)
+
+
+def test_ragged_batch_full_size_sampled():
+    w = wl.get("ragged")
+    a = wl.attention_inputs(w)
+    lens = np.diff(a["cu_kv"])
+    seqs = sorted({0, 5, 31, int(np.argmax(lens)), int(np.argmin(lens))})
+    _check(a, CAUSAL, seqs=seqs)
+
+
+def test_drafter_bidir_full_size_sampled():
+    a = wl.attention_inputs(wl.get("drafter_bidir"))
+    _check(a, BIDIR, seqs=[0, 9, 15])
+
+
+def test_long_context_full_size_sampled():
+    a = wl.attention_inputs(wl.get("long_context"))
+    o, lse = run_attention(a, CAUSAL)
+    for s, kvh in ((0, 0), (7, 5), (3, 7)):
+        err, lerr = attention_errors(o, lse, a, CAUSAL, [s], kv_head=kvh)
+        assert err <= ATTN_TOL and lerr <= LSE_TOL, (s, kvh, err, lerr)
+
+
+def test_tiny_fp32():
+    a = wl.attention_inputs(wl.get("tiny"))
+    for mask in (CAUSAL, BIDIR):
+        o, lse = run_attention(a, mask)
+        err, lerr = attention_errors(o, lse, a, mask, [0])
+        assert err <= 1e-5 and lerr <= 1e-5, (err, lerr)
+
+
+def test_causal_last_row_equals_bidir_last_row():
+    a = wl.attention_inputs(wl.custom(seed=5, ctx=(700, 90), block=(16, 9), num_q_heads=32, num_kv_heads=8))
+    oc, _ = run_attention(a, CAUSAL)
+    ob, _ = run_attention(a, BIDIR)
+    last = a["cu_q"][1:] - 1
+    np.testing.assert_allclose(oc[last], ob[last], rtol=0, atol=1e-2)
+
+
+def test_empty_blocks_and_empty_batch():
+    a = wl.attention_inputs(wl.custom(seed=6, ctx=(10, 0, 40), block=(0, 0, 8), num_q_heads=32, num_kv_heads=8))
+    _check(a, CAUSAL)
+    q = torch.zeros((0, 32, 128), dtype=torch.bfloat16, device="cuda")
+    k = torch.zeros((0, 8, 128), dtype=torch.bfloat16, device="cuda")
+    cu = torch.zeros(1, dtype=torch.int32, device="cuda")
+    o, _ = bp.block_attention(q, k, k, cu, cu, 0, 0)
+    assert o.shape == q.shape
+
+
+def test_invalid_arguments_are_rejected_on_the_host():
+    a = wl.attention_inputs(wl.custom(seed=1, ctx=(10,), block=(4,), num_q_heads=6, num_kv_heads=4))
+    q, k, v = to_dev(a["q"], "bf16"), to_dev(a["k"], "bf16"), to_dev(a["v"], "bf16")
+    cu_q, cu_kv = to_dev(a["cu_q"]), to_dev(a["cu_kv"])
+    with pytest.raises(bp.BlockPilotError) as e:
+        bp.block_attention(q, k, v, cu_q, cu_kv, 4, 14)  # 6 % 4 != 0
+    assert e.value.status == 1
+    w64 = wl.custom(seed=2, ctx=(10,), block=(4,), num_q_heads=4, num_kv_heads=2, head_dim=64)
+    a64 = wl.attention_inputs(w64)
+    with pytest.raises(bp.BlockPilotError) as e:
+        bp.block_attention(to_dev(a64["q"], "bf16"), to_dev(a64["k"], "bf16"), to_dev(a64["v"], "bf16"),
+                           to_dev(a64["cu_q"]), to_dev(a64["cu_kv"]), 4, 14)
+    assert e.value.status == 2
