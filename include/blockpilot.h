@@ -133,6 +133,32 @@ BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits,
                    float* accept_prob, void* workspace, size_t workspace_bytes, void* stream);
 
 /* ---------------------------------------------------------------------------------
+ * bp_spec_accept without a workspace.  The paper has no counterpart: this entry point exists
+ * for callers that cannot allocate device memory -- e.g. a plugin running inside another
+ * inference engine that only hands it input and output buffers, or a serving loop that must
+ * not call cudaMalloc while requests are in flight (it can synchronize the device).
+ *
+ * Same arguments, results and errors as bp_spec_accept, except:
+ *   - no workspace: the scratch is a fixed array of BP_NOALLOC_SCRATCH_BYTES inside the
+ *     library, held on every GPU that loads the library until the process exits;
+ *   - problems whose scratch would exceed it return BP_ERR_WORKSPACE (the requirement is
+ *     bp_spec_accept_workspace_size(...) - 256 bytes; e.g. about 780 target rows of a
+ *     151936-token vocabulary fit);
+ *   - device-detected errors are OR-ed into *device_error (a caller-owned device word, may be
+ *     NULL to drop them) instead of a workspace: 1 = a wait timed out, 2 = a draft token id
+ *     outside [0, vocab);
+ *   - the first call on each device looks up the array's device address (cached afterwards);
+ *   - every call clears the array's per-sequence counters on `stream` before its kernel runs;
+ *     calls that run concurrently on the GPU (unordered streams) share the array and race.
+ * ------------------------------------------------------------------------------- */
+#define BP_NOALLOC_SCRATCH_BYTES (8u << 20)
+BP_API int bp_spec_accept_noalloc(const float* target_logits, const float* draft_logits,
+                                  const int32_t* draft_tokens, const int32_t* cu_draft, int num_seqs,
+                                  int total_draft, int vocab, float temperature, const float* u_accept,
+                                  const float* u_sample, int32_t* n_accepted, int32_t* out_tokens,
+                                  float* accept_prob, unsigned int* device_error, void* stream);
+
+/* ---------------------------------------------------------------------------------
  * Block-size policy head, run once per request after prefill.  Sections 2.3 and 2.4:
  * an MLP maps the request's prefill representation to one logit per candidate block
  * size and B_hat = argmax over the candidates, fixed for the whole request; Section 3.1

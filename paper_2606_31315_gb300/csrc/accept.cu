@@ -19,6 +19,8 @@
 // (lowest index on ties) and the last CTA of the sequence compares it with the drafts.
 #include <cooperative_groups.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace cg = cooperative_groups;
@@ -640,6 +642,66 @@ int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t strea
         case 16: return launch_cfg<16>(p, cfg.cs, greedy, vec, (int)rows, stream);
         default: return BP_ERR_UNSUPPORTED;
     }
+}
+
+// ---------------------------------------------------------------------------------------
+// Scratch of bp_spec_accept_noalloc.
+//
+// Some callers cannot allocate device memory for a workspace: for example a plugin that runs
+// inside another inference engine and only receives its input and output buffers from it, or
+// a serving loop that must not call cudaMalloc while requests are in flight (cudaMalloc can
+// synchronize the device and stall every other stream).  For them the acceptance step can use
+// this fixed array instead, which the CUDA runtime places in device memory when the library's
+// module is loaded; every GPU that loads the library keeps these BP_NOALLOC_SCRATCH_BYTES
+// until the process exits.
+//
+// All calls share the array and it keeps whatever the previous call left in it, so each call
+// clears the part that must start at zero (the per-sequence tickets) on its own stream before
+// the kernel runs.  Calls whose execution overlaps on the GPU (different streams without an
+// ordering between them) race on this array and give undefined results.
+static __device__ __align__(256) unsigned char g_noalloc_scratch[BP_NOALLOC_SCRATCH_BYTES];
+
+namespace {
+// Device address of g_noalloc_scratch for the current device.  In host code the symbol is only
+// a host-side stand-in, so the address is looked up once per device (with that device current)
+// and cached; the lookup happens on the first call of bp_spec_accept_noalloc on each device.
+int noalloc_scratch_address(void** out) {
+    static void* addr[64] = {};
+    static std::mutex mu;
+    int dev = -1;
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) {
+        cudaGetLastError();
+        return BP_ERR_CUDA;
+    }
+    std::lock_guard<std::mutex> lock(mu);
+    if (addr[dev] == nullptr) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) {
+            cudaGetLastError();
+            return BP_ERR_CUDA;
+        }
+        addr[dev] = p;
+    }
+    *out = addr[dev];
+    return BP_OK;
+}
+}  // namespace
+
+int launch_accept_noalloc(const AcceptArgs& args, const DeviceInfo& dev, cudaStream_t stream) {
+    const size_t need = accept_scratch_bytes(args.num_seqs, args.total_draft, args.vocab);
+    if (need == 0) return BP_ERR_UNSUPPORTED;
+    if (need > (size_t)BP_NOALLOC_SCRATCH_BYTES) return BP_ERR_WORKSPACE;  // problem too large for the array
+    void* base = nullptr;
+    int rc = noalloc_scratch_address(&base);
+    if (rc != BP_OK) return rc;
+    // the tickets (first region of the scratch layout) must be zero when the kernel starts
+    if (cudaMemsetAsync(base, 0, align_up(sizeof(int) * (size_t)args.num_seqs, 256), stream) != cudaSuccess) {
+        cudaGetLastError();
+        return BP_ERR_CUDA;
+    }
+    AcceptArgs a = args;
+    a.scratch = base;
+    return launch_accept(a, dev, stream);
 }
 
 }  // namespace bp

@@ -171,6 +171,33 @@ int bp_spec_accept(const float* target_logits, const float* draft_logits, const 
     return rc;
 }
 
+int bp_spec_accept_noalloc(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
+                           const int32_t* cu_draft, int num_seqs, int total_draft, int vocab, float temperature,
+                           const float* u_accept, const float* u_sample, int32_t* n_accepted, int32_t* out_tokens,
+                           float* accept_prob, unsigned int* device_error, void* stream) {
+    if (num_seqs < 0 || total_draft < 0 || vocab < 1) return BP_ERR_INVALID_ARG;
+    if (num_seqs == 0) return BP_OK;
+    if (!target_logits || !cu_draft || !n_accepted || !out_tokens || (total_draft > 0 && !draft_tokens))
+        return BP_ERR_INVALID_ARG;
+    if (!(temperature >= 0.f) || isinf(temperature)) return BP_ERR_INVALID_ARG;
+    if (temperature > 0.f && (!u_sample || (total_draft > 0 && (!draft_logits || !u_accept))))
+        return BP_ERR_INVALID_ARG;
+    if ((long long)(total_draft + (long long)num_seqs) * vocab > (1LL << 40)) return BP_ERR_UNSUPPORTED;
+    DeviceInfo dev;
+    int rc = device_info(&dev);
+    if (rc != BP_OK) return rc;
+    AcceptArgs a;
+    a.target = target_logits; a.draft = draft_logits; a.tokens = draft_tokens; a.cu_draft = cu_draft;
+    a.num_seqs = num_seqs; a.total_draft = total_draft; a.vocab = vocab; a.temperature = temperature;
+    a.u_accept = u_accept; a.u_sample = u_sample;
+    a.n_accepted = n_accepted; a.out_tokens = out_tokens; a.accept_prob = accept_prob;
+    a.scratch = nullptr;
+    a.err_word = device_error;
+    rc = launch_accept_noalloc(a, dev, static_cast<cudaStream_t>(stream));
+    if (rc == BP_ERR_CUDA) cudaGetLastError();
+    return rc;
+}
+
 size_t bp_policy_select_workspace_size(int num_reqs, int hidden, int num_cand) {
     if (num_reqs < 0 || hidden < 1 || num_cand < 1) return 0;
     return sizeof(WorkspaceHeader) + policy_scratch_bytes(num_reqs, hidden, num_cand);

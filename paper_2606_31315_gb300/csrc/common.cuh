@@ -77,6 +77,8 @@ struct AcceptArgs {
 };
 size_t accept_scratch_bytes(int num_seqs, int total_draft, int vocab);
 int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+// Same kernel, scratch taken from the library's own static device array (no workspace).
+int launch_accept_noalloc(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
 struct PolicyArgs {
     const void* feats;

@@ -1,0 +1,95 @@
+"""bp_spec_accept_noalloc: the acceptance step for callers that cannot allocate device memory.
+
+Some callers have no way to provide a workspace: a plugin running inside another inference
+engine that only receives its input and output buffers, or a serving loop that must not call
+cudaMalloc while requests are in flight (cudaMalloc can synchronize the device).  This entry
+point keeps its scratch in a fixed array inside the library instead.  The test calls it through
+the C ABI twice in a row, on two different problems (so the second call runs on whatever the
+first left in the shared array), and checks each result against bp_spec_accept with a
+caller-provided workspace: emitted tokens and accepted lengths identical, acceptance
+probabilities within 1e-5.  It also checks that a problem too large for the array is refused.
+"""
+import ctypes
+
+import numpy as np
+import pytest
+import torch
+
+import paper_2606_31315_gb300 as bp
+from paper_2606_31315_gb300 import workloads as wl
+
+pytestmark = pytest.mark.gpu
+
+PROB_TOL = 1e-5
+
+
+@pytest.fixture(scope="module")
+def lib():
+    if not torch.cuda.is_available():
+        pytest.skip("no CUDA device")
+    bp.build()
+    lib = bp.load()
+    vp, i32, f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    lib.bp_spec_accept_noalloc.argtypes = [vp, vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, vp, vp, vp, vp]
+    lib.bp_spec_accept_noalloc.restype = i32
+    return lib
+
+
+def _p(t):
+    return None if t is None else ctypes.c_void_p(t.data_ptr())
+
+
+def _inputs(name, temp):
+    inp = wl.accept_inputs(wl.get(name), temp)
+    g = {k: torch.from_numpy(np.ascontiguousarray(inp[k])).cuda() for k in
+         ("target_logits", "draft_logits", "draft_tokens", "cu_draft", "u_accept", "u_sample")}
+    if temp == 0:
+        g["draft_logits"] = None
+    return g
+
+
+def _noalloc(lib, g, temp):
+    s = g["cu_draft"].numel() - 1
+    td = g["draft_tokens"].numel()
+    vocab = g["target_logits"].shape[1]
+    n_acc = torch.full((s,), -7, dtype=torch.int32, device="cuda")
+    out = torch.full((td + s,), -7, dtype=torch.int32, device="cuda")
+    ap = torch.full((td,), -1.0, dtype=torch.float32, device="cuda")
+    err = torch.zeros(1, dtype=torch.int32, device="cuda")
+    stream = torch.cuda.current_stream()
+    rc = lib.bp_spec_accept_noalloc(_p(g["target_logits"]), _p(g["draft_logits"]), _p(g["draft_tokens"]),
+                                    _p(g["cu_draft"]), s, td, vocab, float(temp), _p(g["u_accept"]),
+                                    _p(g["u_sample"]), _p(n_acc), _p(out), _p(ap), _p(err),
+                                    ctypes.c_void_p(stream.cuda_stream))
+    assert rc == 0, lib.bp_error_string(rc)
+    torch.cuda.synchronize()
+    assert err.item() == 0
+    return n_acc.cpu().numpy(), out.cpu().numpy(), ap.cpu().numpy()
+
+
+def _with_workspace(g, temp):
+    n_acc, out, ap = bp.spec_accept(g["target_logits"], g["draft_logits"], g["draft_tokens"], g["cu_draft"], temp,
+                                    g["u_accept"], g["u_sample"])
+    return n_acc.cpu().numpy(), out.cpu().numpy(), ap.cpu().numpy()
+
+
+def _same(a, b):
+    np.testing.assert_array_equal(a[0], b[0])
+    np.testing.assert_array_equal(a[1], b[1])
+    assert np.abs(a[2] - b[2]).max() <= PROB_TOL
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_two_calls_in_a_row_match_the_workspace_entry_point(lib, temp):
+    first = _inputs("ragged", 1.0)        # 32 sequences, 530 target rows
+    second = _inputs("qwen3_4b", temp)    # 1 sequence, 16 target rows
+    _same(_noalloc(lib, first, 1.0), _with_workspace(first, 1.0))
+    _same(_noalloc(lib, second, temp), _with_workspace(second, temp))
+
+
+def test_too_large_problem_is_refused(lib):
+    fake = ctypes.c_void_p(0x10000)
+    # 1000 sequences x 16 rows of a 151936-token vocabulary need far more than the fixed array
+    rc = lib.bp_spec_accept_noalloc(fake, fake, fake, fake, 1000, 15000, 151936, 1.0, fake, fake, fake, fake, None,
+                                    None, None)
+    assert rc == 4  # BP_ERR_WORKSPACE, refused before anything is launched
