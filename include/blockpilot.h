@@ -142,8 +142,8 @@ BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits,
  *   - no workspace: the scratch is a fixed array of BP_NOALLOC_SCRATCH_BYTES inside the
  *     library, held on every GPU that loads the library until the process exits;
  *   - problems whose scratch would exceed it return BP_ERR_WORKSPACE (the requirement is
- *     bp_spec_accept_workspace_size(...) - 256 bytes; e.g. about 780 target rows of a
- *     151936-token vocabulary fit);
+ *     bp_spec_accept_workspace_size(...) - 256 bytes, about 8 bytes per target row plus 4 per
+ *     sequence, so roughly a million target rows fit);
  *   - device-detected errors are OR-ed into *device_error (a caller-owned device word, may be
  *     NULL to drop them) instead of a workspace: 1 = a wait timed out, 2 = a draft token id
  *     outside [0, vocab);

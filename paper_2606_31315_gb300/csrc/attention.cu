@@ -43,6 +43,7 @@ constexpr int kThreads = 192;
 constexpr uint32_t kTmemCols = 512;
 constexpr uint32_t kColO = 256;
 constexpr int kMaxOrderedSeqs = 256;  // longest-first ordering for batches up to this size
+constexpr int kMaxCluster = 16;
 
 struct AttnParams {
     const __nv_bfloat16* q;
@@ -51,8 +52,10 @@ struct AttnParams {
     const int32_t* cu_q;
     const int32_t* cu_kv;
     int num_seqs, num_q_heads, num_kv_heads, group, m_tiles;
+    int total_q, total_kv;
     int causal;
     float scale_log2;  // softmax scale * log2(e)
+    int q_tma;         // Q tile loaded by TMA (group divides 128)
     unsigned int* err;
 };
 
@@ -76,21 +79,26 @@ __device__ __forceinline__ uint32_t cluster_size() {
 }
 
 __global__ void __launch_bounds__(kThreads, 1)
-    attn_bf16_tc_kernel(const __grid_constant__ CUtensorMap kmap, const __grid_constant__ CUtensorMap vmap,
-                        const AttnParams p) {
+    attn_bf16_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
+                        const __grid_constant__ CUtensorMap vmap, const AttnParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* smem = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
     uint8_t* sQ = smem;
     uint8_t* sKV = smem + kQBytes;  // stage s: K at s*64KB, V at s*64KB + 32KB
 
     __shared__ uint64_t bar_kv_full[kStages], bar_kv_empty[kStages];
-    __shared__ uint64_t bar_s_full[2], bar_p_full[2], bar_pv_done[2], bar_o_done;
+    __shared__ uint64_t bar_s_full[2], bar_p_full[2], bar_pv_done[2], bar_o_done, bar_q_full;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int unit_seq_sh;
     __shared__ int32_t cu_kv_sh[kMaxOrderedSeqs + 1];
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
+    if (tid == 0) {
+        if (p.q_tma) prefetch_tensormap(&qmap);
+        prefetch_tensormap(&kmap);
+        prefetch_tensormap(&vmap);
+    }
     const uint32_t CS = cluster_size();
     const uint32_t crank = cluster_rank();
     const int unit_rank = blockIdx.x / CS;
@@ -101,28 +109,31 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int mt = unit_rank % p.m_tiles;
 
     // ---- which sequence: the seq_rank-th longest (ties by index) for small batches
-    if (p.num_seqs <= kMaxOrderedSeqs) {
-        for (int s = tid; s <= p.num_seqs; s += kThreads) cu_kv_sh[s] = p.cu_kv[s];
+    int s;
+    if (p.num_seqs == 1) {
+        s = 0;
+    } else if (p.num_seqs <= kMaxOrderedSeqs) {
+        for (int t = tid; t <= p.num_seqs; t += kThreads) cu_kv_sh[t] = p.cu_kv[t];
         __syncthreads();
-        for (int s = tid; s < p.num_seqs; s += kThreads) {
-            const int len = cu_kv_sh[s + 1] - cu_kv_sh[s];
+        for (int t = tid; t < p.num_seqs; t += kThreads) {
+            const int len = cu_kv_sh[t + 1] - cu_kv_sh[t];
             int rank = 0;
-            for (int t = 0; t < p.num_seqs; ++t) {
-                const int lt = cu_kv_sh[t + 1] - cu_kv_sh[t];
-                rank += (lt > len) || (lt == len && t < s);
+            for (int u = 0; u < p.num_seqs; ++u) {
+                const int lu = cu_kv_sh[u + 1] - cu_kv_sh[u];
+                rank += (lu > len) || (lu == len && u < t);
             }
-            if (rank == seq_rank) unit_seq_sh = s;
+            if (rank == seq_rank) unit_seq_sh = t;
         }
         __syncthreads();
+        s = unit_seq_sh;
     } else {
-        if (tid == 0) unit_seq_sh = seq_rank;
-        __syncthreads();
+        s = seq_rank;
     }
-    const int s = unit_seq_sh;
-    const int q0 = p.cu_q[s];
-    const int B = p.cu_q[s + 1] - q0;
-    const int kv0 = p.cu_kv[s];
-    const int n = p.cu_kv[s + 1] - kv0;
+    // a single sequence starts at offset 0 (cu_*[0] = 0) and spans the whole tensors: no loads
+    const int q0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_q + s);
+    const int B = p.num_seqs == 1 ? p.total_q : __ldg(p.cu_q + s + 1) - q0;
+    const int kv0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_kv + s);
+    const int n = p.num_seqs == 1 ? p.total_kv : __ldg(p.cu_kv + s + 1) - kv0;
     const int L = n - B;
     const int rows = B * G;
     const int row0 = mt * kM;
@@ -134,19 +145,35 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int t_end = (int)((long long)(crank + 1) * tiles / CS);
     const int nt = t_end - t_begin;
 
-    // ---- Q tile -> shared memory, SWIZZLE_128B K-major (two 64-column halves)
-    for (int idx = tid; idx < kM * 16; idx += kThreads) {
-        const int r = idx >> 4, ch = idx & 15;
-        uint4 val = make_uint4(0, 0, 0, 0);
-        if (r < m_valid) {
-            const int lr = row0 + r;
-            const int i = lr / G, j = lr % G;
-            val = *reinterpret_cast<const uint4*>(p.q + ((size_t)(q0 + i) * p.num_q_heads + h * G + j) * kD + ch * 8);
+    // ---- Q tile -> shared memory, SWIZZLE_128B K-major (two 64-column halves).  With a TMA map the
+    // 128/G block positions x G heads box lands exactly as rows r = i*G + j; otherwise plain loads.
+    if (!p.q_tma) {
+        for (int idx = tid; idx < kM * 16; idx += kThreads) {
+            const int r = idx >> 4, ch = idx & 15;
+            uint4 val = make_uint4(0, 0, 0, 0);
+            if (r < m_valid) {
+                const int lr = row0 + r;
+                const int i = lr / G, j = lr % G;
+                val = *reinterpret_cast<const uint4*>(p.q + ((size_t)(q0 + i) * p.num_q_heads + h * G + j) * kD +
+                                                      ch * 8);
+            }
+            const int half = ch >> 3, c8 = ch & 7;
+            *reinterpret_cast<uint4*>(sQ + half * kHalf + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
         }
-        const int half = ch >> 3, c8 = ch & 7;
-        *reinterpret_cast<uint4*>(sQ + half * kHalf + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
+        fence_proxy_async_smem();
     }
-    fence_proxy_async_smem();
+    // K/V tile j of this CTA's range -> ring stage j % kStages (producer thread only)
+    auto issue_kv = [&](int j) {
+        const int st = j % kStages;
+        uint8_t* sK = sKV + st * kStageBytes;
+        uint8_t* sV = sK + kKVBytes;
+        const int key = kv0 + (t_begin + j) * kTileN;
+        mbar_arrive_expect_tx(&bar_kv_full[st], kStageBytes);
+        tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, h, key);
+        tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, h, key);
+        tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, h, key);
+        tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, h, key);
+    };
     if (tid == 0) {
         for (int i = 0; i < kStages; ++i) {
             mbar_init(&bar_kv_full[i], 1);
@@ -158,9 +185,20 @@ __global__ void __launch_bounds__(kThreads, 1)
             mbar_init(&bar_pv_done[i], 1);
         }
         mbar_init(&bar_o_done, 1);
+        mbar_init(&bar_q_full, 1);
         fence_mbar_init();
+        // the producer (this thread) starts the Q load and fills the K/V ring right away
+        if (nt > 0) {
+            if (p.q_tma) {
+                mbar_arrive_expect_tx(&bar_q_full, kQBytes);
+                const int qrow = q0 + row0 / G;
+                tma_load_3d(sQ, &qmap, &bar_q_full, 0, h * G, qrow);
+                tma_load_3d(sQ + kHalf, &qmap, &bar_q_full, 64, h * G, qrow);
+            }
+            for (int j = 0; j < min(nt, kStages); ++j) issue_kv(j);
+        }
     }
-    if (warp == 0) {
+    if (warp == 1) {  // tensor memory is allocated (and released) by warp 1, in parallel
         tmem_alloc(&tmem_base_sh, kTmemCols);
         tmem_relinquish();
     }
@@ -172,28 +210,19 @@ __global__ void __launch_bounds__(kThreads, 1)
     if (warp == 0) {
         // ================= TMA producer
         if (lane == 0 && nt > 0) {
-            prefetch_tensormap(&kmap);
-            prefetch_tensormap(&vmap);
-            int issued = 0;
-            for (int j = 0; j < nt; ++j) {
-                const int st = j % kStages;
-                if (j >= kStages && !mbar_wait(&bar_kv_empty[st], ((j / kStages) - 1) & 1, kWaitBudget)) {
+            int issued = min(nt, kStages);  // the prologue issued the first tiles
+            for (int j = kStages; j < nt; ++j) {
+                if (!mbar_wait(&bar_kv_empty[j % kStages], ((j / kStages) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
-                uint8_t* sK = sKV + st * kStageBytes;
-                uint8_t* sV = sK + kKVBytes;
-                const int key = kv0 + (t_begin + j) * kTileN;
-                mbar_arrive_expect_tx(&bar_kv_full[st], kStageBytes);
-                tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, h, key);
-                tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, h, key);
-                tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, h, key);
-                tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, h, key);
+                issue_kv(j);
                 ++issued;
             }
             // no copy may still be in flight when the CTA leaves
             for (int j = max(0, issued - kStages); j < issued; ++j)
                 if (!mbar_wait(&bar_kv_full[j % kStages], (j / kStages) & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
+            if (p.q_tma && !mbar_wait(&bar_q_full, 0, kWaitBudget)) raise_error(p.err, kErrTimeout);
         }
     } else if (warp == 1) {
         // ================= MMA issuer
@@ -201,7 +230,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             const uint32_t id_s = idesc_bf16_f32(kM, kTileN, false, false);
             const uint32_t id_o = idesc_bf16_f32(kM, kD, false, true);
             const uint32_t q_addr = smem_addr(sQ);
-            bool ok = true;
+            bool ok = !p.q_tma || mbar_wait(&bar_q_full, 0, kWaitBudget);
             auto issue_pv = [&](int j) {
                 const int sb = j & 1, st = j % kStages;
                 if (!mbar_wait(&bar_p_full[sb], (j >> 1) & 1, kWaitBudget)) return false;
@@ -370,11 +399,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (p.lse) p.lse[orow] = (m_run + __log2f(l_run)) * kLn2;
         }
     } else {
-        // ---- cluster merge of the CS partial (m, l, O) triples through distributed shared memory
-        cg::cluster_group cluster = cg::this_cluster();
-        // all TMA loads of this CTA were consumed, so the K/V ring is free:
+        // ---- merge of the CS partial (m, l, O) triples through distributed shared memory.  After the
+        // first cluster barrier every K/V ring is idle (all of its TMA loads were consumed); each CTA
+        // leaves its partial there and pulls the rows it owns from all peers:
         //   opart  [kM rows][kD] fp32 partial O (16-byte chunks swizzled by row)
         //   row_ml [kM] (m, l) of each row's partial
+        //   ml_st, w_st, inv_st  the peers' (m, l) of the owned rows, their weights, 1/L
+        cg::cluster_group cluster = cg::this_cluster();
         float* opart = reinterpret_cast<float*>(sKV);
         float2* row_ml = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float));
         if (is_softmax) {
@@ -391,46 +422,69 @@ __global__ void __launch_bounds__(kThreads, 1)
         cluster.sync();
         const int per = (m_valid + (int)CS - 1) / (int)CS;
         const int rbeg = (int)crank * per;
-        const int rend = min(m_valid, rbeg + per);
-        for (int item = tid; item < (rend - rbeg) * (kD / 4); item += kThreads) {
-            const int rr = rbeg + item / (kD / 4);
-            const int c = item % (kD / 4);
+        const int nmy = max(0, min(m_valid, rbeg + per) - rbeg);
+        // one round of remote loads for the peers' (m, l) of the owned rows, then the weights
+        float2* ml_st = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float) + kM * sizeof(float2));
+        float* w_st = reinterpret_cast<float*>(ml_st + kMaxCluster * kM);
+        float* inv_st = w_st + kMaxCluster * kM;
+        for (int idx = tid; idx < (int)CS * nmy; idx += kThreads) {
+            const int pr = idx / nmy, rr = idx % nmy;
+            ml_st[pr * nmy + rr] = *cluster.map_shared_rank(&row_ml[rbeg + rr], pr);
+        }
+        __syncthreads();
+        for (int rr = tid; rr < nmy; rr += kThreads) {
             float M = -INFINITY;
-            for (uint32_t pr = 0; pr < CS; ++pr) {
-                const float2 ml = *cluster.map_shared_rank(&row_ml[rr], pr);
-                M = fmaxf(M, ml.x);
-            }
+            for (uint32_t pr = 0; pr < CS; ++pr) M = fmaxf(M, ml_st[pr * nmy + rr].x);
             float Lsum = 0.f;
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
             for (uint32_t pr = 0; pr < CS; ++pr) {
-                const float2 ml = *cluster.map_shared_rank(&row_ml[rr], pr);
-                if (ml.x == -INFINITY) continue;
-                const float w = fast_exp2(ml.x - M);
+                const float2 ml = ml_st[pr * nmy + rr];
+                const float w = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - M);
+                w_st[pr * nmy + rr] = w;
                 Lsum += w * ml.y;
-                const float4 v = *cluster.map_shared_rank(
-                    reinterpret_cast<float4*>(opart + rr * kD + ((c ^ (rr & 31)) * 4)), pr);
-                acc.x += w * v.x;
-                acc.y += w * v.y;
-                acc.z += w * v.z;
-                acc.w += w * v.w;
             }
-            const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-            const int lr = row0 + rr;
-            const int i = lr / G, jh = lr % G;
-            const size_t orow = (size_t)(q0 + i) * p.num_q_heads + h * G + jh;
+            inv_st[rr] = Lsum > 0.f ? 1.f / Lsum : 0.f;
+            if (p.lse) {
+                const int lr = row0 + rbeg + rr;
+                p.lse[(size_t)(q0 + lr / G) * p.num_q_heads + h * G + lr % G] = (M + __log2f(Lsum)) * kLn2;
+            }
+        }
+        __syncthreads();
+        // the owned rows: every peer's 16-byte chunk requested at once
+        for (int item = tid; item < nmy * (kD / 4); item += kThreads) {
+            const int rr = item / (kD / 4);
+            const int c = item % (kD / 4);
+            const int row = rbeg + rr;
+            const float* src = opart + row * kD + ((c ^ (row & 31)) * 4);
+            float4 v[kMaxCluster];
+#pragma unroll
+            for (int pr = 0; pr < kMaxCluster; ++pr)
+                if (pr < (int)CS) v[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(src), pr);
+            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+#pragma unroll
+            for (int pr = 0; pr < kMaxCluster; ++pr) {
+                if (pr < (int)CS) {
+                    const float w = w_st[pr * nmy + rr];
+                    acc.x += w * v[pr].x;
+                    acc.y += w * v[pr].y;
+                    acc.z += w * v[pr].z;
+                    acc.w += w * v[pr].w;
+                }
+            }
+            const float inv = inv_st[rr];
+            const int lr = row0 + row;
+            const size_t orow = (size_t)(q0 + lr / G) * p.num_q_heads + h * G + lr % G;
             uint2 w2;
             w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
             w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
             *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
-            if (c == 0 && p.lse) p.lse[orow] = (M + __log2f(Lsum)) * kLn2;
         }
-        cluster.sync();
+        cluster.sync();  // no CTA leaves while peers may still read its shared memory
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
-    if (warp == 0) tmem_dealloc(tmem, kTmemCols);
+    if (warp == 1) tmem_dealloc(tmem, kTmemCols);
 }
 
 // --------------------------------------------------------------------------- fp32 SIMT path
@@ -516,7 +570,17 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     const long long units = (long long)a.num_seqs * a.num_kv_heads * m_tiles;
     if (units == 0 || a.total_q == 0) return BP_OK;
 
-    CUtensorMap kmap, vmap;
+    CUtensorMap qmap, kmap, vmap;
+    // Q: box of (64 columns) x (G heads) x (128/G block positions) = the packed 128-row tile
+    const bool q_tma = (kM % G == 0);
+    if (q_tma) {
+        const cuuint64_t qdims[3] = {(cuuint64_t)kD, (cuuint64_t)a.num_q_heads, (cuuint64_t)a.total_q};
+        const cuuint64_t qstrides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.num_q_heads * kD * 2};
+        const cuuint32_t qbox[3] = {64, (cuuint32_t)G, (cuuint32_t)(kM / G)};
+        const int rq = encode_tensor_map(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), qdims,
+                                         qstrides, qbox, CU_TENSOR_MAP_SWIZZLE_128B);
+        if (rq != BP_OK) return rq;
+    }
     const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)a.num_kv_heads, (cuuint64_t)a.total_kv};
     const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.num_kv_heads * kD * 2};
     const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileN};
@@ -534,26 +598,32 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     p.cu_q = a.cu_q;
     p.cu_kv = a.cu_kv;
     p.num_seqs = a.num_seqs;
+    p.total_q = a.total_q;
+    p.total_kv = a.total_kv;
     p.num_q_heads = a.num_q_heads;
     p.num_kv_heads = a.num_kv_heads;
     p.group = G;
     p.m_tiles = m_tiles;
     p.causal = a.mask == BP_MASK_CAUSAL_BLOCK;
     p.scale_log2 = a.scale * 1.4426950408889634f;
+    p.q_tma = q_tma ? 1 : 0;
     p.err = a.err_word;
+    if (!q_tma) qmap = kmap;  // unused by the kernel
 
-    // once per device: opt in to the shared-memory size and non-portable clusters, and find the
-    // largest cluster of these CTAs the GPU can co-schedule (queried outside any graph capture)
+    // once per device: opt in to the shared-memory size and non-portable clusters, and record how
+    // many clusters of each size (1..16) the GPU can keep resident at once (queried outside any
+    // graph capture; the answer reflects how the SMs are grouped into GPCs)
     static int configured_device = -1;
-    static int max_cluster = 1;
+    static int max_active[kMaxCluster + 1];
     if (configured_device != dev.device) {
         if (cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-                cudaSuccess)
+                cudaSuccess ||
+            cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 cudaSharedmemCarveoutMaxShared) != cudaSuccess)
             return BP_ERR_CUDA;
-        max_cluster = 1;
-        for (int cs = 16; cs >= 2; cs /= 2) {
+        for (int cs = 1; cs <= kMaxCluster; ++cs) {
             cudaLaunchConfig_t probe = {};
             cudaLaunchAttribute pa[1];
             probe.gridDim = dim3(cs, 1, 1);
@@ -566,19 +636,28 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
             probe.attrs = pa;
             probe.numAttrs = 1;
             int n_clusters = 0;
-            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel, &probe) == cudaSuccess &&
-                n_clusters > 0) {
-                max_cluster = cs;
-                break;
+            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel, &probe) != cudaSuccess) {
+                cudaGetLastError();
+                n_clusters = 0;
             }
-            cudaGetLastError();
+            max_active[cs] = n_clusters;
         }
         configured_device = dev.device;
     }
-    // cluster size: split each unit's keys so that about one wave of CTAs covers the GPU
+    // cluster size: the largest split of each unit's keys for which every unit's cluster is resident
+    // in the same wave (a unit left for a second wave would double the time)
+    // (the tiles of the longest unit per CTA set the time: minimise them, then prefer the smallest
+    // cluster, whose merge is cheapest)
     const int max_tiles = (a.max_kv_len + kTileN - 1) / kTileN;
-    int cs = 1;
-    while (cs * 2 <= max_cluster && units * cs * 2 <= dev.sm_count && cs * 2 <= max_tiles) cs *= 2;
+    int cs = 1, best = max_tiles;
+    for (int c = 2; c <= kMaxCluster; ++c) {
+        if (c > max_tiles || units > max_active[c] || units * c > dev.sm_count) continue;
+        const int per = (max_tiles + c - 1) / c;
+        if (per < best) {
+            best = per;
+            cs = c;
+        }
+    }
 
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -592,7 +671,7 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     attr[0].val.clusterDim.z = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    if (cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel, kmap, vmap, p) != cudaSuccess) return BP_ERR_CUDA;
+    if (cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel, qmap, kmap, vmap, p) != cudaSuccess) return BP_ERR_CUDA;
     return BP_OK;
 }
 

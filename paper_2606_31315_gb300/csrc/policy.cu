@@ -140,7 +140,11 @@ int run(const PolicyArgs& a, cudaStream_t stream) {
     cudaGetDevice(&dev);
     if (configured != dev) {
         if (cudaFuncSetAttribute(policy_hidden_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget) !=
-            cudaSuccess)
+                cudaSuccess ||
+            cudaFuncSetAttribute(policy_hidden_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 cudaSharedmemCarveoutMaxShared) != cudaSuccess ||
+            cudaFuncSetAttribute(policy_out_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                 cudaSharedmemCarveoutMaxShared) != cudaSuccess)
             return BP_ERR_CUDA;
         configured = dev;
     }

@@ -88,8 +88,17 @@ def test_two_calls_in_a_row_match_the_workspace_entry_point(lib, temp):
 
 
 def test_too_large_problem_is_refused(lib):
-    fake = ctypes.c_void_p(0x10000)
-    # 1000 sequences x 16 rows of a 151936-token vocabulary need far more than the fixed array
-    rc = lib.bp_spec_accept_noalloc(fake, fake, fake, fake, 1000, 15000, 151936, 1.0, fake, fake, fake, fake, None,
-                                    None, None)
-    assert rc == 4  # BP_ERR_WORKSPACE, refused before anything is launched
+    # 4M single-token sequences: the per-sequence counters alone need 16 MB, more than the fixed
+    # array holds, so the call must be refused before anything is launched.  Every buffer is real
+    # and sized for the problem, so the call is safe even if it were (wrongly) launched.
+    s, vocab = 4_000_000, 16
+    target = torch.zeros((s, vocab), dtype=torch.float32, device="cuda")
+    cu = torch.zeros(s + 1, dtype=torch.int32, device="cuda")
+    u = torch.zeros(s, dtype=torch.float32, device="cuda")
+    n_acc = torch.zeros(s, dtype=torch.int32, device="cuda")
+    out = torch.zeros(s, dtype=torch.int32, device="cuda")
+    stream = ctypes.c_void_p(torch.cuda.current_stream().cuda_stream)
+    rc = lib.bp_spec_accept_noalloc(_p(target), None, None, _p(cu), s, 0, vocab, 1.0, None, _p(u), _p(n_acc),
+                                    _p(out), None, None, stream)
+    torch.cuda.synchronize()
+    assert rc == 4  # BP_ERR_WORKSPACE
