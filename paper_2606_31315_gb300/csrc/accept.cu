@@ -36,6 +36,7 @@ constexpr int kThreads = 256;
 constexpr int kWarps = kThreads / 32;
 constexpr int kMaxSmemSeqs = 512;  // sequence offsets cached in shared memory (else binary search in L2)
 constexpr int kMaxCS = 16;
+constexpr int kMaxSeg = 16;  // 128-entry segments per warp range (pass 2 keeps one sum per segment per lane)
 
 struct AccParams {
     const float* target;
@@ -53,6 +54,7 @@ struct AccParams {
     float* a_ws;   // [total_draft] ratio a_i
     int* tok_ws;   // [total_rows] token each row would emit (argmax when greedy)
     int chunk4;    // float4 slots per CTA slice
+    int wr;        // float4 slots per warp range of a slice
     unsigned int* err;
 };
 
@@ -78,11 +80,6 @@ __device__ __forceinline__ unsigned long long to_fix(float x) {
     return sh > -24 ? mant >> (-sh) : 0ull;
 }
 
-__device__ __forceinline__ float warp_sum(float v) {
-#pragma unroll
-    for (int o = 16; o; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
-    return v;
-}
 __device__ __forceinline__ float warp_incl_scan_f(float v, int lane) {
 #pragma unroll
     for (int o = 1; o < 32; o <<= 1) {
@@ -141,53 +138,77 @@ __device__ __forceinline__ float4 resid4(float4 p, float4 q) {
                        fmaxf(0.f, __fsub_rn(p.z, q.z)), fmaxf(0.f, __fsub_rn(p.w, q.w)));
 }
 
-// Shared-memory layout of one CTA (dynamic part), for a slice of up to chunk4 float4 slots:
-//   sT [chunk4] float4   target slice: raw logits, then (pass 1) the weights 2^(l*c2 - m_batch)
-//   sD [chunk4] float4   draft slice, likewise
-//   bmT, bmD [nb*256]    m_batch of every (batch, thread): the reference of the stored weights
-//   segR, segP [nseg]    fixed-point segment sums of r and p
-// Thread tid owns slots k*256 + tid; batch b is slots 4b..4b+3 of a thread; segment k*8 + w is
-// the 128 entries of slot k held by warp w (in vocabulary order).
-struct Smem {
-    float4 *sT, *sD;
-    float *bmT, *bmD;
-    unsigned long long *segR, *segP;
-};
-__host__ __device__ inline size_t smem_bytes(int chunk4, bool greedy) {
-    const int K = (chunk4 + kThreads - 1) / kThreads;
-    const int nb = (K + 3) / 4;
-    if (greedy) return (size_t)chunk4 * 16;
-    return (size_t)chunk4 * 32 + (size_t)nb * kThreads * 8 + (size_t)K * kWarps * 16;
-}
-__device__ inline Smem carve(uint8_t* base, int chunk4) {
-    const int K = (chunk4 + kThreads - 1) / kThreads;
-    const int nb = (K + 3) / 4;
-    Smem m;
-    m.sT = reinterpret_cast<float4*>(base);
-    m.sD = m.sT + chunk4;
-    m.bmT = reinterpret_cast<float*>(m.sD + chunk4);
-    m.bmD = m.bmT + nb * kThreads;
-    m.segR = reinterpret_cast<unsigned long long*>(m.bmD + nb * kThreads);
-    m.segP = m.segR + K * kWarps;
-    return m;
+// Shared memory of one CTA: the target slice sT and (sampling only) the draft slice sD, up to
+// chunk4 float4 slots each.  Warp w owns the contiguous slot range [w*wr, w*wr + wr) of both
+// slices and brings it in with its own bulk copies (one mbarrier per range and row), so every
+// warp starts on its range as soon as that range has landed.  Lane l works on the slots
+// w*wr + 32j + l: slot row j of a range is a segment of 128 consecutive vocabulary entries,
+// the leaf of the inverse-CDF search (a range has at most kMaxSeg segments).
+__host__ __device__ inline size_t smem_bytes(int chunk4, bool greedy) { return (size_t)chunk4 * (greedy ? 16 : 32); }
+__host__ __device__ inline int warp_range(int chunk4) { return (chunk4 + kWarps - 1) / kWarps; }
+
+// Lane `lane` of a warp holding the values v[0..31] (per lane) ends with the warp-wide sum of
+// value `lane`: a butterfly that halves the values it carries at every step (31 shuffles).
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int q = 0; q < o; ++q) {
+            const float send = up ? v[q] : v[q + o];
+            const float keep = up ? v[q + o] : v[q];
+            v[q] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    return v[0];
 }
 
-// Brings a slice into shared memory: one bulk copy (16-byte aligned rows) or scalar loads.
+// A warp's range of one row slice -> shared memory: one bulk copy (16-byte aligned rows, lane 0
+// issues it) or plain loads by the warp (padding past the vocabulary reads -inf).
 template <bool VEC>
-__device__ __forceinline__ void fetch_slice(float4* dst, const float* row, int f0, int n4, int V, uint64_t* bar,
-                                            int tid) {
+__device__ __forceinline__ void fetch_range(float4* dst, const float* row, int first4, int nw, int V, uint64_t* bar,
+                                            int lane) {
+    if (nw <= 0) return;
     if (VEC) {
-        if (tid == 0 && n4 > 0) {
-            mbar_arrive_expect_tx(bar, (uint32_t)n4 * 16u);
-            bulk_load(dst, row + (size_t)f0 * 4, (uint32_t)n4 * 16u, bar);
+        if (lane == 0) {
+            mbar_arrive_expect_tx(bar, (uint32_t)nw * 16u);
+            bulk_load(dst, row + (size_t)first4 * 4, (uint32_t)nw * 16u, bar);
         }
     } else {
         float* d = reinterpret_cast<float*>(dst);
-        for (int idx = tid; idx < n4 * 4; idx += kThreads) {
-            const int x = f0 * 4 + idx;
+        for (int idx = lane; idx < nw * 4; idx += 32) {
+            const int x = first4 * 4 + idx;
             d[idx] = x < V ? __ldg(row + x) : -INFINITY;
         }
+        __syncwarp();
     }
+}
+template <bool VEC>
+__device__ __forceinline__ void wait_range(uint64_t* bar, int nw, unsigned int* err) {
+    if (VEC && nw > 0 && !mbar_wait(bar, 0, kWaitBudget)) raise_error(err, kErrTimeout);
+}
+
+// Scaled maximum l*c2 of a lane's entries of a range (-inf if none is finite), then the weights
+// 2^(l*c2 - m) replace the logits in place; returns (m, sum of the weights).
+__device__ __forceinline__ float2 weigh_range(float4* s, int w0, int nw, int Kw, int lane, float c2) {
+    float m = -INFINITY;
+    for (int j = 0; j < Kw; ++j) {
+        const int f = j * 32 + lane;
+        if (f < nw) m = fmaxf(m, max4(s[w0 + f]));
+    }
+    float sum = 0.f;
+    if (m != -INFINITY) {
+        m = __fmul_rn(m, c2);
+        for (int j = 0; j < Kw; ++j) {
+            const int f = j * 32 + lane;
+            if (f < nw) {
+                const float4 e = ex2_4(s[w0 + f], c2, m);
+                sum += sum4(e);
+                s[w0 + f] = e;
+            }
+        }
+    }
+    return make_float2(m, sum);
 }
 
 template <bool GREEDY, bool VEC>
@@ -200,33 +221,39 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     const int V = p.vocab;
 
     extern __shared__ __align__(128) uint8_t dyn_smem[];
-    __shared__ uint64_t bar_t, bar_d;
-    __shared__ int32_t cu_sh[kMaxSmemSeqs + 1];
+    __shared__ uint64_t bar_t[kWarps], bar_d[kWarps];
+    __shared__ int32_t cu_sh[kMaxSmemSeqs + 1];  // sequence offsets; the final step reuses it
     __shared__ float4 red4[kWarps];
     __shared__ int red_i[kWarps];
     __shared__ float4 peer_stat[kMaxCS];     // (scaled max t, sum t, scaled max d, sum d)
     __shared__ float4 peer_x[kMaxCS];        // (t[x_i], d[x_i], owns x_i, -); greedy: (max, index)
     __shared__ ulonglong2 peer_tot[kMaxCS];  // slice totals of r and p (fixed point)
+    __shared__ unsigned long long segR[kWarps * kMaxSeg], segP[kWarps * kMaxSeg];
+    __shared__ ulonglong2 wtot[kWarps];      // range totals of r and p (fixed point)
     __shared__ float4 own_sh;
-    __shared__ ulonglong2 tot_sh[kWarps];
-    __shared__ int sel_sh, last_sh, k_sh;
-    __shared__ unsigned long long base_sh;
+    __shared__ int last_sh, k_sh;
 
     cluster_arrive_relaxed();  // peers must be running before any distributed shared memory write
-    const Smem sm = carve(dyn_smem, p.chunk4);
+    griddep_launch_dependents();
+    float4* sT = reinterpret_cast<float4*>(dyn_smem);
+    float4* sD = sT + p.chunk4;
     const int v4 = (V + 3) / 4;
     const int f0 = c * p.chunk4;
     const int n4 = max(0, min(v4, f0 + p.chunk4) - f0);
+    const int w0 = warp * p.wr;  // this warp's range of the slice
+    const int nw = max(0, min(n4, w0 + p.wr) - w0);
+    const int Kw = (nw + 31) >> 5;
     const float* trow = p.target + (size_t)rt * V;
 
-    // ---- start the target slice's copy at once; the draft row needs the sequence lookup
-    if (tid == 0) {
-        mbar_init(&bar_t, 1);
-        mbar_init(&bar_d, 1);
+    if (lane == 0) {
+        mbar_init(&bar_t[warp], 1);
+        mbar_init(&bar_d[warp], 1);
         fence_mbar_init();
-        own_sh = make_float4(0.f, 0.f, 0.f, 0.f);
     }
-    if (VEC) fetch_slice<VEC>(sm.sT, trow, f0, n4, V, &bar_t, tid);
+    __syncwarp();
+    // inputs may be produced by the previous kernel on the stream: wait for it before any global access
+    griddep_wait();
+    fetch_range<VEC>(sT + w0, trow, f0 + w0, nw, V, &bar_t[warp], lane);  // the target row needs no lookup
     int s, d_begin, d_end;
     if (p.num_seqs == 1) {
         s = 0;
@@ -258,33 +285,29 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     const int i = rt - tstart;
     const bool has_draft = i < gamma;
     const bool use_draft = !GREEDY && has_draft;
-    const float* drow = p.draft + (size_t)(d_begin + i) * V;
-    if (use_draft) fetch_slice<VEC>(sm.sD, drow, f0, n4, V, &bar_d, tid);
-    if (!VEC) fetch_slice<VEC>(sm.sT, trow, f0, n4, V, &bar_t, tid);
+    if (use_draft) fetch_range<VEC>(sD + w0, p.draft + (size_t)(d_begin + i) * V, f0 + w0, nw, V, &bar_d[warp], lane);
     int xi = has_draft ? __ldg(p.tokens + d_begin + i) : -1;
-    __syncthreads();  // barriers initialised, scalar fills complete
     if (has_draft && (xi < 0 || xi >= V)) {
         if (c == 0 && tid == 0) raise_error(p.err, kErrDeviceArg);
         xi = -1;
     }
-    if (VEC && n4 > 0) {
-        bool ok = mbar_wait(&bar_t, 0, kWaitBudget);
-        if (use_draft) ok = mbar_wait(&bar_d, 0, kWaitBudget) && ok;
-        if (!ok) raise_error(p.err, kErrTimeout);
-    }
-    const int K = (n4 + kThreads - 1) / kThreads;  // slots per thread (the last may be partial)
-    const int nb = (K + 3) / 4;
+    // inputs of the final step, read ahead of it (any CTA may turn out to run it)
+    const int my_tok = tid < gamma ? __ldg(p.tokens + d_begin + tid) : -1;
+    const float my_ua = (!GREEDY && tid < gamma) ? __ldg(p.u_accept + d_begin + tid) : 0.f;
     const float c2 = p.c2;
+    bool writer = false;  // the thread that publishes this row's token and takes the ticket
+    int tok_out = 0;
 
     if (GREEDY) {
-        // ================= argmax of the target row
+        // ================= argmax of the target row (lowest index on ties)
+        wait_range<VEC>(&bar_t[warp], nw, p.err);
         float bv = -INFINITY;
         int bi = 0x7fffffff;
-        for (int k = 0; k < K; ++k) {
-            const int f = k * kThreads + tid;
-            if (f < n4) {
-                const float4 v = sm.sT[f];
-                const int x = (f0 + f) * 4;
+        for (int j = 0; j < Kw; ++j) {
+            const int f = j * 32 + lane;
+            if (f < nw) {
+                const float4 v = sT[w0 + f];
+                const int x = (f0 + w0 + f) * 4;
                 amax_merge(bv, bi, v.x, x + 0);
                 amax_merge(bv, bi, v.y, x + 1);
                 amax_merge(bv, bi, v.z, x + 2);
@@ -316,64 +339,28 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
             int ix = 0x7fffffff;
             for (int r = 0; r < CS; ++r) amax_merge(v, ix, peer_x[r].x, __float_as_int(peer_x[r].y));
             if (ix >= V) ix = 0;  // every entry -inf: lowest index
-            p.tok_ws[rt] = ix;
+            writer = true;
+            tok_out = ix;
             if (has_draft && p.accept_prob) p.accept_prob[d_begin + i] = (xi == ix) ? 1.f : 0.f;
         }
     } else {
-        // the drafted token's raw logits, read before pass 1 overwrites the slice
-        if (tid == 0 && xi >= 0 && xi / 4 >= f0 && xi / 4 < f0 + n4) {
-            const int f = xi / 4 - f0;
-            own_sh = make_float4(pick(sm.sT[f], xi & 3), use_draft ? pick(sm.sD[f], xi & 3) : 0.f, 1.f, 0.f);
+        // ================= pass 1: per lane, a reference maximum and the sum of the weights
+        const bool own_x = xi >= 0 && (xi >> 2) >= f0 && (xi >> 2) < f0 + n4;  // this CTA holds x_i
+        const bool own_xw = own_x && (xi >> 2) - f0 >= w0 && (xi >> 2) - f0 < w0 + nw;  // this warp
+        float own_t = 0.f, own_d = 0.f;
+        wait_range<VEC>(&bar_t[warp], nw, p.err);
+        if (own_xw && lane == 0) own_t = pick(sT[(xi >> 2) - f0], xi & 3);  // the raw logit, before weighing
+        __syncwarp();
+        const float2 wt = weigh_range(sT, w0, nw, Kw, lane, c2);
+        float2 wd = make_float2(-INFINITY, 0.f);
+        if (use_draft) {
+            wait_range<VEC>(&bar_d[warp], nw, p.err);
+            if (own_xw && lane == 0) own_d = pick(sD[(xi >> 2) - f0], xi & 3);
+            __syncwarp();
+            wd = weigh_range(sD, w0, nw, Kw, lane, c2);
         }
-        __syncthreads();
-        // ================= pass 1: online (scaled max, sum) per thread; weights stored in place
-        float mt = -INFINITY, st = 0.f, md = -INFINITY, sd = 0.f;
-        for (int b = 0; b < nb; ++b) {
-            float4 tv[4], dv[4];
-            float bt = -INFINITY, bd = -INFINITY;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int f = (4 * b + q) * kThreads + tid;
-                tv[q] = f < n4 ? sm.sT[f] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-                bt = fmaxf(bt, max4(tv[q]));
-                if (use_draft) {
-                    dv[q] = f < n4 ? sm.sD[f] : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-                    bd = fmaxf(bd, max4(dv[q]));
-                }
-            }
-            if (bt != -INFINITY) {
-                const float nm = fmaxf(mt, __fmul_rn(bt, c2));
-                st *= ex2d(mt, nm);
-                mt = nm;
-            }
-            sm.bmT[b * kThreads + tid] = mt;
-#pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int f = (4 * b + q) * kThreads + tid;
-                if (f < n4) {
-                    const float4 e = mt == -INFINITY ? make_float4(0.f, 0.f, 0.f, 0.f) : ex2_4(tv[q], c2, mt);
-                    st += sum4(e);
-                    sm.sT[f] = e;
-                }
-            }
-            if (use_draft) {
-                if (bd != -INFINITY) {
-                    const float nm = fmaxf(md, __fmul_rn(bd, c2));
-                    sd *= ex2d(md, nm);
-                    md = nm;
-                }
-                sm.bmD[b * kThreads + tid] = md;
-#pragma unroll
-                for (int q = 0; q < 4; ++q) {
-                    const int f = (4 * b + q) * kThreads + tid;
-                    if (f < n4) {
-                        const float4 e = md == -INFINITY ? make_float4(0.f, 0.f, 0.f, 0.f) : ex2_4(dv[q], c2, md);
-                        sd += sum4(e);
-                        sm.sD[f] = e;
-                    }
-                }
-            }
-        }
+        if (own_xw && lane == 0) own_sh = make_float4(own_t, own_d, 1.f, 0.f);
+        float mt = wt.x, st = wt.y, md = wd.x, sd = wd.y;
 #pragma unroll
         for (int o = 16; o; o >>= 1) {
             lse_merge(mt, st, __shfl_xor_sync(0xffffffffu, mt, o), __shfl_xor_sync(0xffffffffu, st, o));
@@ -389,7 +376,7 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
                 lse_merge(a.z, a.w, red4[w].z, red4[w].w);
             }
             *cluster.map_shared_rank(&peer_stat[c], tid) = a;
-            *cluster.map_shared_rank(&peer_x[c], tid) = own_sh;
+            *cluster.map_shared_rank(&peer_x[c], tid) = own_x ? own_sh : make_float4(0.f, 0.f, 0.f, 0.f);
         }
         cluster_sync_all();
         // ---- row statistics (same order in every CTA of the cluster)
@@ -416,45 +403,36 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
         // ================= pass 2: fixed-point segment sums of r and p, one multiply per entry
         const float izt = __fdiv_rn(1.f, Zt);
         const float izd = use_draft ? __fdiv_rn(1.f, Zd) : 0.f;
-        unsigned long long totr = 0, totp = 0;
-        for (int b = 0; b < nb; ++b) {
-            const float bmt = sm.bmT[b * kThreads + tid];
-            const float ft = bmt == -INFINITY ? 0.f : __fmul_rn(ex2(__fsub_rn(bmt, Mt)), izt);
-            float fd = 0.f;
-            if (use_draft) {
-                const float bmd = sm.bmD[b * kThreads + tid];
-                fd = bmd == -INFINITY ? 0.f : __fmul_rn(ex2(__fsub_rn(bmd, Md)), izd);
-            }
+        const float ft = wt.x == -INFINITY ? 0.f : __fmul_rn(ex2(__fsub_rn(wt.x, Mt)), izt);
+        const float fd = (use_draft && wd.x != -INFINITY) ? __fmul_rn(ex2(__fsub_rn(wd.x, Md)), izd) : 0.f;
+        float v[2 * kMaxSeg];  // r then p of the lane's entries of each segment
 #pragma unroll
-            for (int q = 0; q < 4; ++q) {
-                const int k = 4 * b + q;
-                if (k < K) {  // warp-uniform
-                    const int f = k * kThreads + tid;
-                    float sp = 0.f, sr = 0.f;
-                    if (f < n4) {
-                        const float4 pv = mul4(sm.sT[f], ft);
-                        sp = sum4(pv);
-                        if (use_draft) sr = sum4(resid4(pv, mul4(sm.sD[f], fd)));
-                    }
-                    sp = warp_sum(sp);
-                    sr = warp_sum(sr);
-                    if (lane == 0) {  // one fixed-point conversion per 128-entry segment
-                        const unsigned long long fr = to_fix(sr), fp = to_fix(sp);
-                        sm.segR[k * kWarps + warp] = fr;
-                        sm.segP[k * kWarps + warp] = fp;
-                        totr += fr;
-                        totp += fp;
-                    }
-                }
+        for (int j = 0; j < kMaxSeg; ++j) {
+            const int f = j * 32 + lane;
+            float sr = 0.f, sp = 0.f;
+            if (j < Kw && f < nw) {
+                const float4 pv = mul4(sT[w0 + f], ft);
+                sp = sum4(pv);
+                if (use_draft) sr = sum4(resid4(pv, mul4(sD[w0 + f], fd)));
             }
+            v[j] = sr;
+            v[kMaxSeg + j] = sp;
         }
-        if (lane == 0) tot_sh[warp] = make_ulonglong2(totr, totp);
+        // lane j < 16 gets the r-sum of segment j, lane 16 + j its p-sum; one conversion each
+        const unsigned long long fx = to_fix(reduce_scatter32(v, lane));
+        if (lane < kMaxSeg) segR[warp * kMaxSeg + lane] = fx;
+        else segP[warp * kMaxSeg + lane - kMaxSeg] = fx;
+        unsigned long long rtot = fx;
+#pragma unroll
+        for (int o = kMaxSeg / 2; o; o >>= 1) rtot += __shfl_xor_sync(0xffffffffu, rtot, o);
+        if (lane == 0) wtot[warp].x = rtot;
+        if (lane == kMaxSeg) wtot[warp].y = rtot;
         __syncthreads();
         if (tid < CS) {
-            ulonglong2 t = tot_sh[0];
+            ulonglong2 t = wtot[0];
             for (int w = 1; w < kWarps; ++w) {
-                t.x += tot_sh[w].x;
-                t.y += tot_sh[w].y;
+                t.x += wtot[w].x;
+                t.y += wtot[w].y;
             }
             *cluster.map_shared_rank(&peer_tot[c], tid) = t;
         }
@@ -482,62 +460,57 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
             if (c != 0) return;
             if (tid == 0) {
                 raise_error(p.err, kErrDeviceArg);
-                p.tok_ws[rt] = 0;
+                writer = true;
+                tok_out = 0;
             }
         } else {
             if (!(below <= thr && thr < below + mine)) return;  // the crossing is in another slice
-            // ---- segment of this slice (block scan of the segment sums, exact)
-            const unsigned long long* seg = use_r ? sm.segR : sm.segP;
-            const int nseg = K * kWarps;
-            const int per = (nseg + kThreads - 1) / kThreads;
-            const int sb = min(nseg, tid * per), se = min(nseg, sb + per);
-            unsigned long long loc = 0;
-            for (int q = sb; q < se; ++q) loc += seg[q];
-            const unsigned long long incl = warp_incl_scan(loc, lane);
-            if (lane == 31) tot_sh[warp].x = incl;
-            if (tid == 0) sel_sh = 0x7fffffff;
-            __syncthreads();
-            unsigned long long cum = below + incl - loc;
-            for (int w = 0; w < warp; ++w) cum += tot_sh[w].x;
-            for (int q = sb; q < se; ++q) {
-                if (seg[q] > 0 && cum <= thr && thr < cum + seg[q]) {
-                    sel_sh = q;  // exact integer sums: exactly one segment holds the threshold
-                    base_sh = cum;
-                    break;
+            // ---- the warp range, then the segment holding the threshold (exact integer sums:
+            // exactly one of each holds it)
+            unsigned long long cum = below, wbase = 0;
+            int wsel = -1;
+            for (int q = 0; q < kWarps; ++q) {
+                const unsigned long long x = use_r ? wtot[q].x : wtot[q].y;
+                if (wsel < 0 && x > 0 && cum <= thr && thr < cum + x) {
+                    wsel = q;
+                    wbase = cum;
                 }
-                cum += seg[q];
+                cum += x;
             }
-            __syncthreads();
-            const int sel = sel_sh;
-            // ---- entry of the segment (warp 0): the stored weights of its owner thread
-            if (warp == 0) {
-                if (sel >= nseg) {  // unreachable with exact sums: report, emit the slice's first entry
+            if (wsel < 0) {  // unreachable with exact sums: report, emit the slice's first entry
+                if (tid == 0) {
+                    raise_error(p.err, kErrDeviceArg);
+                    writer = true;
+                    tok_out = f0 * 4;
+                }
+            } else if (warp == wsel) {
+                const unsigned long long sg =
+                    lane < kMaxSeg ? (use_r ? segR : segP)[warp * kMaxSeg + lane] : 0ull;
+                const unsigned long long incl = warp_incl_scan(sg, lane);
+                const unsigned long long sb = wbase + incl - sg;
+                const unsigned hm = __ballot_sync(0xffffffffu, sg > 0 && sb <= thr && thr < sb + sg);
+                if (hm == 0u) {  // unreachable with exact sums
                     if (lane == 0) {
                         raise_error(p.err, kErrDeviceArg);
-                        p.tok_ws[rt] = f0 * 4;
+                        writer = true;
+                        tok_out = (f0 + w0) * 4;
                     }
                 } else {
-                    const int k = sel / kWarps, w = sel % kWarps;
-                    const int owner = w * 32 + lane;  // thread whose slot k holds this lane's entries
-                    const int f = k * kThreads + owner;
-                    const int b = k / 4;
+                    const int j = __ffs(hm) - 1;
+                    const unsigned long long base = __shfl_sync(0xffffffffu, sb, j);
+                    // ---- entry of segment j: this lane's slot, weighed exactly as in pass 2
+                    const int f = j * 32 + lane;
                     float4 wv = make_float4(0.f, 0.f, 0.f, 0.f);
-                    if (f < n4) {
-                        const float bmt = sm.bmT[b * kThreads + owner];
-                        const float ft = bmt == -INFINITY ? 0.f : __fmul_rn(ex2(__fsub_rn(bmt, Mt)), izt);
-                        wv = mul4(sm.sT[f], ft);
-                        if (use_r) {
-                            const float bmd = sm.bmD[b * kThreads + owner];
-                            const float fd = bmd == -INFINITY ? 0.f : __fmul_rn(ex2(__fsub_rn(bmd, Md)), izd);
-                            wv = resid4(wv, mul4(sm.sD[f], fd));
-                        }
+                    if (f < nw) {
+                        wv = mul4(sT[w0 + f], ft);
+                        if (use_r) wv = resid4(wv, mul4(sD[w0 + f], fd));
                     }
                     const float wa[4] = {wv.x, wv.y, wv.z, wv.w};
                     // offset of the threshold inside the segment, back in probability units
-                    const float off = __ull2float_rn(thr - base_sh) * 2.220446049250313e-16f;
+                    const float off = __ull2float_rn(thr - base) * 2.220446049250313e-16f;
                     const float lsum = (wa[0] + wa[1]) + (wa[2] + wa[3]);
                     float run = warp_incl_scan_f(lsum, lane) - lsum;
-                    const int x0 = (f0 + f) * 4;
+                    const int x0 = (f0 + w0 + f) * 4;
                     int hit = -1, lastpos = -1;
 #pragma unroll
                     for (int e = 0; e < 4; ++e) {
@@ -551,14 +524,18 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
                     // then the segment's last entry with positive weight
                     const int first = any ? __shfl_sync(0xffffffffu, hit, __ffs(any) - 1)
                                           : (pos ? __shfl_sync(0xffffffffu, lastpos, 31 - __clz(pos)) : x0);
-                    if (lane == 0) p.tok_ws[rt] = first;
+                    if (lane == 0) {
+                        writer = true;
+                        tok_out = first;
+                    }
                 }
             }
         }
     }
 
-    // ---- this CTA wrote the row's token: take a ticket; the last row of the sequence resolves it
-    if (tid == 0) {
+    // ---- publish the row's token and take a ticket; the last row of the sequence resolves it
+    if (writer) {
+        p.tok_ws[rt] = tok_out;
         __threadfence();
         const int old = atomicAdd(p.tickets + s, 1);
         last_sh = (old == gamma);
@@ -568,23 +545,28 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     if (!last_sh) return;
     __threadfence();
     if (tid == 0) p.tickets[s] = 0;  // ready for the next call
-    int my_tok = -1;  // drafted token of position tid (first iteration)
+    // one round of loads: the rows' tokens and ratios, then the first rejection k
     for (int ii = tid; ii <= gamma; ii += kThreads) {
-        const int tok = ii < gamma ? __ldg(p.tokens + d_begin + ii) : -1;
+        const int tw = __ldcg(p.tok_ws + tstart + ii);
         bool rej = false;
         if (ii < gamma) {
-            rej = GREEDY ? (tok != __ldcg(p.tok_ws + tstart + ii))
-                         : !(__ldg(p.u_accept + d_begin + ii) < __ldcg(p.a_ws + d_begin + ii));
+            const int tok = ii == tid ? my_tok : __ldg(p.tokens + d_begin + ii);
+            if (GREEDY) {
+                rej = tok != tw;
+            } else {
+                const float ua = ii == tid ? my_ua : __ldg(p.u_accept + d_begin + ii);
+                rej = !(ua < __ldcg(p.a_ws + d_begin + ii));
+            }
         }
         if (rej) atomicMin(&k_sh, ii);
-        if (ii == tid) my_tok = tok;
+        if (ii <= kMaxSmemSeqs) cu_sh[ii] = tw;
     }
     __syncthreads();
     const int k = k_sh;
-    const int token = __ldcg(p.tok_ws + tstart + k);
+    const int token = k <= kMaxSmemSeqs ? cu_sh[k] : __ldcg(p.tok_ws + tstart + k);
     for (int ii = tid; ii <= gamma; ii += kThreads) {
         int v;
-        if (ii < k) v = (ii < kThreads) ? my_tok : __ldg(p.tokens + d_begin + ii);
+        if (ii < k) v = (ii == tid) ? my_tok : __ldg(p.tokens + d_begin + ii);
         else if (ii == k) v = token;
         else v = -1;
         p.out_tokens[tstart + ii] = v;
@@ -592,7 +574,7 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     if (tid == 0) p.n_accepted[s] = k;
 }
 
-constexpr size_t kSmemBudget = 108 * 1024;  // dynamic shared memory per CTA: two CTAs per SM
+constexpr size_t kSmemBudget = 104 * 1024;  // dynamic shared memory per CTA: two CTAs per SM with the static part
 
 struct Variant {
     int max_active[kMaxCS + 1];
@@ -658,6 +640,8 @@ int launch_variant(const AccParams& prm0, int rows, const DeviceInfo& dev, cudaS
     }
     AccParams p = prm0;
     p.chunk4 = (v4 + cs - 1) / cs;
+    p.wr = warp_range(p.chunk4);
+    if (!GREEDY && p.wr > kMaxSeg * 32) return BP_ERR_UNSUPPORTED;  // excluded by the shared-memory budget
     const size_t smem = smem_bytes(p.chunk4, GREEDY);
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[1];
@@ -669,6 +653,9 @@ int launch_variant(const AccParams& prm0, int rows, const DeviceInfo& dev, cudaS
     attr[0].val.clusterDim.x = cs;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    // No programmatic (early) launch here: clusters placed while the previous kernel still holds
+    // SMs land in whatever is left of each GPC and a wide cluster then needs a second wave (a
+    // measured 3 us loss after block attention).  The kernel still releases its own dependents early.
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     return cudaLaunchKernelEx(&cfg, accept_kernel<GREEDY, VEC>, p) == cudaSuccess ? BP_OK : BP_ERR_CUDA;
@@ -712,6 +699,7 @@ int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t strea
     p.out_tokens = a.out_tokens;
     p.accept_prob = a.accept_prob;
     p.chunk4 = 0;
+    p.wr = 0;
     p.err = a.err_word;
     const bool vec = (a.vocab % 4 == 0) && (reinterpret_cast<uintptr_t>(a.target) % 16 == 0) &&
                      (greedy || reinterpret_cast<uintptr_t>(a.draft) % 16 == 0);

@@ -99,6 +99,8 @@ __global__ void __launch_bounds__(kThreads, 1)
         prefetch_tensormap(&kmap);
         prefetch_tensormap(&vmap);
     }
+    griddep_launch_dependents();
+    if (p.num_seqs > 1) griddep_wait();  // the sequence offsets are read from global memory
     const uint32_t CS = cluster_size();
     const uint32_t crank = cluster_rank();
     const int unit_rank = blockIdx.x / CS;
@@ -138,7 +140,10 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int rows = B * G;
     const int row0 = mt * kM;
     const int m_valid = min(kM, rows - row0);
-    if (m_valid <= 0) return;  // uniform across the cluster: every CTA decodes the same unit
+    if (m_valid <= 0) {  // uniform across the cluster: every CTA decodes the same unit
+        griddep_wait();  // this grid must not complete before the one it depends on
+        return;
+    }
 
     const int tiles = (n + kTileN - 1) / kTileN;
     const int t_begin = (int)((long long)crank * tiles / CS);
@@ -148,6 +153,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     // ---- Q tile -> shared memory, SWIZZLE_128B K-major (two 64-column halves).  With a TMA map the
     // 128/G block positions x G heads box lands exactly as rows r = i*G + j; otherwise plain loads.
     if (!p.q_tma) {
+        griddep_wait();
         for (int idx = tid; idx < kM * 16; idx += kThreads) {
             const int r = idx >> 4, ch = idx & 15;
             uint4 val = make_uint4(0, 0, 0, 0);
@@ -187,16 +193,6 @@ __global__ void __launch_bounds__(kThreads, 1)
         mbar_init(&bar_o_done, 1);
         mbar_init(&bar_q_full, 1);
         fence_mbar_init();
-        // the producer (this thread) starts the Q load and fills the K/V ring right away
-        if (nt > 0) {
-            if (p.q_tma) {
-                mbar_arrive_expect_tx(&bar_q_full, kQBytes);
-                const int qrow = q0 + row0 / G;
-                tma_load_3d(sQ, &qmap, &bar_q_full, 0, h * G, qrow);
-                tma_load_3d(sQ + kHalf, &qmap, &bar_q_full, 64, h * G, qrow);
-            }
-            for (int j = 0; j < min(nt, kStages); ++j) issue_kv(j);
-        }
     }
     if (warp == 1) {  // tensor memory is allocated (and released) by warp 1, in parallel
         tmem_alloc(&tmem_base_sh, kTmemCols);
@@ -206,6 +202,17 @@ __global__ void __launch_bounds__(kThreads, 1)
     __syncthreads();
     tc_fence_after();
     const uint32_t tmem = tmem_base_sh;
+    // inputs may be produced by the previous kernel on the stream: wait for it before any global access
+    griddep_wait();
+    if (tid == 0 && nt > 0) {  // the producer starts the Q load and fills the K/V ring
+        if (p.q_tma) {
+            mbar_arrive_expect_tx(&bar_q_full, kQBytes);
+            const int qrow = q0 + row0 / G;
+            tma_load_3d(sQ, &qmap, &bar_q_full, 0, h * G, qrow);
+            tma_load_3d(sQ + kHalf, &qmap, &bar_q_full, 64, h * G, qrow);
+        }
+        for (int j = 0; j < min(nt, kStages); ++j) issue_kv(j);
+    }
 
     if (warp == 0) {
         // ================= TMA producer
@@ -499,6 +506,8 @@ __global__ void __launch_bounds__(128) attn_f32_simt_kernel(const float* __restr
                                                             int total_q, int hq, int hkv, int D, int causal,
                                                             float scale) {
     __shared__ float qs[4][kF32MaxD];
+    griddep_launch_dependents();
+    griddep_wait();
     const int wib = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const long long row = (long long)blockIdx.x * 4 + wib;
     if (row >= (long long)total_q * hq) return;
@@ -660,7 +669,7 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     }
 
     cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[1];
+    cudaLaunchAttribute attr[2];
     cfg.gridDim = dim3((unsigned)(units * cs), 1, 1);
     cfg.blockDim = dim3(kThreads, 1, 1);
     cfg.dynamicSmemBytes = kDynSmem;
@@ -669,8 +678,10 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     attr[0].val.clusterDim.x = cs;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = 2;
     if (cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel, qmap, kmap, vmap, p) != cudaSuccess) return BP_ERR_CUDA;
     return BP_OK;
 }
@@ -679,12 +690,20 @@ int launch_attention_f32(const AttentionArgs& a, cudaStream_t stream) {
     if (a.head_dim > kF32MaxD) return BP_ERR_UNSUPPORTED;
     const long long rows = (long long)a.total_q * a.num_q_heads;
     if (rows == 0) return BP_OK;
-    const unsigned blocks = (unsigned)((rows + 3) / 4);
-    attn_f32_simt_kernel<<<blocks, 128, 0, stream>>>(
-        static_cast<const float*>(a.q), static_cast<const float*>(a.k), static_cast<const float*>(a.v),
-        static_cast<float*>(a.o), a.lse, a.cu_q, a.cu_kv, a.num_seqs, a.total_q, a.num_q_heads, a.num_kv_heads,
-        a.head_dim, a.mask == BP_MASK_CAUSAL_BLOCK, a.scale);
-    return cudaGetLastError() == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.gridDim = dim3((unsigned)((rows + 3) / 4), 1, 1);
+    cfg.blockDim = dim3(128, 1, 1);
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    const cudaError_t e = cudaLaunchKernelEx(
+        &cfg, attn_f32_simt_kernel, static_cast<const float*>(a.q), static_cast<const float*>(a.k),
+        static_cast<const float*>(a.v), static_cast<float*>(a.o), a.lse, a.cu_q, a.cu_kv, a.num_seqs, a.total_q,
+        a.num_q_heads, a.num_kv_heads, a.head_dim, (int)(a.mask == BP_MASK_CAUSAL_BLOCK), a.scale);
+    return e == cudaSuccess ? BP_OK : BP_ERR_CUDA;
 }
 
 }  // namespace bp

@@ -9,6 +9,7 @@
 #include <cuda_bf16.h>
 
 #include "common.cuh"
+#include "ptx_sm103.cuh"
 
 namespace bp {
 namespace {
@@ -51,6 +52,8 @@ __global__ void __launch_bounds__(kThreads1) policy_hidden_kernel(const T* __res
     extern __shared__ uint8_t smem_raw[];
     T* xs = reinterpret_cast<T*>(smem_raw);  // [ng][d_in]
     const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    griddep_launch_dependents();
+    griddep_wait();
     // stage the pooled rows of this request group (16-byte copies)
     const int per_row = d_in * (int)sizeof(T) / 16;
     for (int idx = tid; idx < ng * per_row; idx += kThreads1) {
@@ -102,6 +105,8 @@ __global__ void __launch_bounds__(256) policy_out_kernel(const float* __restrict
     __shared__ float red[8];
     __shared__ float logits[64];
     const int n = blockIdx.x, tid = threadIdx.x;
+    griddep_launch_dependents();
+    griddep_wait();
     const float* h = hbuf + (size_t)n * hidden;
     for (int c = 0; c < num_cand; ++c) {
         float acc = 0.f;
@@ -148,16 +153,30 @@ int run(const PolicyArgs& a, cudaStream_t stream) {
             return BP_ERR_CUDA;
         configured = dev;
     }
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.stream = stream;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
     for (int n0 = 0; n0 < a.num_reqs; n0 += group) {
         const int ng = a.num_reqs - n0 < group ? a.num_reqs - n0 : group;
-        const size_t smem = (size_t)ng * a.d_in * sizeof(T);
-        policy_hidden_kernel<T><<<blocks, kThreads1, smem, stream>>>(
-            static_cast<const T*>(a.feats), a.row_stride, a.row_index, n0, ng, a.d_in, static_cast<const T*>(a.w1),
-            a.b1, a.hidden, hbuf);
+        cfg.gridDim = dim3(blocks, 1, 1);
+        cfg.blockDim = dim3(kThreads1, 1, 1);
+        cfg.dynamicSmemBytes = (size_t)ng * a.d_in * sizeof(T);
+        if (cudaLaunchKernelEx(&cfg, policy_hidden_kernel<T>, static_cast<const T*>(a.feats), a.row_stride,
+                               a.row_index, n0, ng, a.d_in, static_cast<const T*>(a.w1), a.b1, a.hidden,
+                               hbuf) != cudaSuccess)
+            return BP_ERR_CUDA;
     }
-    policy_out_kernel<T><<<a.num_reqs, 256, 0, stream>>>(hbuf, a.hidden, static_cast<const T*>(a.w2), a.b2,
-                                                         a.num_cand, a.candidates, a.logits_out, a.block_size_out);
-    return cudaGetLastError() == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+    cfg.gridDim = dim3((unsigned)a.num_reqs, 1, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.dynamicSmemBytes = 0;
+    if (cudaLaunchKernelEx(&cfg, policy_out_kernel<T>, (const float*)hbuf, a.hidden, static_cast<const T*>(a.w2), a.b2,
+                           a.num_cand, a.candidates, a.logits_out, a.block_size_out) != cudaSuccess)
+        return BP_ERR_CUDA;
+    return BP_OK;
 }
 
 }  // namespace

@@ -184,3 +184,16 @@ __device__ __forceinline__ uint32_t pack_bf16x2(float lo, float hi) {
 }
 
 }  // namespace bp
+
+namespace bp {
+// ---------------------------------------------------------------- programmatic dependent launch
+// Kernels are launched with programmatic stream serialization: a kernel may begin (and run its
+// prologue) while its predecessor on the stream finishes.  griddep_wait() blocks until every
+// prerequisite grid has completed and its memory is visible, so it precedes the first global
+// access of every kernel; griddep_launch_dependents() lets the next kernel begin once every CTA
+// of this grid has started.  Without the launch attribute both are no-ops.
+__device__ __forceinline__ void griddep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void griddep_launch_dependents() {
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+}
+}  // namespace bp
