@@ -110,6 +110,12 @@ __device__ __forceinline__ void amax_merge(float& v, int& i, float v2, int i2) {
     }
 }
 
+__device__ __forceinline__ int atomic_add_acq_rel(int* addr, int v) {
+    int old;
+    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(addr), "r"(v) : "memory");
+    return old;
+}
+
 __device__ __forceinline__ void cluster_arrive_relaxed() {
     asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
 }
@@ -231,6 +237,7 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     __shared__ unsigned long long segR[kWarps * kMaxSeg], segP[kWarps * kMaxSeg];
     __shared__ ulonglong2 wtot[kWarps];      // range totals of r and p (fixed point)
     __shared__ float4 own_sh;
+    __shared__ float4 stat_sh;  // (scaled max t, sum t, scaled max d, sum d) of the row
     __shared__ int last_sh, k_sh;
 
     cluster_arrive_relaxed();  // peers must be running before any distributed shared memory write
@@ -294,6 +301,7 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     // inputs of the final step, read ahead of it (any CTA may turn out to run it)
     const int my_tok = tid < gamma ? __ldg(p.tokens + d_begin + tid) : -1;
     const float my_ua = (!GREEDY && tid < gamma) ? __ldg(p.u_accept + d_begin + tid) : 0.f;
+    const float u_s = GREEDY ? 0.f : __ldg(p.u_sample + s);
     const float c2 = p.c2;
     bool writer = false;  // the thread that publishes this row's token and takes the ticket
     int tok_out = 0;
@@ -360,11 +368,18 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
             wd = weigh_range(sD, w0, nw, Kw, lane, c2);
         }
         if (own_xw && lane == 0) own_sh = make_float4(own_t, own_d, 1.f, 0.f);
-        float mt = wt.x, st = wt.y, md = wd.x, sd = wd.y;
+        // warp statistics: the warp maximum, then every lane's sum rescaled to it
+        float mt = wt.x, md = wd.x;
 #pragma unroll
         for (int o = 16; o; o >>= 1) {
-            lse_merge(mt, st, __shfl_xor_sync(0xffffffffu, mt, o), __shfl_xor_sync(0xffffffffu, st, o));
-            lse_merge(md, sd, __shfl_xor_sync(0xffffffffu, md, o), __shfl_xor_sync(0xffffffffu, sd, o));
+            mt = fmaxf(mt, __shfl_xor_sync(0xffffffffu, mt, o));
+            md = fmaxf(md, __shfl_xor_sync(0xffffffffu, md, o));
+        }
+        float st = wt.y * ex2d(wt.x, mt), sd = wd.y * ex2d(wd.x, md);
+#pragma unroll
+        for (int o = 16; o; o >>= 1) {
+            st += __shfl_xor_sync(0xffffffffu, st, o);
+            sd += __shfl_xor_sync(0xffffffffu, sd, o);
         }
         if (lane == 0) red4[warp] = make_float4(mt, st, md, sd);
         __syncthreads();
@@ -379,16 +394,27 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
             *cluster.map_shared_rank(&peer_x[c], tid) = own_x ? own_sh : make_float4(0.f, 0.f, 0.f, 0.f);
         }
         cluster_sync_all();
-        // ---- row statistics (same order in every CTA of the cluster)
-        float Mt = -INFINITY, Zt = 0.f, Md = -INFINITY, Zd = 0.f, tx = -INFINITY, dx = -INFINITY;
-        for (int r = 0; r < CS; ++r) {
-            lse_merge(Mt, Zt, peer_stat[r].x, peer_stat[r].y);
-            lse_merge(Md, Zd, peer_stat[r].z, peer_stat[r].w);
-            if (peer_x[r].z != 0.f) {
-                tx = peer_x[r].x;
-                dx = peer_x[r].y;
+        // ---- row statistics: warp 0 merges the CS slice statistics along a butterfly (the merge is
+        // commutative bit for bit, so every lane and every CTA of the cluster gets the same values)
+        if (warp == 0) {
+            float4 a = lane < CS ? peer_stat[lane] : make_float4(-INFINITY, 0.f, -INFINITY, 0.f);
+#pragma unroll
+            for (int o = 1; o < 32; o <<= 1) {
+                const float4 b = make_float4(__shfl_xor_sync(0xffffffffu, a.x, o), __shfl_xor_sync(0xffffffffu, a.y, o),
+                                             __shfl_xor_sync(0xffffffffu, a.z, o), __shfl_xor_sync(0xffffffffu, a.w, o));
+                lse_merge(a.x, a.y, b.x, b.y);
+                lse_merge(a.z, a.w, b.z, b.w);
+            }
+            const unsigned holder = __ballot_sync(0xffffffffu, lane < CS && peer_x[lane].z != 0.f);
+            if (lane == 0) {
+                stat_sh = a;
+                const float4 x = holder ? peer_x[__ffs(holder) - 1] : make_float4(-INFINITY, -INFINITY, 0.f, 0.f);
+                own_sh = x;  // (t[x_i], d[x_i]) of the row, read below
             }
         }
+        __syncthreads();
+        const float Mt = stat_sh.x, Zt = stat_sh.y, Md = stat_sh.z, Zd = stat_sh.w;
+        const float tx = own_sh.x, dx = own_sh.y;
         if (c == 0 && tid == 0 && has_draft) {
             // a = min(1, p(x)/q(x)) evaluated in the log domain
             float a;
@@ -451,7 +477,7 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
         const unsigned long long total = use_r ? R : P;
         const unsigned long long mine = use_r ? peer_tot[c].x : peer_tot[c].y;
         const unsigned long long below = use_r ? Rb : Pb;
-        float u = __ldg(p.u_sample + s);
+        float u = u_s;
         if (!(u >= 0.f)) u = 0.f;
         u = fminf(u, 0.99999994f);  // u in [0, 1): the crossing always exists
         const unsigned long long thr = __umul64hi(__float2ull_rn(u * 18446744073709551616.f), total);
@@ -536,14 +562,14 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
     // ---- publish the row's token and take a ticket; the last row of the sequence resolves it
     if (writer) {
         p.tok_ws[rt] = tok_out;
-        __threadfence();
-        const int old = atomicAdd(p.tickets + s, 1);
+        // release: this row's token (and, through the cluster barriers, a_i) before the ticket;
+        // acquire: the last ticket sees every other row's results
+        const int old = atomic_add_acq_rel(p.tickets + s, 1);
         last_sh = (old == gamma);
         k_sh = gamma;
     }
     __syncthreads();
     if (!last_sh) return;
-    __threadfence();
     if (tid == 0) p.tickets[s] = 0;  // ready for the next call
     // one round of loads: the rows' tokens and ratios, then the first rejection k
     for (int ii = tid; ii <= gamma; ii += kThreads) {
