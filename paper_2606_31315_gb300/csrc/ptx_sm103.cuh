@@ -197,3 +197,21 @@ __device__ __forceinline__ void griddep_launch_dependents() {
     asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
 }
 }  // namespace bp
+
+namespace bp {
+// ---------------------------------------------------------------- thread-block clusters
+// Split cluster barrier: every thread of every CTA of the cluster arrives, then waits.  The
+// release/acquire forms order shared-memory writes to peers (distributed shared memory) before
+// the peers' reads after the barrier.
+__device__ __forceinline__ void cluster_arrive_relaxed() {
+    asm volatile("barrier.cluster.arrive.relaxed.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_arrive_release() {
+    asm volatile("barrier.cluster.arrive.release.aligned;" ::: "memory");
+}
+__device__ __forceinline__ void cluster_wait() { asm volatile("barrier.cluster.wait.acquire.aligned;" ::: "memory"); }
+__device__ __forceinline__ void cluster_sync_all() {
+    cluster_arrive_release();
+    cluster_wait();
+}
+}  // namespace bp
