@@ -1,15 +1,29 @@
 // Block-size policy head (Sections 2.3-2.4 of the BlockPilot paper): once per request,
 //   h = max(0, W1 x + b1),  o = W2 h + b2,  block size = candidates[argmax o].
 //
-// Kernel 1 streams W1 exactly once for a group of up to 32 requests: the pooled feature
-// rows of the group are staged in shared memory (gathered by row_index), every warp owns
-// hidden rows and reads them with 16-byte loads, fp32 accumulation, warp-shuffle
-// reduction, bias and ReLU fused into the store of h.  Kernel 2 (one CTA per request)
-// applies the small output layer and takes the argmax with the lowest index on ties.
+// bf16 weights -- tensor cores (sm_103a), one launch:
+//   * W1 [hidden x d_in] is cut into 128-row tiles; a thread-block cluster of KS CTAs splits one
+//     tile's d_in into 64-column swizzle atoms.  Each CTA brings its W1 atoms in with TMA
+//     (SWIZZLE_128B), gathers the requests' pooled rows x (row_index) into the matching
+//     K-major layout, and one thread issues M=128 x N=requests tcgen05 MMAs (bf16 in, fp32
+//     accumulated in tensor memory): W1 is read from HBM exactly once for up to 64 requests.
+//   * The KS partial tiles are summed through distributed shared memory; each CTA takes a
+//     share of the rows, adds b1 and applies ReLU, and folds its rows of h straight into the
+//     output layer (W2 columns of those rows), so h never goes to global memory.
+//   * The cluster's output-layer partials go to the workspace; the last tile to finish (an
+//     atomic ticket, no waiting) adds them in tile order with b2 and takes the argmax (lowest
+//     index on ties).  Every sum runs in a fixed order: the result is deterministic.
+// fp32 weights (and bf16 shapes outside the tensor-core limits) -- CUDA cores:
+//   kernel 1 streams W1 once for a group of up to 32 requests (rows staged in shared memory,
+//   a warp per hidden row, fp32 accumulation, bias and ReLU fused into the store of h);
+//   kernel 2 (one CTA per request) applies the output layer and takes the argmax.
+#include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
 #include "common.cuh"
 #include "ptx_sm103.cuh"
+
+namespace cg = cooperative_groups;
 
 namespace bp {
 namespace {
@@ -132,6 +146,309 @@ __global__ void __launch_bounds__(256) policy_out_kernel(const float* __restrict
     }
 }
 
+// ---------------------------------------------------------------- tensor-core path (bf16)
+constexpr int kTcM = 128;          // hidden rows per tile: the MMA M
+constexpr int kTcMaxN = 64;        // requests per group: the MMA N (padded to a multiple of 16)
+constexpr int kTcAtom = 64;        // d_in columns per 128-byte swizzle atom
+constexpr int kTcAtomBytes = kTcM * kTcAtom * 2;  // 16 KB of W1 per atom
+constexpr int kTcMaxAtoms = 8;     // atoms per CTA
+constexpr int kTcMaxKS = 8;        // CTAs per cluster
+constexpr int kTcThreads = 128;    // thread t = tile row t = TMEM lane t
+constexpr uint32_t kTcTmemCols = 64;
+constexpr int kTcMaxSmem = 200 * 1024;
+
+struct PolicyTcParams {
+    const __nv_bfloat16* feats;
+    int64_t row_stride;
+    const int32_t* row_index;
+    int num_reqs, d_in, hidden, num_cand;
+    int atoms_total, atoms_per_cta, tiles, npad;
+    int w_bytes, x_bytes, h_bytes;  // dynamic shared-memory regions
+    const float* b1;
+    const __nv_bfloat16* w2;
+    const float* b2;
+    const int32_t* candidates;
+    float* logits_out;
+    int32_t* block_size_out;
+    float* part;    // [groups][tiles][kTcMaxN][num_cand] output-layer partials of each tile
+    int* counters;  // [groups] tickets, zero between calls
+    unsigned int* err;
+};
+
+__device__ __forceinline__ int atomic_add_acq_rel_gpu(int* addr, int v) {
+    int old;
+    asm volatile("atom.add.acq_rel.gpu.s32 %0, [%1], %2;" : "=r"(old) : "l"(addr), "r"(v) : "memory");
+    return old;
+}
+
+__global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_constant__ CUtensorMap w1map,
+                                                              const PolicyTcParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sW = base;                                         // W1 atoms, later the partial tile
+    uint8_t* sX = base + p.w_bytes;                             // x atoms
+    float* hs = reinterpret_cast<float*>(sX + p.x_bytes);       // h of the owned rows [rows][npad]
+    float* op = reinterpret_cast<float*>(sX + p.x_bytes + p.h_bytes);  // output-layer partial [n][c]
+    __shared__ uint64_t bar_w[kTcMaxAtoms], bar_mma;
+    __shared__ uint32_t tmem_sh;
+    __shared__ int last_sh;
+
+    cg::cluster_group cluster = cg::this_cluster();
+    const int KS = (int)cluster.num_blocks();
+    const int rank = (int)cluster.block_rank();
+    const int tid = threadIdx.x, warp = tid >> 5;
+    const int tile = blockIdx.x / KS, g = blockIdx.y;
+    const int m0 = tile * kTcM, n0 = g * kTcMaxN;
+    const int ng = min(kTcMaxN, p.num_reqs - n0);
+    const int npad = p.npad;
+    const int a0 = rank * p.atoms_per_cta;
+    const int na = max(0, min(p.atoms_total, a0 + p.atoms_per_cta) - a0);
+    const int C = p.num_cand;
+
+    cluster_arrive_relaxed();  // peers must be running before any distributed shared memory access
+    if (tid == 0) {
+        prefetch_tensormap(&w1map);
+        for (int a = 0; a < na; ++a) mbar_init(&bar_w[a], 1);
+        mbar_init(&bar_mma, 1);
+        fence_mbar_init();
+    }
+    if (warp == 0) {
+        tmem_alloc(&tmem_sh, kTcTmemCols);
+        tmem_relinquish();
+    }
+    griddep_launch_dependents();
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_sh;
+    griddep_wait();  // inputs may come from the previous kernel on the stream
+    if (tid == 0)
+        for (int a = 0; a < na; ++a) {
+            mbar_arrive_expect_tx(&bar_w[a], kTcAtomBytes);
+            tma_load_2d(sW + a * kTcAtomBytes, &w1map, &bar_w[a], (a0 + a) * kTcAtom, m0);
+        }
+    // x of the group, K-major SWIZZLE_128B: atom a holds rows n of 128 bytes, 16-byte chunk c of
+    // row n stored at chunk c ^ (n & 7); rows past the group and columns past d_in are zero
+    for (int idx = tid; idx < npad * na * 8; idx += kTcThreads) {
+        const int n = idx / (na * 8), rem = idx % (na * 8);
+        const int a = rem >> 3, c = rem & 7;
+        const int k = (a0 + a) * kTcAtom + c * 8;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (n < ng && k < p.d_in) {
+            const long long row = p.row_index ? (long long)p.row_index[n0 + n] : (long long)(n0 + n);
+            v = *reinterpret_cast<const uint4*>(p.feats + row * p.row_stride + k);
+        }
+        *reinterpret_cast<uint4*>(sX + a * npad * 128 + n * 128 + ((c ^ (n & 7)) << 4)) = v;
+    }
+    fence_proxy_async_smem();  // the MMAs read x through the async proxy
+    __syncthreads();
+    if (tid == 0 && na > 0) {
+        const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
+        bool ok = true;
+        for (int a = 0; a < na && ok; ++a) {
+            if (!mbar_wait(&bar_w[a], 0, kWaitBudget)) {
+                ok = false;
+                break;
+            }
+            tc_fence_after();
+            const uint32_t wa = smem_addr(sW + a * kTcAtomBytes), xa = smem_addr(sX + a * npad * 128);
+#pragma unroll
+            for (int kk = 0; kk < kTcAtom / 16; ++kk)
+                umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                        smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (a | kk) ? 1u : 0u);
+        }
+        if (!ok) raise_error(p.err, kErrTimeout);
+        umma_commit(&bar_mma);
+    }
+    // ---- this CTA's partial tile row (thread = row = TMEM lane)
+    float d[kTcMaxN];
+#pragma unroll
+    for (int e = 0; e < kTcMaxN; ++e) d[e] = 0.f;
+    if (na > 0) {
+        if (!mbar_wait(&bar_mma, 0, kWaitBudget)) raise_error(p.err, kErrTimeout);
+        tc_fence_after();
+#pragma unroll
+        for (int c0 = 0; c0 < kTcMaxN; c0 += 16) {
+            if (c0 < npad) {  // uniform: npad is the same in every thread
+                uint32_t v[16];
+                tmem_ld16(tmem + ((uint32_t)(warp * 32) << 16) + (uint32_t)c0, v);
+                tmem_ld_wait();
+#pragma unroll
+                for (int e = 0; e < 16; ++e) d[c0 + e] = __uint_as_float(v[e]);
+            }
+        }
+    }
+    // the W1 atoms are consumed: the partial tile takes their place, rows npad + 4 floats apart
+    // (an odd number of 16-byte chunks, so the row writes of 8 consecutive threads do not collide)
+    float* pd = reinterpret_cast<float*>(sW);
+    const int ldp = npad + 4;
+#pragma unroll
+    for (int c = 0; c < kTcMaxN / 4; ++c)
+        if (4 * c < npad)
+            *reinterpret_cast<float4*>(pd + tid * ldp + 4 * c) = make_float4(d[4 * c], d[4 * c + 1], d[4 * c + 2], d[4 * c + 3]);
+    cluster_wait();  // every peer is running
+    cluster_sync_all();  // partial tiles complete and visible
+    // ---- owned rows: sum of the KS partials, + b1, ReLU
+    const int rpr = (kTcM + KS - 1) / KS;
+    const int rb = rank * rpr;
+    const int nr = max(0, min(kTcM, rb + rpr) - rb);
+    for (int item = tid; item < nr * (npad / 4); item += kTcThreads) {
+        const int rr = item / (npad / 4), c4 = item % (npad / 4);
+        const int row = rb + rr;
+        const float4* src = reinterpret_cast<const float4*>(pd + row * ldp + 4 * c4);
+        float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+        for (int pr = 0; pr < KS; ++pr) {
+            const float4 v = *cluster.map_shared_rank(src, pr);
+            acc.x += v.x;
+            acc.y += v.y;
+            acc.z += v.z;
+            acc.w += v.w;
+        }
+        const int j = m0 + row;
+        float4 h = make_float4(0.f, 0.f, 0.f, 0.f);
+        if (j < p.hidden) {
+            const float bj = p.b1[j];
+            h = make_float4(fmaxf(0.f, acc.x + bj), fmaxf(0.f, acc.y + bj), fmaxf(0.f, acc.z + bj),
+                            fmaxf(0.f, acc.w + bj));
+        }
+        *reinterpret_cast<float4*>(hs + rr * npad + 4 * c4) = h;
+    }
+    __syncthreads();
+    // ---- the owned rows' share of the output layer: op[n][c] = sum_j W2[c][j] h[j][n]
+    for (int item = tid; item < ng * C; item += kTcThreads) {
+        const int n = item / C, c = item % C;
+        const __nv_bfloat16* w2r = p.w2 + (size_t)c * p.hidden + m0 + rb;
+        const int jmax = min(nr, p.hidden - (m0 + rb));
+        float acc = 0.f;
+        for (int rr = 0; rr < jmax; ++rr) acc = fmaf(__bfloat162float(w2r[rr]), hs[rr * npad + n], acc);
+        op[item] = acc;
+    }
+    cluster_sync_all();  // every CTA's share visible to rank 0
+    if (rank == 0) {
+        float* dst = p.part + ((size_t)g * p.tiles + tile) * (kTcMaxN * C);
+        for (int item = tid; item < ng * C; item += kTcThreads) {
+            float sum = 0.f;
+            for (int pr = 0; pr < KS; ++pr) sum += *cluster.map_shared_rank(op + item, pr);
+            dst[item] = sum;
+        }
+        __threadfence();  // this tile's partials before the ticket
+        __syncthreads();
+        if (tid == 0) last_sh = atomic_add_acq_rel_gpu(p.counters + g, 1) == p.tiles - 1;
+        __syncthreads();
+        if (last_sh) {
+            // every tile has published: logits in tile order, then the argmax per request
+            float* logits = hs;  // this CTA's h is no longer needed (ng * C <= npad * rpr floats)
+            for (int item = tid; item < ng * C; item += kTcThreads) {
+                float sum = p.b2[item % C];
+                for (int t = 0; t < p.tiles; ++t) sum += __ldcg(p.part + ((size_t)g * p.tiles + t) * (kTcMaxN * C) + item);
+                logits[item] = sum;
+                if (p.logits_out) p.logits_out[(size_t)n0 * C + item] = sum;
+            }
+            __syncthreads();
+            for (int n = tid; n < ng; n += kTcThreads) {
+                int best = 0;
+                for (int c = 1; c < C; ++c)
+                    if (logits[n * C + c] > logits[n * C + best]) best = c;
+                p.block_size_out[n0 + n] = p.candidates[best];
+            }
+            if (tid == 0) p.counters[g] = 0;  // ready for the next call
+        }
+    }
+    cluster_sync_all();  // no CTA leaves while a peer may still read its shared memory
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    if (warp == 0) tmem_dealloc(tmem, kTcTmemCols);
+}
+
+// Scratch of the tensor-core path: partials and tickets (after the CUDA-core path's h buffer).
+size_t tc_part_bytes(int num_reqs, int hidden, int num_cand) {
+    const size_t groups = ((size_t)num_reqs + kTcMaxN - 1) / kTcMaxN;
+    const size_t tiles = ((size_t)hidden + kTcM - 1) / kTcM;
+    return align_up(sizeof(float) * groups * tiles * kTcMaxN * (size_t)num_cand, 256) +
+           align_up(sizeof(int) * groups, 256);
+}
+
+// Launches the tensor-core path; returns -1 when the shape is outside its limits.
+int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counters, cudaStream_t stream) {
+    if (reinterpret_cast<uintptr_t>(a.w1) % 16 != 0 || a.num_cand > 64) return -1;
+    const int atoms_total = (a.d_in + kTcAtom - 1) / kTcAtom;
+    const int tiles = (a.hidden + kTcM - 1) / kTcM;
+    const int groups = (a.num_reqs + kTcMaxN - 1) / kTcMaxN;
+    const int npad = ((a.num_reqs < kTcMaxN ? a.num_reqs : kTcMaxN) + 15) / 16 * 16;
+    // split d_in over as many CTAs as one wave of SMs holds, 8 at most
+    int ks = dev.sm_count / (tiles * groups);
+    ks = ks < 1 ? 1 : ks;
+    ks = ks > kTcMaxKS ? kTcMaxKS : ks;
+    ks = ks > atoms_total ? atoms_total : ks;
+    const int per = (atoms_total + ks - 1) / ks;
+    if (per > kTcMaxAtoms) return -1;
+    const int pd_bytes = kTcM * (npad + 4) * 4;
+    const int w_bytes = per * kTcAtomBytes > pd_bytes ? per * kTcAtomBytes : pd_bytes;
+    const int x_bytes = per * npad * 128;
+    const int rpr = (kTcM + ks - 1) / ks;
+    int h_bytes = rpr * npad * 4;
+    const int lg_bytes = kTcMaxN * a.num_cand * 4;  // the last tile's logits reuse the h region
+    h_bytes = h_bytes > lg_bytes ? h_bytes : lg_bytes;
+    const int op_bytes = kTcMaxN * a.num_cand * 4;
+    const int smem = 1024 + w_bytes + x_bytes + h_bytes + op_bytes;
+    if (smem > kTcMaxSmem) return -1;
+
+    CUtensorMap w1map;
+    const cuuint64_t dims[2] = {(cuuint64_t)a.d_in, (cuuint64_t)a.hidden};
+    const cuuint64_t strides[1] = {(cuuint64_t)a.d_in * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kTcAtom, (cuuint32_t)kTcM};
+    if (encode_tensor_map(&w1map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(a.w1), dims, strides, box,
+                          CU_TENSOR_MAP_SWIZZLE_128B) != BP_OK)
+        return -1;
+    static int configured[64] = {};
+    if (dev.device >= 0 && dev.device < 64 && !configured[dev.device]) {
+        if (cudaFuncSetAttribute(policy_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
+            cudaSuccess)
+            return BP_ERR_CUDA;
+        configured[dev.device] = 1;
+    }
+    PolicyTcParams p;
+    p.feats = static_cast<const __nv_bfloat16*>(a.feats);
+    p.row_stride = a.row_stride;
+    p.row_index = a.row_index;
+    p.num_reqs = a.num_reqs;
+    p.d_in = a.d_in;
+    p.hidden = a.hidden;
+    p.num_cand = a.num_cand;
+    p.atoms_total = atoms_total;
+    p.atoms_per_cta = per;
+    p.tiles = tiles;
+    p.npad = npad;
+    p.w_bytes = w_bytes;
+    p.x_bytes = x_bytes;
+    p.h_bytes = h_bytes;
+    p.b1 = a.b1;
+    p.w2 = static_cast<const __nv_bfloat16*>(a.w2);
+    p.b2 = a.b2;
+    p.candidates = a.candidates;
+    p.logits_out = a.logits_out;
+    p.block_size_out = a.block_size_out;
+    p.part = part;
+    p.counters = counters;
+    p.err = a.err_word;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[2];
+    cfg.gridDim = dim3((unsigned)(tiles * ks), (unsigned)groups, 1);
+    cfg.blockDim = dim3(kTcThreads, 1, 1);
+    cfg.dynamicSmemBytes = (size_t)smem;
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeClusterDimension;
+    attr[0].val.clusterDim.x = (unsigned)ks;
+    attr[0].val.clusterDim.y = 1;
+    attr[0].val.clusterDim.z = 1;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 2;
+    return cudaLaunchKernelEx(&cfg, policy_tc_kernel, w1map, p) == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+}
+
 template <typename T>
 int run(const PolicyArgs& a, cudaStream_t stream) {
     float* hbuf = static_cast<float*>(a.scratch);
@@ -182,14 +499,22 @@ int run(const PolicyArgs& a, cudaStream_t stream) {
 }  // namespace
 
 size_t policy_scratch_bytes(int num_reqs, int hidden, int num_cand) {
-    (void)num_cand;
-    return align_up(sizeof(float) * (size_t)num_reqs * hidden, 256);
+    return align_up(sizeof(float) * (size_t)num_reqs * hidden, 256) + tc_part_bytes(num_reqs, hidden, num_cand);
 }
 
 int launch_policy(const PolicyArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
-    (void)dev;
     if (a.num_reqs == 0) return BP_OK;
-    return a.wdtype == BP_BF16 ? run<__nv_bfloat16>(a, stream) : run<float>(a, stream);
+    if (a.wdtype == BP_BF16) {
+        uint8_t* w = static_cast<uint8_t*>(a.scratch) + align_up(sizeof(float) * (size_t)a.num_reqs * a.hidden, 256);
+        const size_t groups = ((size_t)a.num_reqs + kTcMaxN - 1) / kTcMaxN;
+        const size_t tiles = ((size_t)a.hidden + kTcM - 1) / kTcM;
+        float* part = reinterpret_cast<float*>(w);
+        int* counters = reinterpret_cast<int*>(w + align_up(sizeof(float) * groups * tiles * kTcMaxN * (size_t)a.num_cand, 256));
+        const int rc = run_tc(a, dev, part, counters, stream);
+        if (rc != -1) return rc;
+        return run<__nv_bfloat16>(a, stream);
+    }
+    return run<float>(a, stream);
 }
 
 }  // namespace bp
