@@ -163,7 +163,7 @@ struct PolicyTcParams {
     const int32_t* row_index;
     int num_reqs, d_in, hidden, num_cand;
     int atoms_total, atoms_per_cta, tiles, npad;
-    int w_bytes, x_bytes, h_bytes;  // dynamic shared-memory regions
+    int w_bytes, x_bytes, h_bytes, op_bytes;  // dynamic shared-memory regions
     const float* b1;
     const __nv_bfloat16* w2;
     const float* b2;
@@ -189,6 +189,10 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     uint8_t* sX = base + p.w_bytes;                             // x atoms
     float* hs = reinterpret_cast<float*>(sX + p.x_bytes);       // h of the owned rows [rows][npad]
     float* op = reinterpret_cast<float*>(sX + p.x_bytes + p.h_bytes);  // output-layer partial [n][c]
+    float* w2s = op + p.op_bytes / 4;  // W2 columns of the owned rows [c][row]
+    __shared__ float b1s[kTcM], b2s[64];
+    __shared__ int cands[64];
+    __shared__ long long row_sh[kTcMaxN];  // feature row of each request of the group
     __shared__ uint64_t bar_w[kTcMaxAtoms], bar_mma;
     __shared__ uint32_t tmem_sh;
     __shared__ int last_sh;
@@ -204,6 +208,9 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     const int a0 = rank * p.atoms_per_cta;
     const int na = max(0, min(p.atoms_total, a0 + p.atoms_per_cta) - a0);
     const int C = p.num_cand;
+    const int rpr = (kTcM + KS - 1) / KS;  // rows of the tile owned by each CTA after the split-K sum
+    const int rb = rank * rpr;
+    const int nr = max(0, min(kTcM, rb + rpr) - rb);
 
     cluster_arrive_relaxed();  // peers must be running before any distributed shared memory access
     if (tid == 0) {
@@ -222,24 +229,38 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
     griddep_wait();  // inputs may come from the previous kernel on the stream
+    if (tid < ng) row_sh[tid] = p.row_index ? (long long)p.row_index[n0 + tid] : (long long)(n0 + tid);
     if (tid == 0)
         for (int a = 0; a < na; ++a) {
             mbar_arrive_expect_tx(&bar_w[a], kTcAtomBytes);
             tma_load_2d(sW + a * kTcAtomBytes, &w1map, &bar_w[a], (a0 + a) * kTcAtom, m0);
         }
+    __syncthreads();  // row_sh
     // x of the group, K-major SWIZZLE_128B: atom a holds rows n of 128 bytes, 16-byte chunk c of
-    // row n stored at chunk c ^ (n & 7); rows past the group and columns past d_in are zero
+    // row n stored at chunk c ^ (n & 7); rows past the group and columns past d_in are zero.
+    // Asynchronous 16-byte copies: every copy of a thread is in flight at once.
     for (int idx = tid; idx < npad * na * 8; idx += kTcThreads) {
         const int n = idx / (na * 8), rem = idx % (na * 8);
         const int a = rem >> 3, c = rem & 7;
         const int k = (a0 + a) * kTcAtom + c * 8;
-        uint4 v = make_uint4(0u, 0u, 0u, 0u);
-        if (n < ng && k < p.d_in) {
-            const long long row = p.row_index ? (long long)p.row_index[n0 + n] : (long long)(n0 + n);
-            v = *reinterpret_cast<const uint4*>(p.feats + row * p.row_stride + k);
-        }
-        *reinterpret_cast<uint4*>(sX + a * npad * 128 + n * 128 + ((c ^ (n & 7)) << 4)) = v;
+        const bool valid = n < ng && k < p.d_in;
+        const long long row = valid ? row_sh[n] : 0;
+        cp_async16(sX + a * npad * 128 + n * 128 + ((c ^ (n & 7)) << 4), p.feats + row * p.row_stride + (valid ? k : 0),
+                   valid);
     }
+    // the small operands of the epilogue, read while the copies are in flight
+    for (int i = tid; i < C * nr; i += kTcThreads) {
+        const int c = i / nr, rr = i % nr;
+        const int j = m0 + rb + rr;
+        w2s[c * rpr + rr] = j < p.hidden ? __bfloat162float(p.w2[(size_t)c * p.hidden + j]) : 0.f;
+    }
+    for (int rr = tid; rr < nr; rr += kTcThreads) b1s[rr] = m0 + rb + rr < p.hidden ? p.b1[m0 + rb + rr] : 0.f;
+    if (rank == 0)
+        for (int c = tid; c < C; c += kTcThreads) {
+            b2s[c] = p.b2[c];
+            cands[c] = p.candidates[c];
+        }
+    cp_async_wait_all();
     fence_proxy_async_smem();  // the MMAs read x through the async proxy
     __syncthreads();
     if (tid == 0 && na > 0) {
@@ -289,25 +310,26 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     cluster_wait();  // every peer is running
     cluster_sync_all();  // partial tiles complete and visible
     // ---- owned rows: sum of the KS partials, + b1, ReLU
-    const int rpr = (kTcM + KS - 1) / KS;
-    const int rb = rank * rpr;
-    const int nr = max(0, min(kTcM, rb + rpr) - rb);
     for (int item = tid; item < nr * (npad / 4); item += kTcThreads) {
         const int rr = item / (npad / 4), c4 = item % (npad / 4);
         const int row = rb + rr;
         const float4* src = reinterpret_cast<const float4*>(pd + row * ldp + 4 * c4);
+        float4 v[kTcMaxKS];  // every remote load in flight at once, then summed in rank order
+#pragma unroll
+        for (int pr = 0; pr < kTcMaxKS; ++pr)
+            v[pr] = pr < KS ? *cluster.map_shared_rank(src, pr) : make_float4(0.f, 0.f, 0.f, 0.f);
         float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
-        for (int pr = 0; pr < KS; ++pr) {
-            const float4 v = *cluster.map_shared_rank(src, pr);
-            acc.x += v.x;
-            acc.y += v.y;
-            acc.z += v.z;
-            acc.w += v.w;
+#pragma unroll
+        for (int pr = 0; pr < kTcMaxKS; ++pr) {
+            acc.x += v[pr].x;
+            acc.y += v[pr].y;
+            acc.z += v[pr].z;
+            acc.w += v[pr].w;
         }
         const int j = m0 + row;
         float4 h = make_float4(0.f, 0.f, 0.f, 0.f);
         if (j < p.hidden) {
-            const float bj = p.b1[j];
+            const float bj = b1s[rr];
             h = make_float4(fmaxf(0.f, acc.x + bj), fmaxf(0.f, acc.y + bj), fmaxf(0.f, acc.z + bj),
                             fmaxf(0.f, acc.w + bj));
         }
@@ -317,18 +339,21 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     // ---- the owned rows' share of the output layer: op[n][c] = sum_j W2[c][j] h[j][n]
     for (int item = tid; item < ng * C; item += kTcThreads) {
         const int n = item / C, c = item % C;
-        const __nv_bfloat16* w2r = p.w2 + (size_t)c * p.hidden + m0 + rb;
-        const int jmax = min(nr, p.hidden - (m0 + rb));
+        const float* w2r = w2s + c * rpr;
         float acc = 0.f;
-        for (int rr = 0; rr < jmax; ++rr) acc = fmaf(__bfloat162float(w2r[rr]), hs[rr * npad + n], acc);
+        for (int rr = 0; rr < nr; ++rr) acc = fmaf(w2r[rr], hs[rr * npad + n], acc);  // zero past hidden
         op[item] = acc;
     }
     cluster_sync_all();  // every CTA's share visible to rank 0
     if (rank == 0) {
         float* dst = p.part + ((size_t)g * p.tiles + tile) * (kTcMaxN * C);
         for (int item = tid; item < ng * C; item += kTcThreads) {
+            float v[kTcMaxKS];
+#pragma unroll
+            for (int pr = 0; pr < kTcMaxKS; ++pr) v[pr] = pr < KS ? *cluster.map_shared_rank(op + item, pr) : 0.f;
             float sum = 0.f;
-            for (int pr = 0; pr < KS; ++pr) sum += *cluster.map_shared_rank(op + item, pr);
+#pragma unroll
+            for (int pr = 0; pr < kTcMaxKS; ++pr) sum += v[pr];
             dst[item] = sum;
         }
         __threadfence();  // this tile's partials before the ticket
@@ -339,8 +364,15 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
             // every tile has published: logits in tile order, then the argmax per request
             float* logits = hs;  // this CTA's h is no longer needed (ng * C <= npad * rpr floats)
             for (int item = tid; item < ng * C; item += kTcThreads) {
-                float sum = p.b2[item % C];
-                for (int t = 0; t < p.tiles; ++t) sum += __ldcg(p.part + ((size_t)g * p.tiles + t) * (kTcMaxN * C) + item);
+                float sum = b2s[item % C];
+                const float* src = p.part + (size_t)g * p.tiles * (kTcMaxN * C) + item;
+                for (int t0 = 0; t0 < p.tiles; t0 += 16) {  // 16 loads in flight, summed in tile order
+                    float v[16];
+#pragma unroll
+                    for (int u = 0; u < 16; ++u) v[u] = t0 + u < p.tiles ? __ldcg(src + (size_t)(t0 + u) * (kTcMaxN * C)) : 0.f;
+#pragma unroll
+                    for (int u = 0; u < 16; ++u) sum += v[u];
+                }
                 logits[item] = sum;
                 if (p.logits_out) p.logits_out[(size_t)n0 * C + item] = sum;
             }
@@ -349,7 +381,7 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
                 int best = 0;
                 for (int c = 1; c < C; ++c)
                     if (logits[n * C + c] > logits[n * C + best]) best = c;
-                p.block_size_out[n0 + n] = p.candidates[best];
+                p.block_size_out[n0 + n] = cands[best];
             }
             if (tid == 0) p.counters[g] = 0;  // ready for the next call
         }
@@ -391,7 +423,8 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     const int lg_bytes = kTcMaxN * a.num_cand * 4;  // the last tile's logits reuse the h region
     h_bytes = h_bytes > lg_bytes ? h_bytes : lg_bytes;
     const int op_bytes = kTcMaxN * a.num_cand * 4;
-    const int smem = 1024 + w_bytes + x_bytes + h_bytes + op_bytes;
+    const int w2s_bytes = a.num_cand * rpr * 4;
+    const int smem = 1024 + w_bytes + x_bytes + h_bytes + op_bytes + w2s_bytes;
     if (smem > kTcMaxSmem) return -1;
 
     CUtensorMap w1map;
@@ -423,6 +456,7 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     p.w_bytes = w_bytes;
     p.x_bytes = x_bytes;
     p.h_bytes = h_bytes;
+    p.op_bytes = op_bytes;
     p.b1 = a.b1;
     p.w2 = static_cast<const __nv_bfloat16*>(a.w2);
     p.b2 = a.b2;
