@@ -276,7 +276,7 @@ def run_ours(args):
         "a3_drafter_attention_bidir": row(t_bidir, attention_bytes(w), ["attn_bf16_tc_kernel"]),
         "a5_a6_accept_t1": row(t_acc, accept_bytes(w, 1.0), ["accept_kernel<false,true>"]),
         "a7_accept_greedy_t0": row(t_acc0, accept_bytes(w, 0.0), ["accept_kernel<true,true>"]),
-        "a1_policy_head_32req_2560x2048": row(t_pol, policy_bytes(pin), ["policy_hidden_kernel", "policy_out_kernel"]),
+        "a1_policy_head_32req_2560x2048": row(t_pol, policy_bytes(pin), ["policy_tc_kernel"]),
     }
     dom_name, dom_t, dom_bytes = ("accept_kernel", t_acc, accept_bytes(w, 1.0))
     traffic = committed_traffic(dom_name)
