@@ -3,22 +3,23 @@
 //
 // One thread-block cluster of CS CTAs per target row; the CTA of cluster rank c owns the
 // c-th slice of the vocabulary of that target row and of the matching draft row.
-//   load    one thread issues a single bulk copy (cp.async.bulk) per row slice into shared
-//           memory, so each slice is one transfer in flight and the logits are read from HBM
-//           exactly once;
-//   pass 1  each thread walks its slots in batches of 16 entries keeping an online maximum
-//           and sum of 2^(l*log2e/T - max); the weights replace the logits in place and each
-//           batch records the maximum they are relative to.  Warp shuffles, then every CTA
-//           pushes its slice statistics into every other CTA's shared memory (one cluster
-//           barrier) and each derives the row's log-sum-exp and a_i = min(1, p(x_i)/q(x_i));
+//   load    each warp owns a contiguous range of the slice and brings it into shared memory
+//           with one bulk copy (cp.async.bulk) per row, so the logits are read from HBM once
+//           and a warp starts on its range as soon as that range has landed;
+//   pass 1  each lane finds a reference maximum m over its entries of the range, then the
+//           weights 2^(l*log2e/T - m) replace the logits in place and are summed.  Warp and
+//           CTA reductions, then every CTA pushes its slice statistics into every other CTA's
+//           shared memory (one cluster barrier); one warp merges them into the row's
+//           log-sum-exp, and the CTA holding x_i gives a_i = min(1, p(x_i)/q(x_i));
 //   pass 2  one multiply per entry turns the stored weights into p and r = max(0, p - q);
 //           128-entry segment sums go to exact 2^-52 fixed point, a second cluster exchange
-//           of the slice totals locates the slice, then the segment, then the entry where the
-//           inverse CDF of this row's own distribution crosses u_s * Z -- the token the
-//           sequence emits if its first rejection falls on this row (a residual draw; a bonus
-//           draw from p on the last row), computed speculatively by every row in parallel;
-//   final   the CTA that wrote the last row token of a sequence (atomic ticket, no waiting)
-//           finds the first rejection k from the a_i and emits the tokens of row k.
+//           of the slice totals locates the slice, then one warp finds the range, the segment
+//           and the entry where the inverse CDF of this row's own distribution crosses u_s * Z
+//           -- the token the sequence emits if its first rejection falls on this row (a
+//           residual draw; a bonus draw from p on the last row), computed speculatively by
+//           every row in parallel;
+//   final   the thread that publishes the last row token of a sequence (atomic ticket, no
+//           waiting) finds the first rejection k from the a_i and emits the tokens of row k.
 // Temperature 0 (greedy): one pass reduces the argmax (lowest index on ties).
 #include <cooperative_groups.h>
 
