@@ -40,7 +40,7 @@
 extern "C" {
 #endif
 
-#define BP_ABI_VERSION 1
+#define BP_ABI_VERSION 2
 
 /* Symbols of the ABI are exported; everything else in the library is hidden. */
 #if defined(__GNUC__)
@@ -176,7 +176,7 @@ BP_API int bp_spec_accept_noalloc(const float* target_logits, const float* draft
  * Limits: d_in % 8 == 0 and 16-byte aligned rows for bf16 (d_in % 4 == 0 for fp32),
  * num_cand <= 64.
  * ------------------------------------------------------------------------------- */
-BP_API size_t bp_policy_select_workspace_size(int num_reqs, int hidden, int num_cand);
+BP_API size_t bp_policy_select_workspace_size(int num_reqs, int d_in, int hidden, int num_cand);
 BP_API int bp_policy_select(const void* feats, int64_t feat_row_stride, const int32_t* row_index, int num_reqs, int d_in,
                      const void* w1, const float* b1, int hidden, const void* w2, const float* b2, int num_cand,
                      const int32_t* candidates, int wdtype, float* logits_out, int32_t* block_size_out,

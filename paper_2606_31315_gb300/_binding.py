@@ -63,7 +63,7 @@ def load():
     lib.bp_spec_accept_workspace_size.restype = sz
     lib.bp_spec_accept.argtypes = [vp, vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bp_spec_accept.restype = i32
-    lib.bp_policy_select_workspace_size.argtypes = [i32, i32, i32]
+    lib.bp_policy_select_workspace_size.argtypes = [i32, i32, i32, i32]
     lib.bp_policy_select_workspace_size.restype = sz
     lib.bp_policy_select.argtypes = [vp, i64, vp, i32, i32, vp, vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, sz, vp]
     lib.bp_policy_select.restype = i32
@@ -162,8 +162,8 @@ def spec_accept(target_logits, draft_logits, draft_tokens, cu_draft, temperature
 
 
 # --------------------------------------------------------------------------- policy head
-def policy_select_workspace_size(num_reqs, hidden, num_cand) -> int:
-    return int(load().bp_policy_select_workspace_size(num_reqs, hidden, num_cand))
+def policy_select_workspace_size(num_reqs, d_in, hidden, num_cand) -> int:
+    return int(load().bp_policy_select_workspace_size(num_reqs, d_in, hidden, num_cand))
 
 
 def policy_select(feats, w1, b1, w2, b2, candidates, row_index=None, num_reqs=None, block_size=None, logits=None,
@@ -185,7 +185,7 @@ def policy_select(feats, w1, b1, w2, b2, candidates, row_index=None, num_reqs=No
     if logits is None and want_logits:
         logits = torch.empty((n, c), dtype=torch.float32, device=dev)
     if ws is None:
-        ws = workspace(lib.bp_policy_select_workspace_size(n, hidden, c), dev)
+        ws = workspace(lib.bp_policy_select_workspace_size(n, d_in, hidden, c), dev)
     rc = lib.bp_policy_select(_ptr(feats), feats.stride(0), _ptr(row_index), n, d_in, _ptr(w1), _ptr(b1), hidden,
                               _ptr(w2), _ptr(b2), c, _ptr(candidates), wdtype, _ptr(logits), _ptr(block_size),
                               _ptr(ws), ws.numel(), _stream(stream))

@@ -198,9 +198,9 @@ int bp_spec_accept_noalloc(const float* target_logits, const float* draft_logits
     return rc;
 }
 
-size_t bp_policy_select_workspace_size(int num_reqs, int hidden, int num_cand) {
-    if (num_reqs < 0 || hidden < 1 || num_cand < 1) return 0;
-    return sizeof(WorkspaceHeader) + policy_scratch_bytes(num_reqs, hidden, num_cand);
+size_t bp_policy_select_workspace_size(int num_reqs, int d_in, int hidden, int num_cand) {
+    if (num_reqs < 0 || d_in < 1 || hidden < 1 || num_cand < 1) return 0;
+    return sizeof(WorkspaceHeader) + policy_scratch_bytes(num_reqs, d_in, hidden, num_cand);
 }
 
 int bp_policy_select(const void* feats, int64_t feat_row_stride, const int32_t* row_index, int num_reqs, int d_in,
@@ -215,7 +215,7 @@ int bp_policy_select(const void* feats, int64_t feat_row_stride, const int32_t* 
     const int elt = wdtype == BP_BF16 ? 2 : 4;
     if ((d_in * elt) % 16 != 0 || (feat_row_stride * elt) % 16 != 0 || !aligned(feats, 16) || !aligned(w1, 16))
         return BP_ERR_UNSUPPORTED;
-    int rc = check_workspace(workspace, workspace_bytes, bp_policy_select_workspace_size(num_reqs, hidden, num_cand));
+    int rc = check_workspace(workspace, workspace_bytes, bp_policy_select_workspace_size(num_reqs, d_in, hidden, num_cand));
     if (rc != BP_OK) return rc;
     DeviceInfo dev;
     if ((rc = device_info(&dev)) != BP_OK) return rc;

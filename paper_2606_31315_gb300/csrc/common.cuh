@@ -98,7 +98,7 @@ struct PolicyArgs {
     void* scratch;
     unsigned int* err_word;
 };
-size_t policy_scratch_bytes(int num_reqs, int hidden, int num_cand);
+size_t policy_scratch_bytes(int num_reqs, int d_in, int hidden, int num_cand);
 int launch_policy(const PolicyArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
 }  // namespace bp

@@ -151,7 +151,8 @@ constexpr int kTcM = 128;          // hidden rows per tile: the MMA M
 constexpr int kTcMaxN = 64;        // requests per group: the MMA N (padded to a multiple of 16)
 constexpr int kTcAtom = 64;        // d_in columns per 128-byte swizzle atom
 constexpr int kTcAtomBytes = kTcM * kTcAtom * 2;  // 16 KB of W1 per atom
-constexpr int kTcMaxAtoms = 8;     // atoms per CTA
+constexpr int kTcMaxAtoms = 8;     // atoms per CTA when all of them are loaded at once
+constexpr int kTcStages = 4;       // ring depth when the atoms of a CTA are streamed (large d_in)
 constexpr int kTcMaxKS = 8;        // CTAs per cluster
 constexpr int kTcThreads = 128;    // thread t = tile row t = TMEM lane t
 constexpr uint32_t kTcTmemCols = 64;
@@ -181,7 +182,37 @@ __device__ __forceinline__ int atomic_add_acq_rel_gpu(int* addr, int v) {
     return old;
 }
 
+// Gathers the pooled rows of every request group into a contiguous [groups*64][d_in] buffer (rows
+// past the last request zero), so that the streamed path can load x with TMA like W1.
+__global__ void __launch_bounds__(256) policy_gather_kernel(const __nv_bfloat16* __restrict__ feats,
+                                                            int64_t row_stride, const int32_t* __restrict__ row_index,
+                                                            int num_reqs, int d_in, int groups, int npad,
+                                                            __nv_bfloat16* __restrict__ xg) {
+    griddep_launch_dependents();
+    griddep_wait();
+    const int chunks = d_in / 8;
+    const long long total = (long long)groups * npad * chunks;
+    for (long long idx = blockIdx.x * (long long)blockDim.x + threadIdx.x; idx < total;
+         idx += (long long)gridDim.x * blockDim.x) {
+        const int c = (int)(idx % chunks);
+        const long long gn = idx / chunks;
+        const int n = (int)(gn % npad), g = (int)(gn / npad);
+        const int req = g * kTcMaxN + n;
+        uint4 v = make_uint4(0u, 0u, 0u, 0u);
+        if (req < num_reqs) {
+            const long long row = row_index ? (long long)row_index[req] : (long long)req;
+            v = *reinterpret_cast<const uint4*>(feats + row * row_stride + c * 8);
+        }
+        *reinterpret_cast<uint4*>(xg + (size_t)req * d_in + c * 8) = v;
+    }
+}
+
+// RING = false: every W1 and x atom of the CTA is loaded at once (x gathered by the CTA itself).
+// RING = true: the atoms stream through a kTcStages-deep ring (W1 and the gathered x by TMA), for
+// any d_in; thread 0 produces, thread 32 issues the MMAs.
+template <bool RING>
 __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_constant__ CUtensorMap w1map,
+                                                              const __grid_constant__ CUtensorMap xmap,
                                                               const PolicyTcParams p) {
     extern __shared__ uint8_t smem_raw[];
     uint8_t* base = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
@@ -193,7 +224,8 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     __shared__ float b1s[kTcM], b2s[64];
     __shared__ int cands[64];
     __shared__ long long row_sh[kTcMaxN];  // feature row of each request of the group
-    __shared__ uint64_t bar_w[kTcMaxAtoms], bar_mma;
+    __shared__ uint64_t bar_w[kTcMaxAtoms], bar_mma;  // one-shot: an atom's landing; ring: full stages
+    __shared__ uint64_t bar_empty[kTcStages];
     __shared__ uint32_t tmem_sh;
     __shared__ int last_sh;
 
@@ -215,7 +247,11 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     cluster_arrive_relaxed();  // peers must be running before any distributed shared memory access
     if (tid == 0) {
         prefetch_tensormap(&w1map);
-        for (int a = 0; a < na; ++a) mbar_init(&bar_w[a], 1);
+        if (RING) prefetch_tensormap(&xmap);
+        const int nb = RING ? kTcStages : na;
+        for (int a = 0; a < nb; ++a) mbar_init(&bar_w[a], 1);
+        if (RING)
+            for (int st = 0; st < kTcStages; ++st) mbar_init(&bar_empty[st], 1);
         mbar_init(&bar_mma, 1);
         fence_mbar_init();
     }
@@ -229,57 +265,108 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     tc_fence_after();
     const uint32_t tmem = tmem_sh;
     griddep_wait();  // inputs may come from the previous kernel on the stream
-    if (tid < ng) row_sh[tid] = p.row_index ? (long long)p.row_index[n0 + tid] : (long long)(n0 + tid);
-    if (tid == 0)
-        for (int a = 0; a < na; ++a) {
-            mbar_arrive_expect_tx(&bar_w[a], kTcAtomBytes);
-            tma_load_2d(sW + a * kTcAtomBytes, &w1map, &bar_w[a], (a0 + a) * kTcAtom, m0);
-        }
-    __syncthreads();  // row_sh
-    // x of the group, K-major SWIZZLE_128B: atom a holds rows n of 128 bytes, 16-byte chunk c of
-    // row n stored at chunk c ^ (n & 7); rows past the group and columns past d_in are zero.
-    // Asynchronous 16-byte copies: every copy of a thread is in flight at once.
-    for (int idx = tid; idx < npad * na * 8; idx += kTcThreads) {
-        const int n = idx / (na * 8), rem = idx % (na * 8);
-        const int a = rem >> 3, c = rem & 7;
-        const int k = (a0 + a) * kTcAtom + c * 8;
-        const bool valid = n < ng && k < p.d_in;
-        const long long row = valid ? row_sh[n] : 0;
-        cp_async16(sX + a * npad * 128 + n * 128 + ((c ^ (n & 7)) << 4), p.feats + row * p.row_stride + (valid ? k : 0),
-                   valid);
-    }
-    // the small operands of the epilogue, read while the copies are in flight
-    for (int i = tid; i < C * nr; i += kTcThreads) {
-        const int c = i / nr, rr = i % nr;
-        const int j = m0 + rb + rr;
-        w2s[c * rpr + rr] = j < p.hidden ? __bfloat162float(p.w2[(size_t)c * p.hidden + j]) : 0.f;
-    }
-    for (int rr = tid; rr < nr; rr += kTcThreads) b1s[rr] = m0 + rb + rr < p.hidden ? p.b1[m0 + rb + rr] : 0.f;
-    if (rank == 0)
-        for (int c = tid; c < C; c += kTcThreads) {
-            b2s[c] = p.b2[c];
-            cands[c] = p.candidates[c];
-        }
-    cp_async_wait_all();
-    fence_proxy_async_smem();  // the MMAs read x through the async proxy
-    __syncthreads();
-    if (tid == 0 && na > 0) {
-        const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
-        bool ok = true;
-        for (int a = 0; a < na && ok; ++a) {
-            if (!mbar_wait(&bar_w[a], 0, kWaitBudget)) {
-                ok = false;
-                break;
+    if (RING) {
+        const uint32_t stage_bytes = (uint32_t)(kTcAtomBytes + npad * 128);
+        if (tid == 0) {  // producer: W1 and x atoms through the ring
+            for (int j = 0; j < na; ++j) {
+                const int st = j % kTcStages;
+                if (j >= kTcStages && !mbar_wait(&bar_empty[st], ((j / kTcStages) - 1) & 1, kWaitBudget)) {
+                    raise_error(p.err, kErrTimeout);
+                    break;
+                }
+                mbar_arrive_expect_tx(&bar_w[st], stage_bytes);
+                tma_load_2d(sW + st * kTcAtomBytes, &w1map, &bar_w[st], (a0 + j) * kTcAtom, m0);
+                tma_load_2d(sX + st * npad * 128, &xmap, &bar_w[st], (a0 + j) * kTcAtom, n0);
             }
-            tc_fence_after();
-            const uint32_t wa = smem_addr(sW + a * kTcAtomBytes), xa = smem_addr(sX + a * npad * 128);
+        } else if (tid == 32) {  // MMA issuer
+            if (na > 0) {
+                const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
+                bool ok = true;
+                for (int j = 0; j < na; ++j) {
+                    const int st = j % kTcStages;
+                    if (!mbar_wait(&bar_w[st], (j / kTcStages) & 1, kWaitBudget)) {
+                        ok = false;
+                        break;
+                    }
+                    tc_fence_after();
+                    const uint32_t wa = smem_addr(sW + st * kTcAtomBytes), xa = smem_addr(sX + st * npad * 128);
 #pragma unroll
-            for (int kk = 0; kk < kTcAtom / 16; ++kk)
-                umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
-                        smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (a | kk) ? 1u : 0u);
+                    for (int kk = 0; kk < kTcAtom / 16; ++kk)
+                        umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                                smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (j | kk) ? 1u : 0u);
+                    umma_commit(&bar_empty[st]);  // the stage is free once these MMAs have read it
+                }
+                if (!ok) raise_error(p.err, kErrTimeout);
+                umma_commit(&bar_mma);
+            }
+        } else if (warp >= 2) {  // the small operands of the epilogue, while the ring runs
+            const int t = tid - 64;
+            for (int i = t; i < C * nr; i += kTcThreads - 64) {
+                const int c = i / nr, rr = i % nr;
+                const int j = m0 + rb + rr;
+                w2s[c * rpr + rr] = j < p.hidden ? __bfloat162float(p.w2[(size_t)c * p.hidden + j]) : 0.f;
+            }
+            for (int rr = t; rr < nr; rr += kTcThreads - 64) b1s[rr] = m0 + rb + rr < p.hidden ? p.b1[m0 + rb + rr] : 0.f;
+            if (rank == 0)
+                for (int c = t; c < C; c += kTcThreads - 64) {
+                    b2s[c] = p.b2[c];
+                    cands[c] = p.candidates[c];
+                }
         }
-        if (!ok) raise_error(p.err, kErrTimeout);
-        umma_commit(&bar_mma);
+        __syncthreads();  // the epilogue operands
+    } else {
+        if (tid < ng) row_sh[tid] = p.row_index ? (long long)p.row_index[n0 + tid] : (long long)(n0 + tid);
+        if (tid == 0)
+            for (int a = 0; a < na; ++a) {
+                mbar_arrive_expect_tx(&bar_w[a], kTcAtomBytes);
+                tma_load_2d(sW + a * kTcAtomBytes, &w1map, &bar_w[a], (a0 + a) * kTcAtom, m0);
+            }
+        __syncthreads();  // row_sh
+        // x of the group, K-major SWIZZLE_128B: atom a holds rows n of 128 bytes, 16-byte chunk c of
+        // row n stored at chunk c ^ (n & 7); rows past the group and columns past d_in are zero.
+        // Asynchronous 16-byte copies: every copy of a thread is in flight at once.
+        for (int idx = tid; idx < npad * na * 8; idx += kTcThreads) {
+            const int n = idx / (na * 8), rem = idx % (na * 8);
+            const int a = rem >> 3, c = rem & 7;
+            const int k = (a0 + a) * kTcAtom + c * 8;
+            const bool valid = n < ng && k < p.d_in;
+            const long long row = valid ? row_sh[n] : 0;
+            cp_async16(sX + a * npad * 128 + n * 128 + ((c ^ (n & 7)) << 4), p.feats + row * p.row_stride + (valid ? k : 0),
+                       valid);
+        }
+        // the small operands of the epilogue, read while the copies are in flight
+        for (int i = tid; i < C * nr; i += kTcThreads) {
+            const int c = i / nr, rr = i % nr;
+            const int j = m0 + rb + rr;
+            w2s[c * rpr + rr] = j < p.hidden ? __bfloat162float(p.w2[(size_t)c * p.hidden + j]) : 0.f;
+        }
+        for (int rr = tid; rr < nr; rr += kTcThreads) b1s[rr] = m0 + rb + rr < p.hidden ? p.b1[m0 + rb + rr] : 0.f;
+        if (rank == 0)
+            for (int c = tid; c < C; c += kTcThreads) {
+                b2s[c] = p.b2[c];
+                cands[c] = p.candidates[c];
+            }
+        cp_async_wait_all();
+        fence_proxy_async_smem();  // the MMAs read x through the async proxy
+        __syncthreads();
+        if (tid == 0 && na > 0) {
+            const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
+            bool ok = true;
+            for (int a = 0; a < na && ok; ++a) {
+                if (!mbar_wait(&bar_w[a], 0, kWaitBudget)) {
+                    ok = false;
+                    break;
+                }
+                tc_fence_after();
+                const uint32_t wa = smem_addr(sW + a * kTcAtomBytes), xa = smem_addr(sX + a * npad * 128);
+#pragma unroll
+                for (int kk = 0; kk < kTcAtom / 16; ++kk)
+                    umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                            smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (a | kk) ? 1u : 0u);
+            }
+            if (!ok) raise_error(p.err, kErrTimeout);
+            umma_commit(&bar_mma);
+        }
     }
     // ---- this CTA's partial tile row (thread = row = TMEM lane)
     float d[kTcMaxN];
@@ -400,9 +487,15 @@ size_t tc_part_bytes(int num_reqs, int hidden, int num_cand) {
     return align_up(sizeof(float) * groups * tiles * kTcMaxN * (size_t)num_cand, 256) +
            align_up(sizeof(int) * groups, 256);
 }
+// The gathered x of the streamed path: [groups * 64][d_in] bf16.
+size_t tc_x_bytes(int num_reqs, int d_in) {
+    const size_t groups = ((size_t)num_reqs + kTcMaxN - 1) / kTcMaxN;
+    return align_up(groups * kTcMaxN * (size_t)d_in * 2, 256);
+}
 
 // Launches the tensor-core path; returns -1 when the shape is outside its limits.
-int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counters, cudaStream_t stream) {
+int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counters, __nv_bfloat16* xg,
+           cudaStream_t stream) {
     if (reinterpret_cast<uintptr_t>(a.w1) % 16 != 0 || a.num_cand > 64) return -1;
     const int atoms_total = (a.d_in + kTcAtom - 1) / kTcAtom;
     const int tiles = (a.hidden + kTcM - 1) / kTcM;
@@ -414,10 +507,11 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     ks = ks > kTcMaxKS ? kTcMaxKS : ks;
     ks = ks > atoms_total ? atoms_total : ks;
     const int per = (atoms_total + ks - 1) / ks;
-    if (per > kTcMaxAtoms) return -1;
+    const bool ring = per > kTcMaxAtoms;  // too many atoms to hold at once: stream them
+    const int slots = ring ? kTcStages : per;
     const int pd_bytes = kTcM * (npad + 4) * 4;
-    const int w_bytes = per * kTcAtomBytes > pd_bytes ? per * kTcAtomBytes : pd_bytes;
-    const int x_bytes = per * npad * 128;
+    const int w_bytes = slots * kTcAtomBytes > pd_bytes ? slots * kTcAtomBytes : pd_bytes;
+    const int x_bytes = slots * npad * 128;
     const int rpr = (kTcM + ks - 1) / ks;
     int h_bytes = rpr * npad * 4;
     const int lg_bytes = kTcMaxN * a.num_cand * 4;  // the last tile's logits reuse the h region
@@ -427,17 +521,27 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     const int smem = 1024 + w_bytes + x_bytes + h_bytes + op_bytes + w2s_bytes;
     if (smem > kTcMaxSmem) return -1;
 
-    CUtensorMap w1map;
+    CUtensorMap w1map, xmap;
     const cuuint64_t dims[2] = {(cuuint64_t)a.d_in, (cuuint64_t)a.hidden};
     const cuuint64_t strides[1] = {(cuuint64_t)a.d_in * 2};
     const cuuint32_t box[2] = {(cuuint32_t)kTcAtom, (cuuint32_t)kTcM};
     if (encode_tensor_map(&w1map, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(a.w1), dims, strides, box,
                           CU_TENSOR_MAP_SWIZZLE_128B) != BP_OK)
         return -1;
+    xmap = w1map;  // not read by the one-shot kernel
+    if (ring) {
+        const cuuint64_t xdims[2] = {(cuuint64_t)a.d_in, (cuuint64_t)groups * kTcMaxN};
+        const cuuint32_t xbox[2] = {(cuuint32_t)kTcAtom, (cuuint32_t)npad};
+        if (encode_tensor_map(&xmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, xg, xdims, strides, xbox,
+                              CU_TENSOR_MAP_SWIZZLE_128B) != BP_OK)
+            return -1;
+    }
     static int configured[64] = {};
     if (dev.device >= 0 && dev.device < 64 && !configured[dev.device]) {
-        if (cudaFuncSetAttribute(policy_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
-            cudaSuccess)
+        if (cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
+                cudaSuccess)
             return BP_ERR_CUDA;
         configured[dev.device] = 1;
     }
@@ -466,6 +570,23 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     p.part = part;
     p.counters = counters;
     p.err = a.err_word;
+    cudaLaunchAttribute pdl[1];
+    pdl[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    pdl[0].val.programmaticStreamSerializationAllowed = 1;
+    if (ring) {
+        const long long total = (long long)groups * npad * (a.d_in / 8);
+        long long blocks = (total + 255) / 256;
+        const long long cap = 4LL * dev.sm_count;
+        cudaLaunchConfig_t gcfg = {};
+        gcfg.gridDim = dim3((unsigned)(blocks < cap ? blocks : cap), 1, 1);
+        gcfg.blockDim = dim3(256, 1, 1);
+        gcfg.stream = stream;
+        gcfg.attrs = pdl;
+        gcfg.numAttrs = 1;
+        if (cudaLaunchKernelEx(&gcfg, policy_gather_kernel, p.feats, a.row_stride, a.row_index, a.num_reqs, a.d_in,
+                               groups, npad, xg) != cudaSuccess)
+            return BP_ERR_CUDA;
+    }
     cudaLaunchConfig_t cfg = {};
     cudaLaunchAttribute attr[2];
     cfg.gridDim = dim3((unsigned)(tiles * ks), (unsigned)groups, 1);
@@ -476,11 +597,12 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     attr[0].val.clusterDim.x = (unsigned)ks;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
+    attr[1] = pdl[0];
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    return cudaLaunchKernelEx(&cfg, policy_tc_kernel, w1map, p) == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+    const cudaError_t e = ring ? cudaLaunchKernelEx(&cfg, policy_tc_kernel<true>, w1map, xmap, p)
+                               : cudaLaunchKernelEx(&cfg, policy_tc_kernel<false>, w1map, xmap, p);
+    return e == cudaSuccess ? BP_OK : BP_ERR_CUDA;
 }
 
 template <typename T>
@@ -532,19 +654,21 @@ int run(const PolicyArgs& a, cudaStream_t stream) {
 
 }  // namespace
 
-size_t policy_scratch_bytes(int num_reqs, int hidden, int num_cand) {
-    return align_up(sizeof(float) * (size_t)num_reqs * hidden, 256) + tc_part_bytes(num_reqs, hidden, num_cand);
+size_t policy_scratch_bytes(int num_reqs, int d_in, int hidden, int num_cand) {
+    return align_up(sizeof(float) * (size_t)num_reqs * hidden, 256) + tc_part_bytes(num_reqs, hidden, num_cand) +
+           tc_x_bytes(num_reqs, d_in);
 }
 
 int launch_policy(const PolicyArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
     if (a.num_reqs == 0) return BP_OK;
     if (a.wdtype == BP_BF16) {
         uint8_t* w = static_cast<uint8_t*>(a.scratch) + align_up(sizeof(float) * (size_t)a.num_reqs * a.hidden, 256);
+        float* part = reinterpret_cast<float*>(w);
         const size_t groups = ((size_t)a.num_reqs + kTcMaxN - 1) / kTcMaxN;
         const size_t tiles = ((size_t)a.hidden + kTcM - 1) / kTcM;
-        float* part = reinterpret_cast<float*>(w);
         int* counters = reinterpret_cast<int*>(w + align_up(sizeof(float) * groups * tiles * kTcMaxN * (size_t)a.num_cand, 256));
-        const int rc = run_tc(a, dev, part, counters, stream);
+        __nv_bfloat16* xg = reinterpret_cast<__nv_bfloat16*>(w + tc_part_bytes(a.num_reqs, a.hidden, a.num_cand));
+        const int rc = run_tc(a, dev, part, counters, xg, stream);
         if (rc != -1) return rc;
         return run<__nv_bfloat16>(a, stream);
     }

@@ -43,7 +43,7 @@ def test_exports_match_header(lib):
 
 
 def test_version_and_error_strings(lib):
-    assert lib.bp_abi_version() == 1
+    assert lib.bp_abi_version() == 2
     for code in range(7):
         assert lib.bp_error_string(code).startswith(b"BP_")
     assert lib.bp_error_string(99) == b"unknown bp_status"
@@ -54,7 +54,7 @@ def test_workspace_sizes(lib):
     w = bp.spec_accept_workspace_size(1, 15, 151936)
     assert w > 256 and w % 256 == 0
     assert bp.spec_accept_workspace_size(32, 500, 151936) > w
-    assert bp.policy_select_workspace_size(32, 2048, 9) >= 256 + 32 * 2048 * 4
+    assert bp.policy_select_workspace_size(32, 2560, 2048, 9) >= 256 + 32 * 2048 * 4 + 64 * 2560 * 2
     assert lib.bp_spec_accept_workspace_size(-1, 0, 10) == 0
 
 

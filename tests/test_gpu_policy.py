@@ -66,3 +66,17 @@ def test_ties_choose_lowest_index():
     pin["b2"] = np.array([0, 1, 3, 2, 3, 3, 0, 1, 3], dtype=np.float32)
     bs, _ = _run(pin)
     assert np.all(bs == pin["candidates"][2])
+
+
+def test_paper_input_width_streams_w1():
+    # Section 3.1 feeds the predictor the last-token logit vector, so d_in = V = 151936: far more
+    # 64-column W1 atoms per CTA than fit in shared memory at once, so they stream through a ring.
+    w = wl.custom(seed=6, policy=dict(num_reqs=4, d_in=151936, hidden=256, wdtype="bf16", feat_std=3.0))
+    _compare(wl.policy_inputs(w))
+
+
+def test_streamed_path_with_d_in_tail_and_two_request_groups():
+    # d_in = 4104 is not a multiple of 64 (the last atom is zero-filled), 70 requests span two
+    # groups (the second only partly filled) and hidden = 300 leaves the last W1 tile partial.
+    w = wl.custom(seed=7, policy=dict(num_reqs=70, d_in=4104, hidden=300, wdtype="bf16", feat_std=1.0))
+    _compare(wl.policy_inputs(w))
