@@ -174,7 +174,9 @@ BP_API int bp_spec_accept_noalloc(const float* target_logits, const float* draft
  *   candidates  [num_cand] int32 device array of block sizes
  *   logits_out  [num_reqs][num_cand] fp32 out, may be NULL; block_size_out [num_reqs] int32 out
  * Limits: d_in % 8 == 0 and 16-byte aligned rows for bf16 (d_in % 4 == 0 for fp32),
- * num_cand <= 64.
+ * num_cand <= 64.  Any d_in: wide inputs (such as the V-sized logit vector of Section 3.1) are
+ * streamed; the workspace then also holds the gathered bf16 rows (num_reqs rounded up to 64) x d_in,
+ * which is why its size depends on d_in.
  * ------------------------------------------------------------------------------- */
 BP_API size_t bp_policy_select_workspace_size(int num_reqs, int d_in, int hidden, int num_cand);
 BP_API int bp_policy_select(const void* feats, int64_t feat_row_stride, const int32_t* row_index, int num_reqs, int d_in,
