@@ -13,6 +13,9 @@
  *                       vocabulary -- the longest accepted prefix plus one corrected or bonus
  *                       token (Figure 1; Section 1)
  *
+ * bp_block_attention_paged and bp_kv_append run the attention over a paged KV cache (pages of
+ * a shared pool named by a per-sequence block table) and append a block's K/V to it.
+ *
  * Conventions shared by every entry point
  *   - Pointers to tensors are DEVICE pointers (cudaMalloc / torch allocations), owned by
  *     the caller; the library never allocates, frees or retains them after the call.
@@ -97,6 +100,42 @@ BP_API int bp_block_attention(const void* q, const void* k, const void* v, void*
                        int max_kv_len, int num_q_heads, int num_kv_heads, int head_dim, int dtype, int mask,
                        float softmax_scale, void* workspace, size_t workspace_bytes, void* stream);
 
+/* ---------------------------------------------------------------------------------
+ * Block attention over a paged KV cache.  The same operation as bp_block_attention
+ * (Section 2.1, Figure 1 caption), with the keys and values of every sequence held in
+ * fixed-size pages of a shared pool, as a serving engine keeps them:
+ *
+ *   key/value j of sequence s  =  pool row  block_table[s*pages_per_seq + j/page_size]*page_size
+ *                                           + j % page_size
+ *
+ *   k_cache, v_cache  [num_pages*page_size][num_kv_heads][128] bf16, 16-byte aligned
+ *   block_table  [num_seqs][pages_per_seq] int32 device array of page ids (< num_pages);
+ *            the first ceil((cu_kv[s+1]-cu_kv[s]) / page_size) entries of row s are used
+ *   cu_kv    [num_seqs+1] prefix sums of the sequences' key counts L_s + B_s (only the
+ *            counts matter here: the rows come from the pages); total_kv = cu_kv[num_seqs]
+ *   page_size  a power of two >= 16; pages_per_seq * page_size >= max_kv_len
+ *   everything else as bp_block_attention (bf16, head_dim 128 only; same workspace size).
+ * The pages of a sequence may be anywhere in the pool and in any order; every row of every
+ * page the block table names must be finite.
+ * ------------------------------------------------------------------------------- */
+BP_API int bp_block_attention_paged(const void* q, const void* k_cache, const void* v_cache, void* o, float* lse,
+                                    const int32_t* cu_q, const int32_t* cu_kv, const int32_t* block_table,
+                                    int pages_per_seq, int page_size, int num_pages, int num_seqs, int total_q,
+                                    int total_kv, int max_q_len, int max_kv_len, int num_q_heads, int num_kv_heads,
+                                    int head_dim, int dtype, int mask, float softmax_scale, void* workspace,
+                                    size_t workspace_bytes, void* stream);
+
+/* Appends the new K/V rows of every sequence (its block) to its pages: new row i of sequence
+ * s, rows [cu_new[s], cu_new[s+1]) of k_new / v_new, becomes key L_s + i, with
+ * L_s = (cu_kv[s+1]-cu_kv[s]) - (cu_new[s+1]-cu_new[s]) -- cu_kv already counts the block.
+ *   k_new, v_new  [total_new][num_kv_heads][head_dim] dtype (bf16 or fp32),
+ *                 head_dim * element size a multiple of 16 bytes
+ *   k_cache, v_cache, block_table, pages_per_seq, page_size as bp_block_attention_paged
+ * The pages that receive the rows must already be in the block table.  No workspace. */
+BP_API int bp_kv_append(void* k_cache, void* v_cache, const void* k_new, const void* v_new, const int32_t* cu_new,
+                        const int32_t* cu_kv, const int32_t* block_table, int pages_per_seq, int page_size,
+                        int num_pages, int num_seqs, int total_new, int num_kv_heads, int head_dim, int dtype,
+                        void* stream);
 /* ---------------------------------------------------------------------------------
  * Lossless speculative acceptance over the full vocabulary.  Figure 1 caption (the
  * target accepts the longest consistent prefix of the drafted block), Section 1 and

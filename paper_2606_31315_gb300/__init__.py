@@ -12,8 +12,10 @@ from ._binding import (  # noqa: F401
     MASK_CAUSAL,
     BlockPilotError,
     block_attention,
+    block_attention_paged,
     block_attention_workspace_size,
     get_status,
+    kv_append,
     library_path,
     load,
     policy_select,

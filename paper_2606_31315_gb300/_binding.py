@@ -59,6 +59,11 @@ def load():
     lib.bp_block_attention.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, i32, i32, i32,
                                        f32, vp, sz, vp]
     lib.bp_block_attention.restype = i32
+    lib.bp_block_attention_paged.argtypes = [vp, vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, i32,
+                                             i32, i32, i32, i32, i32, f32, vp, sz, vp]
+    lib.bp_block_attention_paged.restype = i32
+    lib.bp_kv_append.argtypes = [vp, vp, vp, vp, vp, vp, vp, i32, i32, i32, i32, i32, i32, i32, i32, vp]
+    lib.bp_kv_append.restype = i32
     lib.bp_spec_accept_workspace_size.argtypes = [i32, i32, i32]
     lib.bp_spec_accept_workspace_size.restype = sz
     lib.bp_spec_accept.argtypes = [vp, vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, vp, vp, vp, sz, vp]
@@ -127,6 +132,52 @@ def block_attention(q, k, v, cu_q, cu_kv, max_q_len: int, max_kv_len: int, mask:
                                 float(softmax_scale), _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "bp_block_attention")
     return out, lse
+
+
+def block_attention_paged(q, k_cache, v_cache, cu_q, cu_kv, block_table, page_size: int, total_kv: int,
+                          max_q_len: int, max_kv_len: int, mask: int = MASK_CAUSAL, softmax_scale: float = 0.0,
+                          out=None, lse=None, ws=None, stream=None):
+    """Block attention over a paged KV cache; see ``bp_block_attention_paged`` in include/blockpilot.h.
+
+    q [total_q, Hq, 128] bf16; k_cache/v_cache [num_pages * page_size, Hkv, 128] bf16; block_table int32
+    [S, pages_per_seq]; cu_q/cu_kv int32 [S+1] on the device; total_kv = cu_kv[S].  Returns (o, lse_or_None)."""
+    lib = load()
+    for t, n in ((q, "q"), (k_cache, "k_cache"), (v_cache, "v_cache"), (cu_q, "cu_q"), (cu_kv, "cu_kv"),
+                 (block_table, "block_table"), (out, "out"), (lse, "lse")):
+        _cuda(t, n)
+    dtype = {torch.bfloat16: BF16, torch.float32: F32}.get(q.dtype)
+    if dtype is None or k_cache.dtype != q.dtype or v_cache.dtype != q.dtype:
+        raise ValueError("q, k_cache, v_cache must share one dtype")
+    total_q, hq, d = q.shape
+    pool_rows, hkv, _ = k_cache.shape
+    s = cu_q.numel() - 1
+    if out is None:
+        out = torch.empty_like(q)
+    if ws is None:
+        ws = workspace(lib.bp_block_attention_workspace_size(s, max_q_len, hq, hkv, d), q.device)
+    rc = lib.bp_block_attention_paged(_ptr(q), _ptr(k_cache), _ptr(v_cache), _ptr(out), _ptr(lse), _ptr(cu_q),
+                                      _ptr(cu_kv), _ptr(block_table), block_table.shape[1], int(page_size),
+                                      pool_rows // int(page_size), s, total_q, int(total_kv), int(max_q_len),
+                                      int(max_kv_len), hq, hkv, d, dtype, int(mask), float(softmax_scale), _ptr(ws),
+                                      ws.numel(), _stream(stream))
+    _check(rc, "bp_block_attention_paged")
+    return out, lse
+
+
+def kv_append(k_cache, v_cache, k_new, v_new, cu_new, cu_kv, block_table, page_size: int, stream=None):
+    """Writes each sequence's new K/V rows into its pages; see ``bp_kv_append``."""
+    lib = load()
+    for t, n in ((k_cache, "k_cache"), (v_cache, "v_cache"), (k_new, "k_new"), (v_new, "v_new"), (cu_new, "cu_new"),
+                 (cu_kv, "cu_kv"), (block_table, "block_table")):
+        _cuda(t, n)
+    dtype = {torch.bfloat16: BF16, torch.float32: F32}.get(k_new.dtype)
+    if dtype is None or any(t.dtype != k_new.dtype for t in (k_cache, v_cache, v_new)):
+        raise ValueError("caches and new rows must share one dtype (bf16 or fp32)")
+    total_new, hkv, d = k_new.shape
+    rc = lib.bp_kv_append(_ptr(k_cache), _ptr(v_cache), _ptr(k_new), _ptr(v_new), _ptr(cu_new), _ptr(cu_kv),
+                          _ptr(block_table), block_table.shape[1], int(page_size), k_cache.shape[0] // int(page_size),
+                          cu_new.numel() - 1, total_new, hkv, d, dtype, _stream(stream))
+    _check(rc, "bp_kv_append")
 
 
 # --------------------------------------------------------------------------- acceptance

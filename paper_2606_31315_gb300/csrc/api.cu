@@ -129,8 +129,85 @@ int bp_block_attention(const void* q, const void* k, const void* v, void* o, flo
     a.mask = mask;
     a.scale = softmax_scale == 0.f ? 1.f / sqrtf((float)head_dim) : softmax_scale;
     a.err_word = err_word(workspace);
+    a.block_table = nullptr;
+    a.pages_per_seq = a.page_size = a.num_pages = 0;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     rc = dtype == BP_BF16 ? launch_attention_bf16(a, dev, st) : launch_attention_f32(a, st);
+    if (rc == BP_ERR_CUDA) cudaGetLastError();
+    return rc;
+}
+
+namespace {
+bool valid_page_size(int page_size) { return page_size >= 16 && page_size <= (1 << 20) && (page_size & (page_size - 1)) == 0; }
+}  // namespace
+
+int bp_block_attention_paged(const void* q, const void* k_cache, const void* v_cache, void* o, float* lse,
+                             const int32_t* cu_q, const int32_t* cu_kv, const int32_t* block_table,
+                             int pages_per_seq, int page_size, int num_pages, int num_seqs, int total_q,
+                             int total_kv, int max_q_len, int max_kv_len, int num_q_heads, int num_kv_heads,
+                             int head_dim,
+                             int dtype, int mask, float softmax_scale, void* workspace, size_t workspace_bytes,
+                             void* stream) {
+    if (num_seqs < 0 || total_q < 0 || total_kv < 0 || max_q_len < 0 || max_kv_len < 0) return BP_ERR_INVALID_ARG;
+    if (num_seqs == 0 || total_q == 0) return BP_OK;  // nothing to compute
+    if (!q || !k_cache || !v_cache || !o || !cu_q || !cu_kv || !block_table) return BP_ERR_INVALID_ARG;
+    if (num_q_heads < 1 || num_kv_heads < 1 || head_dim < 1 || num_q_heads % num_kv_heads != 0)
+        return BP_ERR_INVALID_ARG;
+    if (mask != BP_MASK_CAUSAL_BLOCK && mask != BP_MASK_BIDIR_BLOCK) return BP_ERR_INVALID_ARG;
+    if (dtype != BP_F32 && dtype != BP_BF16) return BP_ERR_INVALID_ARG;
+    if (!(softmax_scale >= 0.f) || isinf(softmax_scale)) return BP_ERR_INVALID_ARG;
+    if (max_q_len > max_kv_len || total_q > total_kv || !valid_page_size(page_size) || num_pages < 1)
+        return BP_ERR_INVALID_ARG;
+    if ((long long)pages_per_seq * page_size < max_kv_len || (long long)num_pages * page_size > INT32_MAX)
+        return BP_ERR_INVALID_ARG;
+    if (max_q_len > 64) return BP_ERR_UNSUPPORTED;
+    if (dtype != BP_BF16 || head_dim != 128) return BP_ERR_UNSUPPORTED;  // tensor-core path only
+    if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(o, 16)) return BP_ERR_INVALID_ARG;
+    int rc = check_workspace(workspace, workspace_bytes,
+                             bp_block_attention_workspace_size(num_seqs, max_q_len, num_q_heads, num_kv_heads,
+                                                               head_dim));
+    if (rc != BP_OK) return rc;
+    DeviceInfo dev;
+    if ((rc = device_info(&dev)) != BP_OK) return rc;
+    AttentionArgs a;
+    a.q = q; a.k = k_cache; a.v = v_cache; a.o = o; a.lse = lse; a.cu_q = cu_q; a.cu_kv = cu_kv;
+    a.num_seqs = num_seqs; a.total_q = total_q; a.total_kv = total_kv;
+    a.max_q_len = max_q_len; a.max_kv_len = max_kv_len;
+    a.num_q_heads = num_q_heads; a.num_kv_heads = num_kv_heads; a.head_dim = head_dim;
+    a.mask = mask;
+    a.scale = softmax_scale == 0.f ? 1.f / sqrtf((float)head_dim) : softmax_scale;
+    a.err_word = err_word(workspace);
+    a.block_table = block_table;
+    a.pages_per_seq = pages_per_seq;
+    a.page_size = page_size;
+    a.num_pages = num_pages;
+    rc = launch_attention_bf16(a, dev, static_cast<cudaStream_t>(stream));
+    if (rc == BP_ERR_CUDA) cudaGetLastError();
+    return rc;
+}
+
+int bp_kv_append(void* k_cache, void* v_cache, const void* k_new, const void* v_new, const int32_t* cu_new,
+                 const int32_t* cu_kv, const int32_t* block_table, int pages_per_seq, int page_size, int num_pages,
+                 int num_seqs, int total_new, int num_kv_heads, int head_dim, int dtype, void* stream) {
+    if (num_seqs < 0 || total_new < 0) return BP_ERR_INVALID_ARG;
+    if (num_seqs == 0 || total_new == 0) return BP_OK;
+    if (!k_cache || !v_cache || !k_new || !v_new || !cu_new || !cu_kv || !block_table) return BP_ERR_INVALID_ARG;
+    if (num_kv_heads < 1 || head_dim < 1 || pages_per_seq < 1 || num_pages < 1 || !valid_page_size(page_size))
+        return BP_ERR_INVALID_ARG;
+    if (dtype != BP_F32 && dtype != BP_BF16) return BP_ERR_INVALID_ARG;
+    const int row_bytes = head_dim * (dtype == BP_BF16 ? 2 : 4);
+    if (row_bytes % 16 != 0) return BP_ERR_UNSUPPORTED;
+    if (!aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(k_new, 16) || !aligned(v_new, 16))
+        return BP_ERR_INVALID_ARG;
+    DeviceInfo dev;
+    int rc = device_info(&dev);
+    if (rc != BP_OK) return rc;
+    KvAppendArgs a;
+    a.k_cache = k_cache; a.v_cache = v_cache; a.k_new = k_new; a.v_new = v_new;
+    a.cu_new = cu_new; a.cu_kv = cu_kv; a.block_table = block_table;
+    a.pages_per_seq = pages_per_seq; a.page_size = page_size; a.num_seqs = num_seqs; a.total_new = total_new;
+    a.num_kv_heads = num_kv_heads; a.row_bytes = row_bytes;
+    rc = launch_kv_append(a, static_cast<cudaStream_t>(stream));
     if (rc == BP_ERR_CUDA) cudaGetLastError();
     return rc;
 }

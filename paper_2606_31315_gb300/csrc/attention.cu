@@ -56,8 +56,13 @@ struct AttnParams {
     int causal;
     float scale_log2;  // softmax scale * log2(e)
     int q_tma;         // Q tile loaded by TMA (group divides 128)
+    // paged KV cache: sequence s's key j lives in page block_table[s * pages_per_seq + (j >> page_shift)]
+    // at row j & (page size - 1); NULL block_table = contiguous K/V rows from cu_kv[s]
+    const int32_t* block_table;
+    int pages_per_seq, page_shift;
     unsigned int* err;
 };
+constexpr int kMaxSub = kTileN / 16;  // sub-boxes per K/V tile at the smallest page size (16 keys)
 
 __device__ __forceinline__ uint32_t col_s(int sb) { return sb ? 128u : 0u; }  // TMEM column of S buffer sb
 
@@ -168,17 +173,48 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         fence_proxy_async_smem();
     }
+    // paged cache: the pool rows of tile j's sub-boxes (sub_rows keys each); keys past the end of
+    // the sequence read the rows of its last page (finite values the mask then drops)
+    const bool paged = p.block_table != nullptr;
+    const int sub_rows = paged ? min(kTileN, 1 << p.page_shift) : kTileN;
+    const int nsub = kTileN / sub_rows;
+    auto tile_rows = [&](int j, int (&row)[kMaxSub]) {
+        if (!paged) return;
+        const int32_t* bt = p.block_table + (size_t)s * p.pages_per_seq;
+        const int last_page = max(0, (n - 1) >> p.page_shift);
+        const int key0 = (t_begin + j) * kTileN;
+#pragma unroll
+        for (int sb = 0; sb < kMaxSub; ++sb)
+            if (sb < nsub) {
+                const int key = key0 + sb * sub_rows;
+                const int pi = min(key >> p.page_shift, last_page);
+                row[sb] = __ldg(bt + pi) * (1 << p.page_shift) + (key & ((1 << p.page_shift) - 1));
+            }
+    };
     // K/V tile j of this CTA's range -> ring stage j % kStages (producer thread only)
-    auto issue_kv = [&](int j) {
+    auto issue_kv = [&](int j, const int (&row)[kMaxSub]) {
         const int st = j % kStages;
         uint8_t* sK = sKV + st * kStageBytes;
         uint8_t* sV = sK + kKVBytes;
-        const int key = kv0 + (t_begin + j) * kTileN;
         mbar_arrive_expect_tx(&bar_kv_full[st], kStageBytes);
-        tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, h, key);
-        tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, h, key);
-        tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, h, key);
-        tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, h, key);
+        if (!paged) {
+            const int key = kv0 + (t_begin + j) * kTileN;
+            tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, h, key);
+            tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, h, key);
+            tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, h, key);
+            tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, h, key);
+        } else {
+#pragma unroll
+            for (int sb = 0; sb < kMaxSub; ++sb) {  // sub-box sb lands at row sb * sub_rows of the tile
+                if (sb < nsub) {
+                    const int off = sb * sub_rows * 128;
+                    tma_load_3d(sK + off, &kmap, &bar_kv_full[st], 0, h, row[sb]);
+                    tma_load_3d(sK + kHalf + off, &kmap, &bar_kv_full[st], 64, h, row[sb]);
+                    tma_load_3d(sV + off, &vmap, &bar_kv_full[st], 0, h, row[sb]);
+                    tma_load_3d(sV + kHalf + off, &vmap, &bar_kv_full[st], 64, h, row[sb]);
+                }
+            }
+        }
     };
     if (tid == 0) {
         for (int i = 0; i < kStages; ++i) {
@@ -211,7 +247,13 @@ __global__ void __launch_bounds__(kThreads, 1)
             tma_load_3d(sQ, &qmap, &bar_q_full, 0, h * G, qrow);
             tma_load_3d(sQ + kHalf, &qmap, &bar_q_full, 64, h * G, qrow);
         }
-        for (int j = 0; j < min(nt, kStages); ++j) issue_kv(j);
+        int rows0[kStages][kMaxSub];  // the first tiles' page lookups, all in flight together
+#pragma unroll
+        for (int j = 0; j < kStages; ++j)
+            if (j < nt) tile_rows(j, rows0[j]);
+#pragma unroll
+        for (int j = 0; j < kStages; ++j)
+            if (j < nt) issue_kv(j, rows0[j]);
     }
 
     if (warp == 0) {
@@ -219,11 +261,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (lane == 0 && nt > 0) {
             int issued = min(nt, kStages);  // the prologue issued the first tiles
             for (int j = kStages; j < nt; ++j) {
+                int rows[kMaxSub];
+                tile_rows(j, rows);  // page lookups in flight while the stage drains
                 if (!mbar_wait(&bar_kv_empty[j % kStages], ((j / kStages) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
-                issue_kv(j);
+                issue_kv(j, rows);
                 ++issued;
             }
             // no copy may still be in flight when the CTA leaves
@@ -590,9 +634,12 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
                                          qstrides, qbox, CU_TENSOR_MAP_SWIZZLE_128B);
         if (rq != BP_OK) return rq;
     }
-    const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)a.num_kv_heads, (cuuint64_t)a.total_kv};
+    // K/V: contiguous rows, or the page pool with boxes of one page (at most one 128-key tile)
+    const bool paged = a.block_table != nullptr;
+    const cuuint64_t kv_rows = paged ? (cuuint64_t)a.num_pages * a.page_size : (cuuint64_t)a.total_kv;
+    const cuuint64_t dims[3] = {(cuuint64_t)kD, (cuuint64_t)a.num_kv_heads, kv_rows};
     const cuuint64_t strides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.num_kv_heads * kD * 2};
-    const cuuint32_t box[3] = {64, 1, (cuuint32_t)kTileN};
+    const cuuint32_t box[3] = {64, 1, (cuuint32_t)(paged && a.page_size < kTileN ? a.page_size : kTileN)};
     int rc = encode_tensor_map(&kmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.k), dims, strides,
                                box, CU_TENSOR_MAP_SWIZZLE_128B);
     if (rc != BP_OK) return rc;
@@ -616,6 +663,10 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     p.causal = a.mask == BP_MASK_CAUSAL_BLOCK;
     p.scale_log2 = a.scale * 1.4426950408889634f;
     p.q_tma = q_tma ? 1 : 0;
+    p.block_table = a.block_table;
+    p.pages_per_seq = paged ? a.pages_per_seq : 0;
+    p.page_shift = 0;
+    while (paged && (1 << p.page_shift) < a.page_size) ++p.page_shift;
     p.err = a.err_word;
     if (!q_tma) qmap = kmap;  // unused by the kernel
 
@@ -704,6 +755,64 @@ int launch_attention_f32(const AttentionArgs& a, cudaStream_t stream) {
         static_cast<const float*>(a.v), static_cast<float*>(a.o), a.lse, a.cu_q, a.cu_kv, a.num_seqs, a.total_q,
         a.num_q_heads, a.num_kv_heads, a.head_dim, (int)(a.mask == BP_MASK_CAUSAL_BLOCK), a.scale);
     return e == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+}
+
+// --------------------------------------------------------------------------- paged KV append
+// Writes each sequence's new K/V rows (its block) into their slots of the paged cache: new row
+// i of sequence s is key L_s + i, with L_s = (cu_kv[s+1] - cu_kv[s]) - (cu_new[s+1] - cu_new[s]).
+// One warp per (new row, KV head): 16-byte copies of the K row and of the V row.
+__global__ void __launch_bounds__(256) kv_append_kernel(uint8_t* __restrict__ kc, uint8_t* __restrict__ vc,
+                                                        const uint8_t* __restrict__ kn,
+                                                        const uint8_t* __restrict__ vn,
+                                                        const int32_t* __restrict__ cu_new,
+                                                        const int32_t* __restrict__ cu_kv,
+                                                        const int32_t* __restrict__ bt, int pages_per_seq,
+                                                        int page_shift, int num_seqs, int total_new, int hkv,
+                                                        int row_bytes) {
+    griddep_launch_dependents();
+    griddep_wait();
+    const int warp = (int)((blockIdx.x * (size_t)blockDim.x + threadIdx.x) >> 5), lane = threadIdx.x & 31;
+    if (warp >= total_new * hkv) return;
+    const int t = warp / hkv, hh = warp % hkv;
+    int lo = 0, hi = num_seqs;  // largest s with cu_new[s] <= t
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (__ldg(cu_new + mid) <= t) lo = mid; else hi = mid;
+    }
+    const int s = lo;
+    const int nb = __ldg(cu_new + s + 1) - __ldg(cu_new + s);
+    const int len = __ldg(cu_kv + s + 1) - __ldg(cu_kv + s);
+    const int pos = len - nb + (t - __ldg(cu_new + s));
+    const long long page = __ldg(bt + (size_t)s * pages_per_seq + (pos >> page_shift));
+    const long long slot = (page << page_shift) + (pos & ((1 << page_shift) - 1));
+    const size_t dst = ((size_t)slot * hkv + hh) * row_bytes;
+    const size_t src = ((size_t)t * hkv + hh) * row_bytes;
+    for (int b = lane * 16; b < row_bytes; b += 32 * 16) {
+        *reinterpret_cast<uint4*>(kc + dst + b) = *reinterpret_cast<const uint4*>(kn + src + b);
+        *reinterpret_cast<uint4*>(vc + dst + b) = *reinterpret_cast<const uint4*>(vn + src + b);
+    }
+}
+
+int launch_kv_append(const KvAppendArgs& a, cudaStream_t stream) {
+    if (a.total_new == 0) return BP_OK;
+    int shift = 0;
+    while ((1 << shift) < a.page_size) ++shift;
+    const long long warps = (long long)a.total_new * a.num_kv_heads;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[1];
+    cfg.gridDim = dim3((unsigned)((warps + 7) / 8), 1, 1);
+    cfg.blockDim = dim3(256, 1, 1);
+    cfg.stream = stream;
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, kv_append_kernel, static_cast<uint8_t*>(a.k_cache), static_cast<uint8_t*>(a.v_cache),
+                              static_cast<const uint8_t*>(a.k_new), static_cast<const uint8_t*>(a.v_new), a.cu_new,
+                              a.cu_kv, a.block_table, a.pages_per_seq, shift, a.num_seqs, a.total_new,
+                              a.num_kv_heads, a.row_bytes) == cudaSuccess
+               ? BP_OK
+               : BP_ERR_CUDA;
 }
 
 }  // namespace bp

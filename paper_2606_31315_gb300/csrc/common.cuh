@@ -56,8 +56,23 @@ struct AttentionArgs {
     int mask;
     float scale;
     unsigned int* err_word;
+    // paged KV cache (NULL block_table: contiguous rows from cu_kv); pool of num_pages pages
+    const int32_t* block_table;
+    int pages_per_seq, page_size, num_pages;
 };
 int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+
+struct KvAppendArgs {
+    void* k_cache;
+    void* v_cache;
+    const void* k_new;
+    const void* v_new;
+    const int32_t* cu_new;
+    const int32_t* cu_kv;
+    const int32_t* block_table;
+    int pages_per_seq, page_size, num_seqs, total_new, num_kv_heads, row_bytes;  // row_bytes = head_dim * elt
+};
+int launch_kv_append(const KvAppendArgs& a, cudaStream_t stream);
 int launch_attention_f32(const AttentionArgs& a, cudaStream_t stream);
 
 struct AcceptArgs {

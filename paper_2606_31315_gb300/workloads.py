@@ -134,6 +134,48 @@ def attention_inputs(w: Workload) -> dict:
     return out
 
 
+def paged_kv(k: np.ndarray, v: np.ndarray, cu_kv, page_size: int, seed: int = 0, spare_pages: int = 3,
+             rows_per_seq=None) -> dict:
+    """Scatters contiguous K/V rows [total_kv, Hkv, D] into a pool of pages of page_size rows, the
+    pages of every sequence in shuffled order, as a serving engine's cache would hold them.
+
+    Rows of the pool no sequence owns are filled with other seeded values (finite), so a wrong
+    page lookup changes the result.  rows_per_seq (default: all of each sequence's rows) limits
+    how many leading rows of each sequence are copied in; the block table still covers all of
+    cu_kv's rows, so the rest can be appended later.  Returns the pools, the block table
+    [S, pages_per_seq] and the page count."""
+    cu_kv = np.asarray(cu_kv, dtype=np.int64)
+    s_count = len(cu_kv) - 1
+    lens = np.diff(cu_kv)
+    pages = [int((l + page_size - 1) // page_size) for l in lens]
+    pps = max(1, max(pages) if s_count else 1)
+    n_pages = int(sum(pages)) + spare_pages
+    rng = _rng(seed, 40)
+    perm = rng.permutation(n_pages)
+    hkv, d = k.shape[1], k.shape[2]
+    fill = rng.standard_normal((n_pages * page_size, hkv, d), dtype=np.float32)
+    if k.dtype == np.uint16:  # bf16 bits
+        fill = f32_to_bf16_bits(fill)
+    else:
+        fill = fill.astype(k.dtype)
+    kp, vp = fill.copy(), fill[::-1].copy()
+    table = np.full((s_count, pps), perm[-1], dtype=np.int32)
+    idx = 0
+    for sq in range(s_count):
+        keep = int(lens[sq]) if rows_per_seq is None else int(rows_per_seq[sq])
+        for pi in range(pages[sq]):
+            page = int(perm[idx])
+            idx += 1
+            table[sq, pi] = page
+            lo = pi * page_size
+            hi = min(keep, lo + page_size)
+            if hi > lo:
+                src = slice(int(cu_kv[sq]) + lo, int(cu_kv[sq]) + hi)
+                kp[page * page_size:page * page_size + hi - lo] = k[src]
+                vp[page * page_size:page * page_size + hi - lo] = v[src]
+    return dict(k_cache=kp, v_cache=vp, block_table=table, num_pages=n_pages, page_size=page_size)
+
+
 def accept_inputs(w: Workload, temperature: float, planted_match: float = 0.0) -> dict:
     """Target / draft logits, draft tokens and uniforms for one acceptance step.
 

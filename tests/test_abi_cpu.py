@@ -94,6 +94,26 @@ def test_host_validation_needs_no_gpu(lib):
     assert rc == 2
 
 
+
+def test_paged_host_validation_needs_no_gpu(lib):
+    vp, f32 = ctypes.c_void_p, ctypes.c_float
+    fake, ws = vp(0x10000), vp(0x20000)
+
+    def paged(block_table=fake, pps=33, page=64, pages=40, dtype=1, max_kv=2064):
+        return lib.bp_block_attention_paged(fake, fake, fake, fake, None, fake, fake, block_table, pps, page, pages, 1,
+                                            16, 2064, 16, max_kv, 32, 8, 128, dtype, 0, f32(0.0), ws, 4096, None)
+    assert paged(block_table=None) == 1                       # no block table
+    assert paged(page=24) == 1 and paged(page=8) == 1         # not a power of two >= 16
+    assert paged(pps=32) == 1                                  # 32 pages of 64 < 2064 keys
+    assert paged(dtype=0) == 2                                 # fp32 has no paged path
+
+    def append(page=64, head_dim=128, dtype=1):
+        return lib.bp_kv_append(fake, fake, fake, fake, fake, fake, fake, 33, page, 40, 1, 16, 8, head_dim, dtype, None)
+    assert append(page=100) == 1
+    assert append(head_dim=4) == 2                            # 8-byte rows: not a multiple of 16 bytes
+    assert lib.bp_kv_append(fake, fake, fake, fake, fake, fake, None, 33, 64, 40, 1, 16, 8, 128, 1, None) == 1
+
+
 def test_no_cpu_fallback_without_gpu(lib):
     import torch
 
