@@ -251,6 +251,20 @@ def run_ours(args):
     t_acc = time_graph(graph_of(accept), reps) / COPIES
     t_bidir = time_graph(graph_of(lambda c: attn(c, bp.MASK_BIDIR)), reps) / COPIES
     t_acc0 = time_graph(graph_of(lambda c: accept(c, 0.0)), reps) / COPIES
+    # next row: the same verify attention over a paged KV cache (64-row pages in shuffled order)
+    page = 64
+    pk = wl.paged_kv(a["k"], a["v"], a["cu_kv"], page, seed=1)
+    for c in copies:
+        c["kc"], c["vc"] = bf(pk["k_cache"]), bf(pk["v_cache"])
+    bt = t(pk["block_table"])
+
+    def attn_paged(c):
+        bp.block_attention_paged(c["q"], c["kc"], c["vc"], cu_q, cu_kv, bt, page, int(a["cu_kv"][-1]),
+                                 a["max_q_len"], a["max_kv_len"], out=c["o"], ws=ws_a, stream=stream)
+
+    t_attn_paged = time_graph(graph_of(attn_paged), reps) / COPIES
+    for c in copies:
+        del c["kc"], c["vc"]
     pw = wl.get("ragged")
     pin = wl.policy_inputs(pw)
     for c in copies:  # one copy of the policy weights per input copy (32 x 10.5 MB > L2)
@@ -307,6 +321,7 @@ def run_ours(args):
         "a5_a6_accept_t1": row(t_acc, accept_bytes(w, 1.0), ["accept_kernel<false,true>"]),
         "a7_accept_greedy_t0": row(t_acc0, accept_bytes(w, 0.0), ["accept_kernel<true,true>"]),
         "a1_policy_head_32req_2560x2048": row(t_pol, policy_bytes(pin), ["policy_tc_kernel"]),
+        "next3_verify_attention_paged_page64": row(t_attn_paged, attention_bytes(w), ["attn_bf16_tc_kernel (paged)"]),
         "next2_policy_head_32req_151936x2048": row(t_pol_big, big_bytes,
                                                    ["policy_gather_kernel", "policy_tc_kernel (streamed)"]),
     }
