@@ -83,6 +83,9 @@ __device__ __forceinline__ uint32_t cluster_size() {
     return r;
 }
 
+// PAGED: K/V rows come from pages named by p.block_table (the contiguous instantiation carries no
+// paging code at all).
+template <bool PAGED>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ CUtensorMap vmap, const AttnParams p) {
@@ -175,7 +178,7 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     // paged cache: the pool rows of tile j's sub-boxes (sub_rows keys each); keys past the end of
     // the sequence read the rows of its last page (finite values the mask then drops)
-    const bool paged = p.block_table != nullptr;
+    constexpr bool paged = PAGED;
     const int sub_rows = paged ? min(kTileN, 1 << p.page_shift) : kTileN;
     const int nsub = kTileN / sub_rows;
     auto tile_rows = [&](int j, int (&row)[kMaxSub]) {
@@ -676,13 +679,12 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     static int configured_device = -1;
     static int max_active[kMaxCluster + 1];
     if (configured_device != dev.device) {
-        if (cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) !=
-                cudaSuccess ||
-            cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-                cudaSuccess ||
-            cudaFuncSetAttribute(attn_bf16_tc_kernel, cudaFuncAttributePreferredSharedMemoryCarveout,
-                                 cudaSharedmemCarveoutMaxShared) != cudaSuccess)
-            return BP_ERR_CUDA;
+        for (auto kern : {attn_bf16_tc_kernel<false>, attn_bf16_tc_kernel<true>})
+            if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) != cudaSuccess ||
+                cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
+                cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
+                                     cudaSharedmemCarveoutMaxShared) != cudaSuccess)
+                return BP_ERR_CUDA;
         for (int cs = 1; cs <= kMaxCluster; ++cs) {
             cudaLaunchConfig_t probe = {};
             cudaLaunchAttribute pa[1];
@@ -696,7 +698,7 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
             probe.attrs = pa;
             probe.numAttrs = 1;
             int n_clusters = 0;
-            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel, &probe) != cudaSuccess) {
+            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel<false>, &probe) != cudaSuccess) {
                 cudaGetLastError();
                 n_clusters = 0;
             }
@@ -733,7 +735,9 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    if (cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel, qmap, kmap, vmap, p) != cudaSuccess) return BP_ERR_CUDA;
+    const cudaError_t e = paged ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true>, qmap, kmap, vmap, p)
+                                : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false>, qmap, kmap, vmap, p);
+    if (e != cudaSuccess) return BP_ERR_CUDA;
     return BP_OK;
 }
 
