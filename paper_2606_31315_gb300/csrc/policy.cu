@@ -152,8 +152,8 @@ constexpr int kTcMaxN = 64;        // requests per group: the MMA N (padded to a
 constexpr int kTcAtom = 64;        // d_in columns per 128-byte swizzle atom
 constexpr int kTcAtomBytes = kTcM * kTcAtom * 2;  // 16 KB of W1 per atom
 constexpr int kTcMaxAtoms = 8;     // atoms per CTA when all of them are loaded at once
-constexpr int kTcStages = 4;       // ring depth when the atoms of a CTA are streamed (large d_in)
-constexpr int kTcMaxKS = 8;        // CTAs per cluster
+constexpr int kTcStages = 5;       // ring depth when the atoms of a CTA are streamed (large d_in)
+constexpr int kTcMaxKS = 9;        // CTAs per cluster (non-portable above 8)
 constexpr int kTcThreads = 128;    // thread t = tile row t = TMEM lane t
 constexpr uint32_t kTcTmemCols = 64;
 constexpr int kTcMaxSmem = 200 * 1024;
@@ -501,7 +501,7 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     const int tiles = (a.hidden + kTcM - 1) / kTcM;
     const int groups = (a.num_reqs + kTcMaxN - 1) / kTcMaxN;
     const int npad = ((a.num_reqs < kTcMaxN ? a.num_reqs : kTcMaxN) + 15) / 16 * 16;
-    // split d_in over as many CTAs as one wave of SMs holds, 8 at most
+    // split d_in over as many CTAs as one wave of SMs holds, kTcMaxKS at most
     int ks = dev.sm_count / (tiles * groups);
     ks = ks < 1 ? 1 : ks;
     ks = ks > kTcMaxKS ? kTcMaxKS : ks;
@@ -541,6 +541,10 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
         if (cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+                cudaSuccess ||
+            cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
                 cudaSuccess)
             return BP_ERR_CUDA;
         configured[dev.device] = 1;
