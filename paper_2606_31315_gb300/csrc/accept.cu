@@ -184,7 +184,8 @@ __device__ __forceinline__ void wait_range(uint64_t* bar, int nw, unsigned int* 
 }
 
 // Scaled maximum l*c2 of a lane's entries of a range (-inf if none is finite), then the weights
-// 2^(l*c2 - m) replace the logits in place; returns (m, sum of the weights).
+// 2^(l*c2 - m) replace the logits in place (zeros when no entry is finite, so that pass 2 never
+// multiplies a -inf logit); returns (m, sum of the weights).
 __device__ __forceinline__ float2 weigh_range(float4* s, int w0, int nw, int Kw, int lane, float c2) {
     float m = -INFINITY;
     for (int j = 0; j < Kw; ++j) {
@@ -201,6 +202,11 @@ __device__ __forceinline__ float2 weigh_range(float4* s, int w0, int nw, int Kw,
                 sum += sum4(e);
                 s[w0 + f] = e;
             }
+        }
+    } else {
+        for (int j = 0; j < Kw; ++j) {
+            const int f = j * 32 + lane;
+            if (f < nw) s[w0 + f] = make_float4(0.f, 0.f, 0.f, 0.f);
         }
     }
     return make_float2(m, sum);

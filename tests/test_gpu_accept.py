@@ -137,3 +137,28 @@ def test_host_side_validation():
     with pytest.raises(bp.BlockPilotError) as e:
         bp.spec_accept(t, None, tok, cu, 1.0, torch.zeros(1, device="cuda"), torch.zeros(1, device="cuda"))
     assert e.value.status == 1  # T > 0 needs draft logits
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_masked_vocabulary(temp):
+    """Logits of -inf (a masked vocabulary: the first 40% and a band in the middle) in every row:
+    whole chunks of some lanes hold no finite entry, and the masked tokens must never be drawn."""
+    w = wl.custom(seed=45, ctx=(0,) * 4, block=(16, 9, 1, 5), vocab=151936)
+    inp = wl.accept_inputs(w, temp)
+    v = inp["target_logits"].shape[1]
+    masked = np.zeros(v, dtype=bool)
+    masked[: (4 * v) // 10] = True
+    masked[v // 2: v // 2 + 5000] = True
+    for key in ("target_logits", "draft_logits"):
+        inp[key] = inp[key].copy()
+        inp[key][:, masked] = -np.inf
+    # redraw the drafted tokens from the masked draft rows (Gumbel-max at T>0, argmax at T=0)
+    rng = np.random.default_rng([45, 99])
+    d = inp["draft_logits"] / (temp if temp > 0 else 1.0)
+    if temp > 0:
+        d = d + rng.gumbel(size=d.shape).astype(np.float32)
+    inp["draft_tokens"] = np.argmax(d, axis=1).astype(np.int32)
+    compare_accept(inp, temp)
+    _, out, _, _ = run_accept(inp, temp)
+    emitted = out[out >= 0]
+    assert not masked[emitted].any()
