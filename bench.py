@@ -50,6 +50,23 @@ def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
 
 
+def max_over_ranks(seconds: float, world: int, device=None) -> float:
+    """The slowest rank's time: the job's time (every rank ran the same number of steps)."""
+    if world <= 1:
+        return seconds
+    import torch
+    import torch.distributed as dist
+
+    t = torch.tensor([seconds], dtype=torch.float64, device=device)
+    dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    return float(t.item())
+
+
+def job_throughput(tokens_per_step: int, steps: int, seconds: float, world: int) -> float:
+    """Whole-job tokens/s: every rank verifies tokens_per_step tokens per step (weak scaling)."""
+    return world * tokens_per_step * steps / seconds
+
+
 # ----------------------------------------------------------------------------- byte counts
 def attention_bytes(w) -> float:
     """K and V read once, Q read and O written once (bf16)."""
@@ -232,15 +249,9 @@ def run_ours(args):
         e1.synchronize()
     torch.cuda.synchronize(dev)
     barrier()
-    elapsed = e0.elapsed_time(e1) / 1e3
-    if world > 1:
-        import torch.distributed as dist
-
-        tt = torch.tensor([elapsed], device=dev, dtype=torch.float64)
-        dist.all_reduce(tt, op=dist.ReduceOp.MAX)
-        elapsed = float(tt.item())
+    elapsed = max_over_ranks(e0.elapsed_time(e1) / 1e3, world, dev)
     tokens_per_step = int(np.sum(w.block))
-    value = world * tokens_per_step * args.steps / elapsed
+    value = job_throughput(tokens_per_step, args.steps, elapsed, world)
     ms_per_step = elapsed / args.steps * 1e3
     step_bytes = attention_bytes(w) + accept_bytes(w, 1.0)
     peak, peak_kind = peaks()
