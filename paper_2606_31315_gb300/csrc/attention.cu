@@ -16,7 +16,10 @@
 //     memory -- no global scratch, one launch.
 //   * Units are issued longest-first so that ragged batches finish together.
 //   Warp roles: warp 0 = TMA producer + TMEM allocator, warp 1 = MMA issuer,
-//   warps 2..5 = softmax / epilogue (one query row per thread, TMEM lane = row).
+//   warps 2..5 = softmax / epilogue (one query row per thread, TMEM lane = row).  Units of at
+//   most 64 rows (a block of up to 64/g positions) use the spread layout instead: the rows fill
+//   16 lanes of each TMEM sub-partition and each half-warp takes one 64-key half of a row, so
+//   all four softmax warps share the exp2 work.
 //
 // fp32 path: a plain SIMT kernel (one warp per output row, online softmax).
 #include <cooperative_groups.h>
@@ -85,7 +88,11 @@ __device__ __forceinline__ uint32_t cluster_size() {
 
 // PAGED: K/V rows come from pages named by p.block_table (the contiguous instantiation carries no
 // paging code at all).
-template <bool PAGED>
+// SPREAD (units of at most 64 query rows, group size dividing 16): logical row r sits at TMEM lane
+// (r / 16) * 32 + r % 16, so the 64 rows fill 16 lanes of each of the four TMEM sub-partitions and
+// all four softmax warps (and their SMSPs' exp2 units) work; the two half-warps take the two
+// 64-column halves of a row (tcgen05 16x32bx2 accesses), combining row statistics by shuffle.
+template <bool PAGED, bool SPREAD>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ CUtensorMap vmap, const AttnParams p) {
@@ -244,7 +251,15 @@ __global__ void __launch_bounds__(kThreads, 1)
     // inputs may be produced by the previous kernel on the stream: wait for it before any global access
     griddep_wait();
     if (tid == 0 && nt > 0) {  // the producer starts the Q load and fills the K/V ring
-        if (p.q_tma) {
+        if (SPREAD) {  // four boxes of 16 rows, at shared-memory rows 0, 32, 64, 96
+            mbar_arrive_expect_tx(&bar_q_full, kQBytes / 2);
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+                const int qrow = q0 + (row0 + 16 * qq) / G;
+                tma_load_3d(sQ + qq * 32 * 128, &qmap, &bar_q_full, 0, h * G, qrow);
+                tma_load_3d(sQ + kHalf + qq * 32 * 128, &qmap, &bar_q_full, 64, h * G, qrow);
+            }
+        } else if (p.q_tma) {
             mbar_arrive_expect_tx(&bar_q_full, kQBytes);
             const int qrow = q0 + row0 / G;
             tma_load_3d(sQ, &qmap, &bar_q_full, 0, h * G, qrow);
@@ -321,16 +336,20 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
     }
 
-    // ================= softmax / epilogue warps (2..5); row = TMEM lane
+    // ================= softmax / epilogue warps (2..5).  Dense: row r = TMEM lane quad*32 + lane, all
+    // columns.  SPREAD: row r = quad*16 + lane%16 at TMEM lane quad*32 + lane%16, columns of half lane/16.
+    constexpr int kCols = SPREAD ? kTileN / 2 : kTileN;  // S / P columns (keys) per thread
+    constexpr int kOCols = SPREAD ? kD / 2 : kD;         // O columns per thread
     const int quad = warp & 3;
-    const int r = quad * 32 + lane;
+    const int half = SPREAD ? (lane >> 4) : 0;
+    const int r = SPREAD ? quad * 16 + (lane & 15) : quad * 32 + lane;
     const bool is_softmax = warp >= 2;
     const bool row_active = is_softmax && r < m_valid;
-    const bool warp_active = is_softmax && (quad * 32 < m_valid);
+    const bool warp_active = is_softmax && ((SPREAD ? quad * 16 : quad * 32) < m_valid);
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
     const int limit = row_active ? (p.causal ? L + (row0 + r) / G + 1 : n) : 0;
-    float m_run = -INFINITY, l_run = 0.f;
-    float o_acc[kD];
+    float m_run = -INFINITY, l_run = 0.f;  // SPREAD: l_run is this half's share of the row sum
+    float o_acc[kOCols];
     bool failed = false;
 
     if (is_softmax) {
@@ -343,21 +362,23 @@ __global__ void __launch_bounds__(kThreads, 1)
             tc_fence_after();
             if (warp_active) {
                 const int nvalid = limit - (t_begin + j) * kTileN;
-                float x[kTileN];
+                float x[kCols];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
+                for (int c = 0; c < kCols / 32; ++c) {
                     uint32_t v[32];
-                    tmem_ld32(tmem + lane_base + col_s(sb) + c * 32, v);
+                    if (SPREAD) tmem_ld16x2_32<kTileN / 2>(tmem + lane_base + col_s(sb) + c * 32, v);
+                    else tmem_ld32(tmem + lane_base + col_s(sb) + c * 32, v);
                     tmem_ld_wait();
 #pragma unroll
                     for (int e = 0; e < 32; ++e) {
-                        const int kidx = c * 32 + e;
-                        x[kidx] = (kidx < nvalid) ? __uint_as_float(v[e]) * p.scale_log2 : -INFINITY;
+                        const int kidx = half * (kTileN / 2) + c * 32 + e;
+                        x[c * 32 + e] = (kidx < nvalid) ? __uint_as_float(v[e]) * p.scale_log2 : -INFINITY;
                     }
                 }
                 float mt_ = -INFINITY;
 #pragma unroll
-                for (int e = 0; e < kTileN; ++e) mt_ = fmaxf(mt_, x[e]);
+                for (int e = 0; e < kCols; ++e) mt_ = fmaxf(mt_, x[e]);
+                if (SPREAD) mt_ = fmaxf(mt_, __shfl_xor_sync(0xffffffffu, mt_, 16));
                 const float m_new = fmaxf(m_run, mt_);
                 const bool need = m_new > m_run + 8.f;
                 const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
@@ -369,18 +390,25 @@ __global__ void __launch_bounds__(kThreads, 1)
                     } else {
                         tc_fence_after();
 #pragma unroll
-                        for (int c = 0; c < 4; ++c) {
+                        for (int c = 0; c < kOCols / 32; ++c) {
                             uint32_t v[32];
-                            tmem_ld32(tmem + lane_base + kColO + c * 32, v);
+                            if (SPREAD) tmem_ld16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
+                            else tmem_ld32(tmem + lane_base + kColO + c * 32, v);
                             tmem_ld_wait();
-                            uint32_t w0[16], w1[16];
+                            if (SPREAD) {
 #pragma unroll
-                            for (int e = 0; e < 16; ++e) {
-                                w0[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-                                w1[e] = __float_as_uint(__uint_as_float(v[16 + e]) * alpha);
+                                for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+                                tmem_st16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
+                            } else {
+                                uint32_t w0[16], w1[16];
+#pragma unroll
+                                for (int e = 0; e < 16; ++e) {
+                                    w0[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+                                    w1[e] = __float_as_uint(__uint_as_float(v[16 + e]) * alpha);
+                                }
+                                tmem_st16(tmem + lane_base + kColO + c * 32, w0);
+                                tmem_st16(tmem + lane_base + kColO + c * 32 + 16, w1);
                             }
-                            tmem_st16(tmem + lane_base + kColO + c * 32, w0);
-                            tmem_st16(tmem + lane_base + kColO + c * 32 + 16, w1);
                         }
                     }
                 }
@@ -390,17 +418,29 @@ __global__ void __launch_bounds__(kThreads, 1)
                 }
                 float lsum = 0.f;
                 const bool any = m_run != -INFINITY;
+                if (SPREAD) {  // this half's 64 keys -> 32 packed P columns (the other half 32 further)
+                    uint32_t pk[32];
 #pragma unroll
-                for (int c = 0; c < 4; ++c) {
-                    uint32_t pk[16];
-#pragma unroll
-                    for (int e = 0; e < 16; ++e) {
-                        const float a = any ? fast_exp2(x[c * 32 + 2 * e] - m_run) : 0.f;
-                        const float b = any ? fast_exp2(x[c * 32 + 2 * e + 1] - m_run) : 0.f;
+                    for (int e = 0; e < 32; ++e) {
+                        const float a = any ? fast_exp2(x[2 * e] - m_run) : 0.f;
+                        const float b = any ? fast_exp2(x[2 * e + 1] - m_run) : 0.f;
                         lsum += a + b;
                         pk[e] = pack_bf16x2(a, b);
                     }
-                    tmem_st16(tmem + lane_base + col_s(sb) + c * 16, pk);
+                    tmem_st16x2_32<kTileN / 4>(tmem + lane_base + col_s(sb), pk);
+                } else {
+#pragma unroll
+                    for (int c = 0; c < 4; ++c) {
+                        uint32_t pk[16];
+#pragma unroll
+                        for (int e = 0; e < 16; ++e) {
+                            const float a = any ? fast_exp2(x[c * 32 + 2 * e] - m_run) : 0.f;
+                            const float b = any ? fast_exp2(x[c * 32 + 2 * e + 1] - m_run) : 0.f;
+                            lsum += a + b;
+                            pk[e] = pack_bf16x2(a, b);
+                        }
+                        tmem_st16(tmem + lane_base + col_s(sb) + c * 16, pk);
+                    }
                 }
                 l_run += lsum;
                 tmem_st_wait();
@@ -416,21 +456,23 @@ __global__ void __launch_bounds__(kThreads, 1)
         tc_fence_after();
         if (warp_active && nt > 0 && !failed) {
 #pragma unroll
-            for (int c = 0; c < 4; ++c) {
+            for (int c = 0; c < kOCols / 32; ++c) {
                 uint32_t v[32];
-                tmem_ld32(tmem + lane_base + kColO + c * 32, v);
+                if (SPREAD) tmem_ld16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
+                else tmem_ld32(tmem + lane_base + kColO + c * 32, v);
                 tmem_ld_wait();
 #pragma unroll
                 for (int e = 0; e < 32; ++e) o_acc[c * 32 + e] = __uint_as_float(v[e]);
             }
         } else {
 #pragma unroll
-            for (int e = 0; e < kD; ++e) o_acc[e] = 0.f;
+            for (int e = 0; e < kOCols; ++e) o_acc[e] = 0.f;
             if (nt == 0 || failed) {
                 m_run = -INFINITY;
                 l_run = 0.f;
             }
         }
+        if (SPREAD) l_run += __shfl_xor_sync(0xffffffffu, l_run, 16);  // the whole row's sum
     }
 
     const float kLn2 = 0.6931471805599453f;
@@ -440,9 +482,9 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int i = lr / G, jh = lr % G;
             const size_t orow = (size_t)(q0 + i) * p.num_q_heads + h * G + jh;
             const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-            __nv_bfloat16* dst = p.o + orow * kD;
+            __nv_bfloat16* dst = p.o + orow * kD + half * kOCols;
 #pragma unroll
-            for (int c = 0; c < kD / 8; ++c) {
+            for (int c = 0; c < kOCols / 8; ++c) {
                 uint4 w;
                 w.x = pack_bf16x2(o_acc[c * 8 + 0] * inv, o_acc[c * 8 + 1] * inv);
                 w.y = pack_bf16x2(o_acc[c * 8 + 2] * inv, o_acc[c * 8 + 3] * inv);
@@ -450,7 +492,7 @@ __global__ void __launch_bounds__(kThreads, 1)
                 w.w = pack_bf16x2(o_acc[c * 8 + 6] * inv, o_acc[c * 8 + 7] * inv);
                 *reinterpret_cast<uint4*>(dst + c * 8) = w;
             }
-            if (p.lse) p.lse[orow] = (m_run + __log2f(l_run)) * kLn2;
+            if (p.lse && half == 0) p.lse[orow] = (m_run + __log2f(l_run)) * kLn2;
         }
     } else {
         // ---- merge of the CS partial (m, l, O) triples through distributed shared memory.  After the
@@ -465,13 +507,13 @@ __global__ void __launch_bounds__(kThreads, 1)
         if (is_softmax) {
             if (row_active) {
 #pragma unroll
-                for (int c = 0; c < kD / 4; ++c) {
-                    const int pc = c ^ (r & 31);
+                for (int c = 0; c < kOCols / 4; ++c) {
+                    const int pc = (half * (kOCols / 4) + c) ^ (r & 31);
                     *reinterpret_cast<float4*>(opart + r * kD + pc * 4) =
                         make_float4(o_acc[c * 4], o_acc[c * 4 + 1], o_acc[c * 4 + 2], o_acc[c * 4 + 3]);
                 }
             }
-            row_ml[r] = make_float2(m_run, l_run);
+            if (half == 0) row_ml[r] = make_float2(m_run, l_run);
         }
         cluster.sync();
         const int per = (m_valid + (int)CS - 1) / (int)CS;
@@ -627,12 +669,14 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     if (units == 0 || a.total_q == 0) return BP_OK;
 
     CUtensorMap qmap, kmap, vmap;
-    // Q: box of (64 columns) x (G heads) x (128/G block positions) = the packed 128-row tile
+    // Q: box of (64 columns) x (G heads) x (128/G block positions) = the packed 128-row tile; for units
+    // of at most 64 rows (spread layout) four boxes of 16 rows (16/G block positions) instead
     const bool q_tma = (kM % G == 0);
+    const bool spread = q_tma && 16 % G == 0 && (long long)a.max_q_len * G <= 64;
     if (q_tma) {
         const cuuint64_t qdims[3] = {(cuuint64_t)kD, (cuuint64_t)a.num_q_heads, (cuuint64_t)a.total_q};
         const cuuint64_t qstrides[2] = {(cuuint64_t)kD * 2, (cuuint64_t)a.num_q_heads * kD * 2};
-        const cuuint32_t qbox[3] = {64, (cuuint32_t)G, (cuuint32_t)(kM / G)};
+        const cuuint32_t qbox[3] = {64, (cuuint32_t)G, (cuuint32_t)((spread ? 16 : kM) / G)};
         const int rq = encode_tensor_map(&qmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 3, const_cast<void*>(a.q), qdims,
                                          qstrides, qbox, CU_TENSOR_MAP_SWIZZLE_128B);
         if (rq != BP_OK) return rq;
@@ -679,7 +723,8 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     static int configured_device = -1;
     static int max_active[kMaxCluster + 1];
     if (configured_device != dev.device) {
-        for (auto kern : {attn_bf16_tc_kernel<false>, attn_bf16_tc_kernel<true>})
+        for (auto kern : {attn_bf16_tc_kernel<false, false>, attn_bf16_tc_kernel<true, false>,
+                          attn_bf16_tc_kernel<false, true>, attn_bf16_tc_kernel<true, true>})
             if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) != cudaSuccess ||
                 cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
                 cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -698,7 +743,8 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
             probe.attrs = pa;
             probe.numAttrs = 1;
             int n_clusters = 0;
-            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel<false>, &probe) != cudaSuccess) {
+            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel<false, false>, &probe) !=
+                cudaSuccess) {
                 cudaGetLastError();
                 n_clusters = 0;
             }
@@ -735,8 +781,11 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    const cudaError_t e = paged ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true>, qmap, kmap, vmap, p)
-                                : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false>, qmap, kmap, vmap, p);
+    cudaError_t e;
+    if (paged) e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, true>, qmap, kmap, vmap, p)
+                          : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, false>, qmap, kmap, vmap, p);
+    else e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, true>, qmap, kmap, vmap, p)
+                    : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, false>, qmap, kmap, vmap, p);
     if (e != cudaSuccess) return BP_ERR_CUDA;
     return BP_OK;
 }
