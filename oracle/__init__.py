@@ -1,7 +1,8 @@
 """BlockPilot fp64 CPU oracle -- test infrastructure only.
 
 A plain, slow restatement of the block-verify hot path (block attention, lossless
-speculative acceptance, block-size policy head) written from the paper, in fp64.
+speculative acceptance, block-size policy head, and the LM-head projection that
+feeds the acceptance) written from the paper, in fp64.
 Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline leg
 may import this package; the product path never does.  It shares no code with the
 CUDA library.  The arithmetic lives in ``bpo.c``; this module only marshals numpy
@@ -56,6 +57,9 @@ def _load():
         lib.bpo_policy_select.argtypes = [dp, ctypes.c_long, ip, ctypes.c_int, ctypes.c_int, dp, dp,
                                           ctypes.c_int, dp, dp, ctypes.c_int, ip, dp, ip, dp]
         lib.bpo_policy_select.restype = ctypes.c_int
+        u16 = ctypes.POINTER(ctypes.c_uint16)
+        lib.bpo_lm_head_logits.argtypes = [u16, u16, ctypes.c_int, ctypes.c_int, ctypes.c_int, dp, dp]
+        lib.bpo_lm_head_logits.restype = ctypes.c_int
         lib.bpo_num_threads.argtypes = []
         lib.bpo_num_threads.restype = ctypes.c_int
         _lib = lib
@@ -155,6 +159,46 @@ def policy_select(feats, w1, b1, w2, b2, candidates, row_index=None):
     if rc != 0:
         raise ValueError(f"oracle policy_select rejected its arguments (rc={rc})")
     return dict(block_size=bs, logits=lo, top2_margin=mg)
+
+
+
+def lm_head_logits(w_bits, h_bits, with_abs: bool = False):
+    """fp64 logits = h @ W^T of bf16 operands given as uint16 bits.
+
+    w_bits: [V, H]; h_bits: [rows, H].  Returns logits [rows, V] (and, with with_abs,
+    sum_k |W[v,k] h[r,k]| of the same shape, the scale of any fp32 rounding error).
+    """
+    w = np.ascontiguousarray(w_bits, dtype=np.uint16)
+    h = np.ascontiguousarray(h_bits, dtype=np.uint16).reshape(-1, w.shape[1])
+    rows, (vocab, hidden) = h.shape[0], w.shape
+    out = np.zeros((rows, vocab), dtype=np.float64)
+    mag = np.zeros((rows, vocab), dtype=np.float64) if with_abs else None
+    u16 = ctypes.c_uint16
+    rc = _load().bpo_lm_head_logits(_p(w, u16), _p(h, u16), rows, vocab, hidden, _p(out, ctypes.c_double),
+                                    _p(mag, ctypes.c_double))
+    if rc != 0:
+        raise ValueError(f"oracle lm_head_logits rejected its arguments (rc={rc})")
+    return (out, mag) if with_abs else out
+
+
+def verify_epilogue(w_bits, h_target_bits, h_draft_bits, draft_tokens, cu_draft, temperature: float,
+                    u_accept=None, u_sample=None, with_abs: bool = False):
+    """The verify step from final hidden states: LM-head logits of the target rows (and, at
+    T > 0, of the drafter's rows) followed by the lossless acceptance over them.
+
+    Returns spec_accept's dict plus target_logits / draft_logits (fp64) and, with with_abs,
+    target_abs / draft_abs (the error scales of lm_head_logits).
+    """
+    greedy = temperature == 0.0
+    t = lm_head_logits(w_bits, h_target_bits, with_abs)
+    d = None if greedy or h_draft_bits is None else lm_head_logits(w_bits, h_draft_bits, with_abs)
+    tl, ta = t if with_abs else (t, None)
+    dl, da = (d if with_abs else (d, None)) if d is not None else (None, None)
+    res = spec_accept(tl, dl, draft_tokens, cu_draft, temperature, u_accept, u_sample)
+    res.update(target_logits=tl, draft_logits=dl)
+    if with_abs:
+        res.update(target_abs=ta, draft_abs=da)
+    return res
 
 
 if __name__ == "__main__":  # pragma: no cover

@@ -9,15 +9,20 @@
  * double precision, with the loops in the order the definition states them.
  *
  * Inputs arrive as fp64 arrays that hold the exact values the GPU path sees
- * (bf16 / fp32 values widened without rounding).  Random numbers the method
+ * (bf16 / fp32 values widened without rounding); the LM-head projection takes
+ * its bf16 operands as raw bits and widens them itself (the weight has 389 M
+ * entries).  Random numbers the method
  * draws (the acceptance uniforms and the resampling uniform) are inputs.
  *
- * Three parts, one per hot-path stage:
+ * Four parts, one per hot-path stage:
  *   bpo_block_attention  -- block attention of a B-token block over a KV cache,
  *                           causal within the block (target verify pass) or
  *                           bidirectional within the block (dLLM drafter pass).
  *   bpo_spec_accept      -- lossless speculative acceptance of a drafted block.
  *   bpo_policy_select    -- the once-per-request block-size predictor.
+ *   bpo_lm_head_logits   -- the output projection that turns the final hidden
+ *                           states of the verified (and drafted) positions into
+ *                           the logits the acceptance reads.
  *
  * Readings of the paper where it is silent are documented at each function.
  */
@@ -365,6 +370,68 @@ int bpo_policy_select(const double *feats, long row_stride,
         free(o);
     }
     return BPO_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* LM head: final hidden states -> logits                                     */
+/* ------------------------------------------------------------------------- */
+/*
+ * Section 2.1 and the Figure 1 caption: the target scores every position of
+ * the drafted block in one parallel pass, and the acceptance compares its
+ * distributions with the drafter's.  The paper does not print the model's
+ * output layer; both distributions come from the standard LM head, a linear
+ * map of the position's final hidden state h (dimension H) onto the
+ * vocabulary:
+ *
+ *   logits[r][v] = sum_{k < H} W[v][k] * h[r][k]        (v < V)
+ *
+ * W is [V][H] row-major, h is [rows][H] row-major, both bf16 given as raw
+ * bits and widened exactly; the sum is formed in fp64 in index order.
+ * abs_dot (may be NULL) receives sum_k |W[v][k] * h[r][k]|, the magnitude
+ * that bounds the rounding error of any lower-precision evaluation of the
+ * same sum.
+ */
+static double bf16_bits_to_double(uint16_t b)
+{
+    union { uint32_t u; float f; } x;
+    x.u = (uint32_t)b << 16;
+    return (double)x.f;
+}
+
+int bpo_lm_head_logits(const uint16_t *w, const uint16_t *h, int rows, int vocab,
+                       int hidden, double *logits, double *abs_dot)
+{
+    if (!w || !h || !logits || rows < 0 || vocab < 1 || hidden < 1) return BPO_BAD_ARG;
+    double *hd = (double *)malloc(sizeof(double) * (size_t)(rows > 0 ? rows : 1) * (size_t)hidden);
+    if (!hd) return BPO_BAD_ARG;
+    for (size_t i = 0; i < (size_t)rows * (size_t)hidden; ++i) hd[i] = bf16_bits_to_double(h[i]);
+    int bad = 0;
+#pragma omp parallel
+    {
+        double *wr = (double *)malloc(sizeof(double) * (size_t)hidden);
+        if (!wr) {
+#pragma omp atomic write
+            bad = 1;
+        }
+#pragma omp for schedule(static)
+        for (int v = 0; v < vocab; ++v) {
+            if (!wr) continue;
+            for (int k = 0; k < hidden; ++k) wr[k] = bf16_bits_to_double(w[(size_t)v * hidden + k]);
+            for (int r = 0; r < rows; ++r) {
+                const double *hr = hd + (size_t)r * hidden;
+                double acc = 0.0, mag = 0.0;
+                for (int k = 0; k < hidden; ++k) {
+                    acc += wr[k] * hr[k];
+                    mag += fabs(wr[k] * hr[k]);
+                }
+                logits[(size_t)r * vocab + v] = acc;
+                if (abs_dot) abs_dot[(size_t)r * vocab + v] = mag;
+            }
+        }
+        free(wr);
+    }
+    free(hd);
+    return bad ? BPO_BAD_ARG : BPO_OK;
 }
 
 /* Number of OpenMP threads the oracle's parallel loops use (1 without OpenMP). */

@@ -228,6 +228,61 @@ def policy_inputs(w: Workload) -> dict:
     return out
 
 
+# hidden size of the final states the LM head projects (Qwen3-4B: 2560)
+LM_HIDDEN = {"tiny": 128, "qwen3_4b": 2560, "ragged": 2560, "long_context": 2560}
+
+
+def lm_head_weight(vocab: int, hidden: int, logit_std: float, seed: int) -> np.ndarray:
+    """LM-head weight [V, H] ~ N(0, logit_std^2 / H) as bf16 bits (so unit-variance states get
+    logits ~ N(0, logit_std^2)); drawn and rounded in chunks of rows to bound host memory."""
+    rng = _rng(seed, 50)
+    out = np.empty((vocab, hidden), dtype=np.uint16)
+    scale = np.float32(logit_std / np.sqrt(hidden))
+    step = max(1, (1 << 24) // hidden)
+    for r0 in range(0, vocab, step):
+        r1 = min(vocab, r0 + step)
+        out[r0:r1] = f32_to_bf16_bits(rng.standard_normal((r1 - r0, hidden), dtype=np.float32) * scale)
+    return out
+
+
+def lm_head_inputs(w: Workload, temperature: float, hidden: int | None = None, push_prob: float = 0.85,
+                   boost: float = 18.0, weight: np.ndarray | None = None) -> dict:
+    """LM-head weight, the final hidden states the verify epilogue projects, draft tokens, uniforms.
+
+    W [V, H] from lm_head_weight.  Target states [sum (gamma_s + 1), H] ~ N(0, 1).  Draft token x_i
+    is uniform over V.  The drafter's state of position i is its target row's state plus
+    N(0, 1 / logit_std^2) noise (its logits are the target's plus unit-variance noise) plus
+    boost * w_x / |w_x|^2, which raises the drafter's logit of x_i by `boost`; with probability
+    push_prob the target row's state gets the same push (the target agrees with the draft),
+    otherwise none.  States are rounded to bf16 last.  At T = 0 the drafter's states are not
+    returned (greedy acceptance reads the target rows only).
+    """
+    gammas = np.asarray(w.block, dtype=np.int64) - 1
+    cu_draft = offsets(gammas)
+    s = w.num_seqs
+    td = int(cu_draft[-1])
+    V = w.vocab
+    H = hidden or LM_HIDDEN.get(w.name, 256)
+    W = weight if weight is not None else lm_head_weight(V, H, w.logit_std, w.seed)
+    base = _rng(w.seed, 51).standard_normal((td + s, H)).astype(np.float64)
+    noise = _rng(w.seed, 52).standard_normal((td, H)) / w.logit_std
+    tokens = _rng(w.seed, 53).integers(0, V, size=td).astype(np.int32)
+    push = _rng(w.seed, 54).random(td) < push_prob
+    seq_of_draft = np.repeat(np.arange(s), gammas)
+    trow = np.arange(td) + seq_of_draft  # target row of drafted position i
+    wx = bf16_bits_to_f32(W[tokens]).astype(np.float64) if td else np.zeros((0, H))
+    dirs = wx / np.maximum((wx * wx).sum(axis=1, keepdims=True), 1e-30) * boost
+    h_draft = base[trow] + noise + dirs
+    h_target = base.copy()
+    h_target[trow[push]] += dirs[push]
+    out = dict(w=W, hidden=H, h_target=f32_to_bf16_bits(h_target.astype(np.float32)), draft_tokens=tokens,
+               cu_draft=cu_draft, vocab=V, temperature=float(temperature),
+               u_accept=_rng(w.seed, 55).random(td, dtype=np.float32),
+               u_sample=_rng(w.seed, 56).random(s, dtype=np.float32))
+    out["h_draft"] = f32_to_bf16_bits(h_draft.astype(np.float32)) if temperature > 0.0 else None
+    return out
+
+
 def as_f64(x: np.ndarray, dtype: str) -> np.ndarray:
     """The exact fp64 values of an f32 array or of bf16 bits."""
     if dtype == "bf16":
