@@ -321,6 +321,62 @@ def run_ours(args):
     big_bytes = float(big["w1"].numel() * 2 + big["feats"].numel() * 2 + big["w2"].numel() * 2)
     del big, g_big
 
+    # next row: the LM head fused with the acceptance -- the Qwen3-4B LM head (151936 x 2560 bf16,
+    # 778 MB, far larger than L2) over the batch-1 step's 16 target and 15 drafter states at T=1;
+    # beside it the unfused path (cuBLAS bf16 GEMM to logits, fp32 cast, acceptance kernel)
+    lm_h, td_q = 2560, int(w.block[0]) - 1
+    w_lm = (torch.randn(w.vocab, lm_h, device=dev, generator=gen) * (w.logit_std / lm_h ** 0.5)).to(torch.bfloat16)
+    h_t = torch.randn(td_q + 1, lm_h, device=dev, generator=gen).to(torch.bfloat16)
+    h_d = (h_t[:td_q].float() + torch.randn(td_q, lm_h, device=dev, generator=gen) / w.logit_std).to(torch.bfloat16)
+    ve_tok = torch.randint(0, w.vocab, (td_q,), device=dev, generator=gen, dtype=torch.int32)
+    ve_cu = torch.tensor([0, td_q], dtype=torch.int32, device=dev)
+    ve_ua, ve_us = torch.rand(td_q, device=dev, generator=gen), torch.rand(1, device=dev, generator=gen)
+    ve_n, ve_o = torch.empty(1, dtype=torch.int32, device=dev), torch.empty(td_q + 1, dtype=torch.int32, device=dev)
+    ws_ve = bp.workspace(bp.verify_epilogue_workspace_size(1, td_q), dev)
+
+    def fused(_c):
+        bp.verify_epilogue(w_lm, h_t, h_d, ve_tok, ve_cu, 1.0, ve_ua, ve_us, n_accepted=ve_n, out_tokens=ve_o,
+                           want_accept_prob=False, ws=ws_ve, stream=stream)
+
+    h_all = torch.cat([h_t, h_d])
+    lg = torch.empty(2 * td_q + 1, w.vocab, dtype=torch.float32, device=dev)
+    ws_u = bp.workspace(bp.spec_accept_workspace_size(1, td_q, w.vocab), dev)
+
+    def unfused(_c):
+        with torch.cuda.stream(stream):
+            lg.copy_(torch.matmul(h_all, w_lm.t()))
+        bp.spec_accept(lg[:td_q + 1], lg[td_q + 1:], ve_tok, ve_cu, 1.0, ve_ua, ve_us, n_accepted=ve_n,
+                       out_tokens=ve_o, want_accept_prob=False, ws=ws_u, stream=stream)
+
+    def time_calls(fn, n_graph=4, reps=10):
+        """Seconds per call: replays of a graph of n_graph calls, or timed eager calls if the launch
+        cannot be captured."""
+        with torch.cuda.stream(stream):
+            for _ in range(3):
+                fn(None)
+        stream.synchronize()
+        try:
+            g = torch.cuda.CUDAGraph()
+            with torch.cuda.graph(g, stream=stream):
+                for _ in range(n_graph):
+                    fn(None)
+            return time_graph(g, reps) / n_graph
+        except RuntimeError:
+            torch.cuda.synchronize(dev)
+            e0, e1 = torch.cuda.Event(enable_timing=True), torch.cuda.Event(enable_timing=True)
+            with torch.cuda.stream(stream):
+                e0.record(stream)
+                for _ in range(reps * n_graph):
+                    fn(None)
+                e1.record(stream)
+            e1.synchronize()
+            return e0.elapsed_time(e1) / 1e3 / (reps * n_graph)
+
+    t_ve = time_calls(fused)
+    t_unfused = time_calls(unfused)
+    ve_bytes = float(w_lm.numel() * 2 + h_all.numel() * 2)
+    del w_lm, lg
+
     def row(tsec, nbytes, kernels):
         gbs = nbytes / tsec / 1e9
         return {"us": round(tsec * 1e6, 3), "bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
@@ -335,6 +391,10 @@ def run_ours(args):
         "next3_verify_attention_paged_page64": row(t_attn_paged, attention_bytes(w), ["attn_bf16_tc_kernel (paged)"]),
         "next2_policy_head_32req_151936x2048": row(t_pol_big, big_bytes,
                                                    ["policy_gather_kernel", "policy_tc_kernel (streamed)"]),
+        "next1_fused_verify_epilogue_qwen3_4b_t1": dict(
+            row(t_ve, ve_bytes, ["verify_epilogue_kernel<false,32>"]),
+            unfused_us=round(t_unfused * 1e6, 3),
+            unfused="cuBLAS bf16 GEMM to logits + fp32 cast + accept_kernel"),
     }
     dom_name, dom_t, dom_bytes = ("accept_kernel", t_acc, accept_bytes(w, 1.0))
     traffic = committed_traffic(dom_name)

@@ -15,6 +15,8 @@
  *
  * bp_block_attention_paged and bp_kv_append run the attention over a paged KV cache (pages of
  * a shared pool named by a per-sequence block table) and append a block's K/V to it.
+ * bp_verify_epilogue fuses the LM head that produces the logits with bp_spec_accept: it takes
+ * the final hidden states of the verified and drafted positions instead of their logits.
  *
  * Conventions shared by every entry point
  *   - Pointers to tensors are DEVICE pointers (cudaMalloc / torch allocations), owned by
@@ -43,7 +45,7 @@
 extern "C" {
 #endif
 
-#define BP_ABI_VERSION 2
+#define BP_ABI_VERSION 3
 
 /* Symbols of the ABI are exported; everything else in the library is hidden. */
 #if defined(__GNUC__)
@@ -222,6 +224,41 @@ BP_API int bp_policy_select(const void* feats, int64_t feat_row_stride, const in
                      const void* w1, const float* b1, int hidden, const void* w2, const float* b2, int num_cand,
                      const int32_t* candidates, int wdtype, float* logits_out, int32_t* block_size_out,
                      void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------
+ * Verify epilogue: the LM-head projection of the final hidden states fused with the lossless
+ * acceptance of bp_spec_accept, without writing the logits to memory.  Section 2.1 and the
+ * Figure 1 caption: the target scores every position of the drafted block in one pass and
+ * keeps the longest accepted prefix; the distributions it compares are
+ *
+ *   p_i = softmax(W h_target_i / T),  q_i = softmax(W h_draft_i / T)
+ *
+ * with W the [vocab][hidden] LM head shared by the target and the drafter.  The acceptance,
+ * its outputs and its conventions are those of bp_spec_accept applied to target_logits =
+ * h_target W^T and draft_logits = h_draft W^T (fp32 accumulation of bf16 products).
+ *
+ *   lm_head      [vocab][hidden] bf16, 16-byte aligned
+ *   h_target     [total_draft + num_seqs][hidden] bf16: the target's final states, rows in the
+ *                target-row order of bp_spec_accept; 16-byte aligned
+ *   h_draft      [total_draft][hidden] bf16: the drafter's final states at its drafted
+ *                positions; NULL allowed iff temperature == 0
+ *   draft_tokens, cu_draft, u_accept, u_sample, n_accepted, out_tokens, accept_prob: as in
+ *                bp_spec_accept
+ *   logits_out   [rows][vocab] fp32, may be NULL: if given, the logits are also written (rows:
+ *                the target rows, then at T > 0 the drafter rows) -- for testing; it adds the
+ *                write traffic the fusion exists to avoid
+ * Limits (else BP_ERR_UNSUPPORTED): hidden % 64 == 0; rows = total_draft + num_seqs (+
+ * total_draft at T > 0) <= 64; the vocabulary split over the SMs must leave each CTA at most
+ * 16 tiles of 128 entries and tiles x (32 if rows <= 32 else 64) <= 512 tensor-memory columns
+ * (152 SMs: vocab <= 155,648 at rows <= 64, 311,296 at rows <= 32).  The kernel is a
+ * cooperative launch of one CTA per SM.
+ * ------------------------------------------------------------------------------- */
+BP_API size_t bp_verify_epilogue_workspace_size(int num_seqs, int total_draft);
+BP_API int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_draft, int hidden, int vocab,
+                              const int32_t* draft_tokens, const int32_t* cu_draft, int num_seqs, int total_draft,
+                              float temperature, const float* u_accept, const float* u_sample,
+                              int32_t* n_accepted, int32_t* out_tokens, float* accept_prob, float* logits_out,
+                              void* workspace, size_t workspace_bytes, void* stream);
 
 /* Reads and clears the sticky device error word of `workspace` (synchronizes `stream`).
  * Returns BP_OK, BP_ERR_TIMEOUT or BP_ERR_DEVICE_FLAG (or BP_ERR_CUDA if the read fails). */

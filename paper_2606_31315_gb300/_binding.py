@@ -72,6 +72,11 @@ def load():
     lib.bp_policy_select_workspace_size.restype = sz
     lib.bp_policy_select.argtypes = [vp, i64, vp, i32, i32, vp, vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, sz, vp]
     lib.bp_policy_select.restype = i32
+    lib.bp_verify_epilogue_workspace_size.argtypes = [i32, i32]
+    lib.bp_verify_epilogue_workspace_size.restype = sz
+    lib.bp_verify_epilogue.argtypes = [vp, vp, vp, i32, i32, vp, vp, i32, i32, f32, vp, vp, vp, vp, vp, vp, vp, sz,
+                                       vp]
+    lib.bp_verify_epilogue.restype = i32
     lib.bp_get_status.argtypes = [vp, vp]
     lib.bp_get_status.restype = i32
     _lib = lib
@@ -209,6 +214,42 @@ def spec_accept(target_logits, draft_logits, draft_tokens, cu_draft, temperature
                             total_draft, vocab, float(temperature), _ptr(u_accept), _ptr(u_sample), _ptr(n_accepted),
                             _ptr(out_tokens), _ptr(accept_prob), _ptr(ws), ws.numel(), _stream(stream))
     _check(rc, "bp_spec_accept")
+    return n_accepted, out_tokens, accept_prob
+
+
+# --------------------------------------------------------------------------- verify epilogue
+def verify_epilogue_workspace_size(num_seqs, total_draft) -> int:
+    return int(load().bp_verify_epilogue_workspace_size(num_seqs, total_draft))
+
+
+def verify_epilogue(lm_head, h_target, h_draft, draft_tokens, cu_draft, temperature: float, u_accept=None,
+                    u_sample=None, n_accepted=None, out_tokens=None, accept_prob=None, want_accept_prob=True,
+                    logits_out=None, ws=None, stream=None):
+    """LM head fused with the lossless acceptance; see ``bp_verify_epilogue``.  Returns
+    (n_accepted, out_tokens, accept_prob)."""
+    lib = load()
+    for t, n in ((lm_head, "lm_head"), (h_target, "h_target"), (h_draft, "h_draft"), (draft_tokens, "draft_tokens"),
+                 (cu_draft, "cu_draft"), (u_accept, "u_accept"), (u_sample, "u_sample"), (logits_out, "logits_out")):
+        _cuda(t, n)
+    if lm_head.dtype != torch.bfloat16 or h_target.dtype != torch.bfloat16:
+        raise TypeError("verify_epilogue: lm_head and the hidden states must be bf16")
+    s = cu_draft.numel() - 1
+    total_draft = draft_tokens.numel()
+    vocab, hidden = lm_head.shape
+    dev = lm_head.device
+    if n_accepted is None:
+        n_accepted = torch.empty(s, dtype=torch.int32, device=dev)
+    if out_tokens is None:
+        out_tokens = torch.empty(total_draft + s, dtype=torch.int32, device=dev)
+    if accept_prob is None and want_accept_prob:
+        accept_prob = torch.empty(total_draft, dtype=torch.float32, device=dev)
+    if ws is None:
+        ws = workspace(lib.bp_verify_epilogue_workspace_size(s, total_draft), dev)
+    rc = lib.bp_verify_epilogue(_ptr(lm_head), _ptr(h_target), _ptr(h_draft), hidden, vocab, _ptr(draft_tokens),
+                                _ptr(cu_draft), s, total_draft, float(temperature), _ptr(u_accept), _ptr(u_sample),
+                                _ptr(n_accepted), _ptr(out_tokens), _ptr(accept_prob), _ptr(logits_out), _ptr(ws),
+                                ws.numel(), _stream(stream))
+    _check(rc, "bp_verify_epilogue")
     return n_accepted, out_tokens, accept_prob
 
 

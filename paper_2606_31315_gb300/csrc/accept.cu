@@ -27,6 +27,7 @@
 
 #include "common.cuh"
 #include "ptx_sm103.cuh"
+#include "softmax_math.cuh"
 
 namespace cg = cooperative_groups;
 
@@ -58,58 +59,6 @@ struct AccParams {
     int wr;        // float4 slots per warp range of a slice
     unsigned int* err;
 };
-
-__device__ __forceinline__ float ex2(float x) {
-    float y;
-    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
-    return y;
-}
-// 2^(a - b) for scaled log-values, 0 when a is -inf
-__device__ __forceinline__ float ex2d(float a, float b) { return a == -INFINITY ? 0.f : ex2(__fsub_rn(a, b)); }
-
-// Probability mass in 2^-52 units: segment, slice and row sums are exact integer additions
-// (a row's masses add up to about 1, i.e. about 2^52 units, far from the 2^64 limit).  Built
-// from the float's fields with integer shifts (truncating below 2^-52): the float -> 64-bit
-// integer conversion instruction runs on the slow FP64 pipe of this GPU.
-__device__ __forceinline__ unsigned long long to_fix(float x) {
-    const unsigned bits = __float_as_uint(x);
-    const int e = (int)((bits >> 23) & 0xffu);  // x = mant * 2^(e - 150) for normal x >= 0
-    if (e == 0 || (bits >> 31)) return 0ull;      // zero, denormal (< 2^-126) or negative
-    const unsigned long long mant = (unsigned long long)((bits & 0x7fffffu) | 0x800000u);
-    const int sh = e - 98;                         // x * 2^52 = mant * 2^(e - 98)
-    if (sh >= 0) return sh < 40 ? mant << sh : ~0ull;  // x >= 2^12 is out of range: saturate
-    return sh > -24 ? mant >> (-sh) : 0ull;
-}
-
-__device__ __forceinline__ float warp_incl_scan_f(float v, int lane) {
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const float y = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= o) v += y;
-    }
-    return v;
-}
-__device__ __forceinline__ unsigned long long warp_incl_scan(unsigned long long v, int lane) {
-#pragma unroll
-    for (int o = 1; o < 32; o <<= 1) {
-        const unsigned long long y = __shfl_up_sync(0xffffffffu, v, o);
-        if (lane >= o) v += y;
-    }
-    return v;
-}
-// merge two (scaled max, sum) pairs of a log-sum-exp
-__device__ __forceinline__ void lse_merge(float& m, float& s, float m2, float s2) {
-    const float M = fmaxf(m, m2);
-    s = s * ex2d(m, M) + s2 * ex2d(m2, M);
-    m = M;
-}
-// argmax with the lowest index winning ties
-__device__ __forceinline__ void amax_merge(float& v, int& i, float v2, int i2) {
-    if (v2 > v || (v2 == v && i2 < i)) {
-        v = v2;
-        i = i2;
-    }
-}
 
 __device__ __forceinline__ int atomic_add_acq_rel(int* addr, int v) {
     int old;

@@ -275,6 +275,47 @@ int bp_spec_accept_noalloc(const float* target_logits, const float* draft_logits
     return rc;
 }
 
+size_t bp_verify_epilogue_workspace_size(int num_seqs, int total_draft) {
+    if (num_seqs < 0 || total_draft < 0) return 0;
+    return sizeof(WorkspaceHeader) + verify_epilogue_scratch_bytes(num_seqs, total_draft);
+}
+
+int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_draft, int hidden, int vocab,
+                       const int32_t* draft_tokens, const int32_t* cu_draft, int num_seqs, int total_draft,
+                       float temperature, const float* u_accept, const float* u_sample, int32_t* n_accepted,
+                       int32_t* out_tokens, float* accept_prob, float* logits_out, void* workspace,
+                       size_t workspace_bytes, void* stream) {
+    if (num_seqs < 0 || total_draft < 0 || vocab < 1 || hidden < 1) return BP_ERR_INVALID_ARG;
+    if (num_seqs == 0) return BP_OK;
+    if (!lm_head || !h_target || !cu_draft || !n_accepted || !out_tokens || (total_draft > 0 && !draft_tokens))
+        return BP_ERR_INVALID_ARG;
+    if (!(temperature >= 0.f) || isinf(temperature)) return BP_ERR_INVALID_ARG;
+    const bool greedy = temperature == 0.f;
+    if (!greedy && (!u_sample || (total_draft > 0 && (!h_draft || !u_accept)))) return BP_ERR_INVALID_ARG;
+    if (hidden % 64 != 0) return BP_ERR_UNSUPPORTED;
+    if (!aligned(lm_head, 16) || !aligned(h_target, 16) || (!greedy && h_draft && !aligned(h_draft, 16)))
+        return BP_ERR_UNSUPPORTED;
+    const long long rows = (long long)total_draft + num_seqs + (greedy ? 0 : total_draft);
+    if (rows > 64) return BP_ERR_UNSUPPORTED;
+    int rc = check_workspace(workspace, workspace_bytes, bp_verify_epilogue_workspace_size(num_seqs, total_draft));
+    if (rc != BP_OK) return rc;
+    DeviceInfo dev;
+    if ((rc = device_info(&dev)) != BP_OK) return rc;
+    int grid, np, per;
+    if ((rc = verify_epilogue_config((int)rows, vocab, dev.sm_count, &grid, &np, &per)) != BP_OK) return rc;
+    VerifyEpilogueArgs a;
+    a.lm_head = lm_head; a.h_target = h_target; a.h_draft = h_draft;
+    a.hidden = hidden; a.vocab = vocab; a.num_seqs = num_seqs; a.total_draft = total_draft;
+    a.temperature = temperature;
+    a.tokens = draft_tokens; a.cu_draft = cu_draft; a.u_accept = u_accept; a.u_sample = u_sample;
+    a.n_accepted = n_accepted; a.out_tokens = out_tokens; a.accept_prob = accept_prob; a.logits_out = logits_out;
+    a.scratch = scratch(workspace);
+    a.err_word = err_word(workspace);
+    rc = launch_verify_epilogue(a, dev, static_cast<cudaStream_t>(stream));
+    if (rc == BP_ERR_CUDA) cudaGetLastError();
+    return rc;
+}
+
 size_t bp_policy_select_workspace_size(int num_reqs, int d_in, int hidden, int num_cand) {
     if (num_reqs < 0 || d_in < 1 || hidden < 1 || num_cand < 1) return 0;
     return sizeof(WorkspaceHeader) + policy_scratch_bytes(num_reqs, d_in, hidden, num_cand);

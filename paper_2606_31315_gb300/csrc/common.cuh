@@ -116,4 +116,26 @@ struct PolicyArgs {
 size_t policy_scratch_bytes(int num_reqs, int d_in, int hidden, int num_cand);
 int launch_policy(const PolicyArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
+struct VerifyEpilogueArgs {
+    const void* lm_head;   // [vocab][hidden] bf16
+    const void* h_target;  // [total_draft + num_seqs][hidden] bf16
+    const void* h_draft;   // [total_draft][hidden] bf16 (unused at T = 0)
+    int hidden, vocab, num_seqs, total_draft;
+    float temperature;
+    const int32_t* tokens;
+    const int32_t* cu_draft;
+    const float* u_accept;
+    const float* u_sample;
+    int32_t* n_accepted;
+    int32_t* out_tokens;
+    float* accept_prob;
+    float* logits_out;
+    void* scratch;
+    unsigned int* err_word;
+};
+size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft);
+// Grid size, padded row count (MMA N) and tiles per CTA; BP_ERR_UNSUPPORTED outside the limits.
+int verify_epilogue_config(int rows, int vocab, int sm_count, int* grid, int* np, int* tiles_per_cta);
+int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+
 }  // namespace bp

@@ -1,0 +1,780 @@
+// Fused verify epilogue: the LM-head projection of the verified positions (and of the drafter's
+// positions) with the lossless acceptance of Section 2.1 applied to it on the fly.  The logits
+// never leave the chip.
+//
+// Section 2.1 / Figure 1: the target scores every position of a drafted block in one pass and
+// keeps the longest prefix the acceptance rule admits; that rule (standard speculative sampling:
+// accept x_i with probability min(1, p_i(x_i) / q_i(x_i)), redraw from norm(max(0, p_k - q_k)) at
+// the first rejection k, a bonus draw from p_gamma when every draft is accepted; greedy at T = 0)
+// reads p = softmax(W h_t / T) and q = softmax(W h_d / T) over the whole vocabulary, W being the
+// [V, H] LM head.  Unfused, the LM-head GEMM writes [rows, V] fp32 logits to HBM and the
+// acceptance reads them back; here the GEMM's accumulators stay in tensor memory until the
+// acceptance has used them, so the only HBM stream is W itself (read once).
+//
+// One persistent cooperative launch, one CTA per SM (every CTA co-resident):
+//   * CTA c owns a contiguous slice of the vocabulary, at most 16 tiles of 128 LM-head rows.  Its
+//     W rows stream once through an 8-stage TMA ring (one 128 x 64 bf16 box per stage, 128-byte
+//     swizzle); warp 2 gathers the same 64 columns of every state row (target rows, then drafter
+//     rows, zero rows up to NP) into the stage with 16-byte cp.async copies; one thread of warp 1
+//     issues M=128 x N=NP x K=16 tcgen05 MMAs into the tile's own NP columns of tensor memory.
+//   * Warps 4-7 read each finished tile (TMEM lane = vocabulary entry, column = row) while the next
+//     one streams: every row's running max and sum of 2^(l*log2e/T - max) (T = 0: running argmax,
+//     lowest index first), and the scaled logits at the draft tokens the slice holds.
+//   * Grid barrier 1.  Every CTA merges the slices' statistics of every row in the same fixed
+//     order, so all CTAs hold bit-identical normalisers, ratios a_i and first rejections k_s; CTA 0
+//     writes n_accepted, the accepted drafts and accept_prob (T = 0: the emitted argmax too).
+//   * T > 0: every CTA sums its slice's mass of max(0, p_k - q_k) (p_gamma for a bonus draw) per
+//     sequence in exact 2^-52 fixed point; grid barrier 2; the CTA whose slice holds the crossing of
+//     u_s * total recomputes its 32-entry chunks, finds the entry and writes the emitted token.
+//   * The last CTA out clears the grid-barrier counters for the next call.
+// Every wait is bounded; an expired wait sets the workspace error word and the kernel winds down.
+#include <cuda.h>
+#include <cuda_bf16.h>
+#include <cuda_runtime.h>
+#include <limits.h>
+#include <math.h>
+
+#include "common.cuh"
+#include "ptx_sm103.cuh"
+#include "softmax_math.cuh"
+
+namespace bp {
+namespace {
+
+constexpr int kVeM = 128;                        // vocabulary entries per tile: the MMA M, TMEM lanes
+constexpr int kVeAtom = 64;                      // hidden columns per 128-byte swizzle atom
+constexpr int kVeWBytes = kVeM * kVeAtom * 2;    // 16 KB of W per stage
+constexpr int kVeStages = 8;
+constexpr int kVeLag = 2;                        // state copies kept in flight before a stage is published
+constexpr int kVeThreads = 256;
+constexpr int kVeEpi = 4;                        // first epilogue warp (lane quarter = warp % 4)
+constexpr int kVeMaxTiles = 16;
+constexpr int kVeMaxGrid = 256;
+
+struct VeParams {
+    const __nv_bfloat16* h_target;  // [rows_t][hidden]
+    const __nv_bfloat16* h_draft;   // [rows - rows_t][hidden]
+    int hidden, vocab, atoms;
+    int num_seqs, total_draft, rows_t, rows;
+    int tiles_base, tiles_extra;    // CTA c: tiles_base + (c < tiles_extra) tiles
+    uint32_t tmem_cols;
+    float c2;                       // log2(e) / T
+    const int32_t* tokens;
+    const int32_t* cu_draft;
+    const float* u_accept;
+    const float* u_sample;
+    int32_t* n_accepted;
+    int32_t* out_tokens;
+    float* accept_prob;
+    float* logits_out;              // [rows][vocab] or null
+    float2* part;                   // [rows][grid] slice statistics (T = 0: value, index bits)
+    float2* xg;                     // [total_draft] scaled (target, drafter) logits at the draft token
+    ulonglong2* tot;                // [num_seqs][grid] slice masses of r and p, 2^-52 units
+    unsigned int* sync;             // [0] grid-barrier arrivals, [1] exits; zero between calls
+    unsigned int* err;
+};
+
+__device__ __forceinline__ void red_release_gpu(unsigned int* a, unsigned int v) {
+    asm volatile("red.release.gpu.global.add.u32 [%0], %1;" ::"l"(a), "r"(v) : "memory");
+}
+__device__ __forceinline__ unsigned int ld_acquire_gpu(const unsigned int* a) {
+    unsigned int v;
+    asm volatile("ld.acquire.gpu.global.u32 %0, [%1];" : "=r"(v) : "l"(a) : "memory");
+    return v;
+}
+__device__ __forceinline__ unsigned int atom_add_acq_rel_gpu(unsigned int* a, unsigned int v) {
+    unsigned int old;
+    asm volatile("atom.add.acq_rel.gpu.u32 %0, [%1], %2;" : "=r"(old) : "l"(a), "r"(v) : "memory");
+    return old;
+}
+// Named barrier among `count` threads (a multiple of 32) of the CTA.
+__device__ __forceinline__ void named_sync(int id, int count) {
+    asm volatile("bar.sync %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+__device__ __forceinline__ void named_arrive(int id, int count) {
+    asm volatile("bar.arrive %0, %1;" ::"r"(id), "r"(count) : "memory");
+}
+
+// Every CTA of the (co-resident) grid arrives, then waits until `target` arrivals are counted.
+// False in every thread if they were not within the wait budget.
+__device__ bool grid_barrier(unsigned int* count, unsigned int target, int* ok_sh) {
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        red_release_gpu(count, 1u);
+        const long long t0 = clock64();
+        int ok = 1;
+        while (ld_acquire_gpu(count) < target) {
+            if (clock64() - t0 > kWaitBudget) {
+                ok = 0;
+                break;
+            }
+            __nanosleep(64);
+        }
+        __threadfence();
+        *ok_sh = ok;
+    }
+    __syncthreads();
+    return *ok_sh != 0;
+}
+
+// Value of column `col` among the NP columns a thread loaded (a select chain: no dynamic indexing).
+template <int NP>
+__device__ __forceinline__ float pick(const uint32_t (&r)[NP], int col) {
+    float x = 0.f;
+#pragma unroll
+    for (int e = 0; e < NP; ++e)
+        if (e == col) x = __uint_as_float(r[e]);
+    return x;
+}
+
+// Lane `lane` ends with the warp-wide merge of column `lane` of the (max, sum) pairs: a butterfly
+// that halves the columns it carries at every step (31 exchanges).
+__device__ __forceinline__ float2 lse_reduce_scatter32(float (&m)[32], float (&s)[32], int lane) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int j = 0; j < o; ++j) {
+            const float sm = up ? m[j] : m[j + o], ss = up ? s[j] : s[j + o];
+            float km = up ? m[j + o] : m[j], ks = up ? s[j + o] : s[j];
+            lse_merge(km, ks, __shfl_xor_sync(0xffffffffu, sm, o), __shfl_xor_sync(0xffffffffu, ss, o));
+            m[j] = km;
+            s[j] = ks;
+        }
+    }
+    return make_float2(m[0], s[0]);
+}
+// The same for (value, index) argmax pairs.
+__device__ __forceinline__ float2 amax_reduce_scatter32(float (&v)[32], int (&ix)[32], int lane) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int j = 0; j < o; ++j) {
+            const float sv = up ? v[j] : v[j + o];
+            const int si = up ? ix[j] : ix[j + o];
+            float kv = up ? v[j + o] : v[j];
+            int ki = up ? ix[j + o] : ix[j];
+            amax_merge(kv, ki, __shfl_xor_sync(0xffffffffu, sv, o), __shfl_xor_sync(0xffffffffu, si, o));
+            v[j] = kv;
+            ix[j] = ki;
+        }
+    }
+    return make_float2(v[0], __int_as_float(ix[0]));
+}
+
+__device__ __forceinline__ float warp_sum_f(float x) {  // xor butterfly: bit-identical in every lane
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
+    return x;
+}
+
+// Weights of this lane's entry in tile t of the slice for one sequence's draw: x.x = r = max(0, p - q)
+// (0 without a draft row), x.y = p.  The crossing search recomputes them with this same code.
+struct DrawRow {
+    int ct, cd;        // TMEM columns of the target row and the drafter row (cd < 0: none)
+    float Mt, izt, Md, izd;
+};
+template <int NP>
+__device__ __forceinline__ float2 entry_weights(uint32_t tmem_q, int t, const DrawRow& d, bool in_vocab, float c2) {
+    const uint32_t col = (uint32_t)(t * NP);
+    const float lt = __uint_as_float(tmem_ld1(tmem_q + col + (uint32_t)d.ct));
+    const float ld = d.cd >= 0 ? __uint_as_float(tmem_ld1(tmem_q + col + (uint32_t)d.cd)) : 0.f;
+    tmem_ld_wait();
+    if (!in_vocab) return make_float2(0.f, 0.f);
+    const float pv = __fmul_rn(ex2(__fsub_rn(__fmul_rn(lt, c2), d.Mt)), d.izt);
+    float rv = 0.f;
+    if (d.cd >= 0) rv = fmaxf(0.f, __fsub_rn(pv, __fmul_rn(ex2(__fsub_rn(__fmul_rn(ld, c2), d.Md)), d.izd)));
+    return make_float2(rv, pv);
+}
+
+template <bool GREEDY, int NP>
+__global__ void __launch_bounds__(kVeThreads, 1)
+    verify_epilogue_kernel(const __grid_constant__ CUtensorMap wmap, const VeParams p) {
+    extern __shared__ uint8_t smem_raw[];
+    uint8_t* sW = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
+    uint8_t* sH = sW + kVeStages * kVeWBytes;  // state rows of each stage: NP rows of 128 bytes
+    __shared__ uint64_t wfull[kVeStages], hfull[kVeStages], empty[kVeStages], acc_full[kVeMaxTiles], mma_done;
+    __shared__ uint32_t tmem_sh;
+    __shared__ int ok_sh, own_n, find_sh, sel_sh;
+    __shared__ float2 wst[4][64];      // per epilogue warp: statistics of each row over its lanes
+    __shared__ float2 rst[64];         // statistics of each row over the whole vocabulary
+    __shared__ int own_v[64], own_ct[64], own_cd[64], own_i[64];  // draft tokens held by the slice
+    __shared__ int cu_sh[65], k_sh[64];
+    __shared__ ulonglong2 wtot[4][64];
+    __shared__ unsigned long long chunk_sh[kVeMaxTiles * 4];
+    __shared__ unsigned long long off_sh, base_sh;
+    __shared__ int use_r_sh;
+
+    const int tid = threadIdx.x, warp = tid >> 5, lane = tid & 31;
+    const int c = (int)blockIdx.x, grid = (int)gridDim.x;
+    const int ntile = p.tiles_base + (c < p.tiles_extra ? 1 : 0);
+    const int tile0 = c * p.tiles_base + min(c, p.tiles_extra);
+    const int v0 = tile0 * kVeM;                        // first vocabulary entry of the slice
+    const int v1 = min(p.vocab, v0 + ntile * kVeM);
+    const int J = ntile * p.atoms;                      // ring stages of this CTA
+    const int S = p.num_seqs;
+
+    if (tid == 0) {
+        prefetch_tensormap(&wmap);
+        for (int st = 0; st < kVeStages; ++st) {
+            mbar_init(&wfull[st], 1);
+            mbar_init(&hfull[st], 1);
+            mbar_init(&empty[st], 1);
+        }
+        for (int t = 0; t < kVeMaxTiles; ++t) mbar_init(&acc_full[t], 1);
+        mbar_init(&mma_done, 1);
+        fence_mbar_init();
+        own_n = 0;
+    }
+    if (warp == 1) {
+        tmem_alloc(&tmem_sh, p.tmem_cols);
+        tmem_relinquish();
+    }
+    for (int i = tid; i <= S; i += kVeThreads) cu_sh[i] = p.cu_draft[i];
+    tc_fence_before();
+    __syncthreads();
+    tc_fence_after();
+    const uint32_t tmem = tmem_sh;
+
+    if (warp == 0) {
+        // ---- W producer: the slice's LM-head rows, tile by tile, 64 hidden columns per stage
+        if (lane == 0) {
+            int issued = 0;
+            for (int j = 0; j < J; ++j) {
+                const int st = j % kVeStages;
+                if (j >= kVeStages && !mbar_wait(&empty[st], ((j / kVeStages) - 1) & 1, kWaitBudget)) {
+                    raise_error(p.err, kErrTimeout);
+                    break;
+                }
+                const int t = j / p.atoms, a = j - t * p.atoms;
+                mbar_arrive_expect_tx(&wfull[st], kVeWBytes);
+                tma_load_2d(sW + st * kVeWBytes, &wmap, &wfull[st], a * kVeAtom, (tile0 + t) * kVeM);
+                issued = j + 1;
+            }
+            if (issued < J)  // wound down early: let the copies still in flight land before exiting
+                for (int j = max(0, issued - kVeStages); j < issued; ++j)
+                    mbar_wait(&wfull[j % kVeStages], (j / kVeStages) & 1, kWaitBudget);
+        }
+    } else if (warp == 2) {
+        // ---- state producer: row n's 16-byte chunk ch of atom a goes to chunk ch ^ (n & 7) of row n
+        int j = 0;
+        for (; j < J; ++j) {
+            const int st = j % kVeStages;
+            const bool ok = j < kVeStages || mbar_wait(&empty[st], ((j / kVeStages) - 1) & 1, kWaitBudget);
+            if (!__all_sync(0xffffffffu, ok)) {
+                if (lane == 0) raise_error(p.err, kErrTimeout);
+                break;
+            }
+            const int a = j % p.atoms;
+            uint8_t* dst = sH + st * (NP * 128);
+#pragma unroll
+            for (int it = 0; it < NP * 8 / 32; ++it) {
+                const int idx = it * 32 + lane;
+                const int n = idx >> 3, ch = idx & 7;
+                const bool valid = n < p.rows;
+                const __nv_bfloat16* row = n < p.rows_t ? p.h_target + (size_t)n * p.hidden
+                                                        : p.h_draft + (size_t)(valid ? n - p.rows_t : 0) * p.hidden;
+                cp_async16(dst + n * 128 + ((ch ^ (n & 7)) << 4), valid ? row + a * kVeAtom + ch * 8 : p.h_target,
+                           valid);
+            }
+            cp_async_commit();
+            if (j >= kVeLag) {
+                cp_async_wait_group<kVeLag>();
+                fence_proxy_async_smem();  // the MMAs read the states through the async proxy
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&hfull[(j - kVeLag) % kVeStages]);
+            }
+        }
+        cp_async_wait_group<0>();
+        fence_proxy_async_smem();
+        __syncwarp();
+        if (lane == 0)
+            for (int jj = max(0, j - kVeLag); jj < j; ++jj) mbar_arrive(&hfull[jj % kVeStages]);
+    } else if (warp == 1) {
+        // ---- MMA issuer: tile t accumulates into TMEM columns [t * NP, t * NP + NP)
+        if (lane == 0) {
+            const uint32_t idesc = idesc_bf16_f32(kVeM, NP, false, false);
+            for (int j = 0; j < J; ++j) {
+                const int st = j % kVeStages;
+                const uint32_t par = (j / kVeStages) & 1;
+                if (!mbar_wait(&wfull[st], par, kWaitBudget) || !mbar_wait(&hfull[st], par, kWaitBudget)) {
+                    raise_error(p.err, kErrTimeout);
+                    break;
+                }
+                tc_fence_after();
+                const int t = j / p.atoms, a = j - t * p.atoms;
+                const uint32_t wa = smem_addr(sW + st * kVeWBytes), ha = smem_addr(sH + st * (NP * 128));
+#pragma unroll
+                for (int kk = 0; kk < kVeAtom / 16; ++kk)
+                    umma_ss(tmem + (uint32_t)(t * NP), smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                            smem_desc(ha + kk * 32, 16, 1024, kSwizzle128B), idesc, (a | kk) ? 1u : 0u);
+                umma_commit(&empty[st]);  // the stage is free once these MMAs have read it
+                if (a == p.atoms - 1) umma_commit(&acc_full[t]);
+            }
+            umma_commit(&mma_done);  // every MMA issued is complete before tensor memory is released
+            mbar_wait(&mma_done, 0, kWaitBudget);
+        }
+    } else if (warp == 3) {
+        // ---- the draft tokens held by this slice (their logits are captured by the epilogue)
+        if (!GREEDY) {
+            for (int i = lane; i < p.total_draft; i += 32) {
+                const int x = p.tokens[i];
+                if (x >= v0 && x < v1) {
+                    int lo = 0, hi = S;  // sequence of draft i: cu[lo] <= i < cu[lo + 1]
+                    while (hi - lo > 1) {
+                        const int mid = (lo + hi) >> 1;
+                        if (cu_sh[mid] <= i) lo = mid; else hi = mid;
+                    }
+                    const int o = atomicAdd(&own_n, 1);
+                    own_v[o] = x - v0;
+                    own_i[o] = i;
+                    own_ct[o] = i + lo;           // target row of draft i
+                    own_cd[o] = p.rows_t + i;     // its drafter row
+                }
+            }
+            __threadfence_block();
+            named_arrive(2, 160);
+        }
+        if (c == 0)
+            for (int i = lane; i < p.total_draft; i += 32) {
+                const int x = p.tokens[i];
+                if (x < 0 || x >= p.vocab) raise_error(p.err, kErrDeviceArg);
+            }
+    } else {
+        // ---- epilogue: the running statistics of every row over this lane's entries, tile by tile
+        const int q = warp & 3;
+        const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
+        float m[NP], s[NP];
+        int ix[NP];
+#pragma unroll
+        for (int e = 0; e < NP; ++e) {
+            m[e] = -INFINITY;
+            s[e] = 0.f;
+            ix[e] = INT_MAX;
+        }
+        int nown = 0;
+        if (!GREEDY) {
+            named_sync(2, 160);
+            nown = own_n;
+        }
+        for (int t = 0; t < ntile; ++t) {
+            if (!mbar_wait(&acc_full[t], 0, kWaitBudget)) {
+                raise_error(p.err, kErrTimeout);
+                break;
+            }
+            tc_fence_after();
+            const int vl = t * kVeM + q * 32 + lane;  // entry within the slice
+            const int v = v0 + vl;
+#pragma unroll
+            for (int h0 = 0; h0 < NP; h0 += 32) {  // 32 columns at a time
+                if (h0 >= p.rows) break;
+                uint32_t r[32];
+                tmem_ld32(tq + (uint32_t)(t * NP + h0), r);
+                tmem_ld_wait();
+                if (v < v1) {
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) {
+                        if (h0 + e < p.rows) {
+                            const float l = __uint_as_float(r[e]);
+                            if (GREEDY) {
+                                if (l > m[h0 + e]) {  // entries arrive in increasing index: ties keep the first
+                                    m[h0 + e] = l;
+                                    ix[h0 + e] = v;
+                                }
+                            } else {
+                                const float x = __fmul_rn(l, p.c2);
+                                const float d = __fsub_rn(x, m[h0 + e]);
+                                const float w = ex2(-fabsf(d));
+                                s[h0 + e] = d > 0.f ? __fmaf_rn(s[h0 + e], w, 1.f) : __fadd_rn(s[h0 + e], w);
+                                m[h0 + e] = fmaxf(m[h0 + e], x);
+                            }
+                            if (p.logits_out) p.logits_out[(size_t)(h0 + e) * p.vocab + v] = l;
+                        }
+                    }
+                    for (int o = 0; o < nown; ++o)
+                        if (own_v[o] == vl) {  // scaled logits of the draft token (each owned by one thread)
+                            const int ct = own_ct[o] - h0, cd = own_cd[o] - h0;
+                            if (ct >= 0 && ct < 32) p.xg[own_i[o]].x = __fmul_rn(pick<32>(r, ct), p.c2);
+                            if (cd >= 0 && cd < 32) p.xg[own_i[o]].y = __fmul_rn(pick<32>(r, cd), p.c2);
+                        }
+                }
+            }
+        }
+        // the statistics of every row over the warp's 32 lanes, then over the four warps
+#pragma unroll
+        for (int h0 = 0; h0 < NP; h0 += 32) {
+            float2 res;
+            if (GREEDY) {
+                float vv[32];
+                int ii[32];
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    vv[e] = m[h0 + e];
+                    ii[e] = ix[h0 + e];
+                }
+                res = amax_reduce_scatter32(vv, ii, lane);
+            } else {
+                float mm[32], ss[32];
+#pragma unroll
+                for (int e = 0; e < 32; ++e) {
+                    mm[e] = m[h0 + e];
+                    ss[e] = s[h0 + e];
+                }
+                res = lse_reduce_scatter32(mm, ss, lane);
+            }
+            wst[q][h0 + lane] = res;
+        }
+        named_sync(1, 128);
+        for (int r = tid - kVeEpi * 32; r < p.rows; r += 128) {
+            float2 a = wst[0][r];
+            for (int w = 1; w < 4; ++w) {
+                if (GREEDY) {
+                    int ai = __float_as_int(a.y);
+                    amax_merge(a.x, ai, wst[w][r].x, __float_as_int(wst[w][r].y));
+                    a.y = __int_as_float(ai);
+                } else {
+                    lse_merge(a.x, a.y, wst[w][r].x, wst[w][r].y);
+                }
+            }
+            p.part[(size_t)r * grid + c] = a;
+        }
+    }
+
+    // ================= grid barrier 1: every slice's statistics and draft-token logits are out
+    if (!grid_barrier(p.sync, (unsigned)grid, &ok_sh)) raise_error(p.err, kErrTimeout);
+
+    // ---- row statistics over the whole vocabulary, merged in one fixed order in every CTA
+    for (int r = warp; r < p.rows; r += kVeThreads / 32) {
+        float a0 = -INFINITY, a1 = 0.f;
+        int ai = INT_MAX;
+        for (int cc = lane; cc < grid; cc += 32) {
+            const float2 x = __ldcg(&p.part[(size_t)r * grid + cc]);
+            if (GREEDY) amax_merge(a0, ai, x.x, __float_as_int(x.y));
+            else lse_merge(a0, a1, x.x, x.y);
+        }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) {
+            const float b0 = __shfl_xor_sync(0xffffffffu, a0, o);
+            if (GREEDY) {
+                amax_merge(a0, ai, b0, __shfl_xor_sync(0xffffffffu, ai, o));
+            } else {
+                lse_merge(a0, a1, b0, __shfl_xor_sync(0xffffffffu, a1, o));
+            }
+        }
+        if (lane == 0) rst[r] = GREEDY ? make_float2(a0, __int_as_float(ai)) : make_float2(a0, a1);
+    }
+    __syncthreads();
+    // ---- ratios and the first rejection of every sequence (identical in every CTA)
+    if (warp == 0) {
+        for (int sq = lane; sq < S; sq += 32) {
+            const int d0 = cu_sh[sq], g = cu_sh[sq + 1] - d0;
+            int k = g;
+            for (int j = 0; j < g; ++j) {
+                const int i = d0 + j, ct = i + sq;
+                const int x = p.tokens[i];
+                float a;
+                if (GREEDY) {
+                    a = (x == __float_as_int(rst[ct].y)) ? 1.f : 0.f;
+                } else if (x < 0 || x >= p.vocab) {
+                    a = 0.f;
+                } else {
+                    const float2 xx = __ldcg(&p.xg[i]);
+                    const float2 st = rst[ct], sd = rst[p.rows_t + i];
+                    a = fminf(1.f, ex2(__fsub_rn(__fsub_rn(xx.x, st.x), __fsub_rn(xx.y, sd.x))) * __fdiv_rn(sd.y, st.y));
+                }
+                if (c == 0 && p.accept_prob) p.accept_prob[i] = a;
+                const bool rej = GREEDY ? (a == 0.f) : !(__ldg(p.u_accept + i) < a);
+                if (rej && k == g) k = j;
+            }
+            k_sh[sq] = k;
+        }
+    }
+    __syncthreads();
+    if (c == 0) {  // n_accepted, the accepted drafts, -1 past the emitted slot (T = 0: the emitted argmax)
+        for (int sq = warp; sq < S; sq += kVeThreads / 32) {
+            const int d0 = cu_sh[sq], g = cu_sh[sq + 1] - d0, k = k_sh[sq], t0 = d0 + sq;
+            for (int j = lane; j <= g; j += 32) {
+                if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
+                else if (j > k) p.out_tokens[t0 + j] = -1;
+                else if (GREEDY) p.out_tokens[t0 + j] = __float_as_int(rst[t0 + k].y);
+            }
+            if (lane == 0) p.n_accepted[sq] = k;
+        }
+    }
+
+    if (!GREEDY) {
+        // ---- this slice's mass of each sequence's draw distribution, exact fixed point
+        const int q = warp & 3;
+        const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
+        if (warp >= kVeEpi) {
+            for (int sq = 0; sq < S; ++sq) {
+                const int d0 = cu_sh[sq], g = cu_sh[sq + 1] - d0, k = k_sh[sq];
+                DrawRow d;
+                d.ct = d0 + sq + k;
+                d.cd = k < g ? p.rows_t + d0 + k : -1;
+                d.Mt = rst[d.ct].x;
+                d.izt = __fdiv_rn(1.f, rst[d.ct].y);
+                d.Md = d.cd >= 0 ? rst[d.cd].x : 0.f;
+                d.izd = d.cd >= 0 ? __fdiv_rn(1.f, rst[d.cd].y) : 0.f;
+                unsigned long long R = 0, P = 0;
+                for (int t = 0; t < ntile; ++t) {
+                    const float2 w = entry_weights<NP>(tq, t, d, v0 + t * kVeM + q * 32 + lane < v1, p.c2);
+                    R += to_fix(warp_sum_f(w.x));
+                    P += to_fix(warp_sum_f(w.y));
+                }
+                if (lane == 0) wtot[q][sq] = make_ulonglong2(R, P);
+            }
+            named_sync(1, 128);
+            for (int sq = tid - kVeEpi * 32; sq < S; sq += 128) {
+                ulonglong2 a = wtot[0][sq];
+                for (int w = 1; w < 4; ++w) {
+                    a.x += wtot[w][sq].x;
+                    a.y += wtot[w][sq].y;
+                }
+                p.tot[(size_t)sq * grid + c] = a;
+            }
+        }
+
+        // ================= grid barrier 2: every slice's masses are out
+        if (!grid_barrier(p.sync, 2u * (unsigned)grid, &ok_sh)) raise_error(p.err, kErrTimeout);
+
+        for (int sq = 0; sq < S; ++sq) {
+            const int d0 = cu_sh[sq], g = cu_sh[sq + 1] - d0, k = k_sh[sq];
+            if (warp == 0) {
+                unsigned long long R = 0, P = 0, Rb = 0, Pb = 0;
+                for (int cc = lane; cc < grid; cc += 32) {
+                    const ulonglong2 x = __ldcg(&p.tot[(size_t)sq * grid + cc]);
+                    R += x.x;
+                    P += x.y;
+                    if (cc < c) {
+                        Rb += x.x;
+                        Pb += x.y;
+                    }
+                }
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) {
+                    R += __shfl_xor_sync(0xffffffffu, R, o);
+                    P += __shfl_xor_sync(0xffffffffu, P, o);
+                    Rb += __shfl_xor_sync(0xffffffffu, Rb, o);
+                    Pb += __shfl_xor_sync(0xffffffffu, Pb, o);
+                }
+                if (lane == 0) {
+                    const ulonglong2 own = __ldcg(&p.tot[(size_t)sq * grid + c]);
+                    const bool use_r = k < g && R > 0;  // a vanishing residual (p == q) draws from p
+                    const unsigned long long total = use_r ? R : P, below = use_r ? Rb : Pb;
+                    const unsigned long long mine = use_r ? own.x : own.y;
+                    float u = __ldg(p.u_sample + sq);
+                    if (!(u >= 0.f)) u = 0.f;
+                    u = fminf(u, 0.99999994f);  // u in [0, 1): the crossing always exists
+                    const unsigned long long thr = __umul64hi(__float2ull_rn(u * 18446744073709551616.f), total);
+                    int find = 0;
+                    if (total == 0) {  // no positive mass at all: report, emit 0
+                        if (c == 0) {
+                            raise_error(p.err, kErrDeviceArg);
+                            p.out_tokens[d0 + sq + k] = 0;
+                        }
+                    } else if (below <= thr && thr < below + mine) {
+                        find = 1;
+                        off_sh = thr - below;
+                    }
+                    find_sh = find;
+                    use_r_sh = use_r;
+                }
+            }
+            __syncthreads();
+            if (find_sh && warp >= kVeEpi) {
+                // ---- the crossing is in this slice: chunk masses in entry order, then the entry
+                DrawRow d;
+                d.ct = d0 + sq + k;
+                d.cd = k < g ? p.rows_t + d0 + k : -1;
+                d.Mt = rst[d.ct].x;
+                d.izt = __fdiv_rn(1.f, rst[d.ct].y);
+                d.Md = d.cd >= 0 ? rst[d.cd].x : 0.f;
+                d.izd = d.cd >= 0 ? __fdiv_rn(1.f, rst[d.cd].y) : 0.f;
+                const bool use_r = use_r_sh != 0;
+                for (int t = 0; t < ntile; ++t) {
+                    const float2 w = entry_weights<NP>(tq, t, d, v0 + t * kVeM + q * 32 + lane < v1, p.c2);
+                    const unsigned long long f = to_fix(warp_sum_f(use_r ? w.x : w.y));
+                    if (lane == 0) chunk_sh[t * 4 + q] = f;
+                }
+                named_sync(1, 128);
+                if (tid == kVeEpi * 32) {
+                    const unsigned long long off = off_sh;
+                    unsigned long long cum = 0;
+                    int sel = -1;
+                    for (int idx = 0; idx < ntile * 4; ++idx) {
+                        const unsigned long long x = chunk_sh[idx];
+                        if (sel < 0 && x > 0 && cum <= off && off < cum + x) {
+                            sel = idx;
+                            base_sh = cum;
+                        }
+                        cum += x;
+                    }
+                    sel_sh = sel;
+                }
+                named_sync(1, 128);
+                const int sel = sel_sh;
+                if (sel < 0) {  // unreachable with exact sums: report, emit the slice's first entry
+                    if (tid == kVeEpi * 32) {
+                        raise_error(p.err, kErrDeviceArg);
+                        p.out_tokens[d0 + sq + k] = v0;
+                    }
+                } else if ((sel & 3) == q) {
+                    const int t = sel >> 2;
+                    const int v = v0 + t * kVeM + q * 32 + lane;
+                    const float2 w2 = entry_weights<NP>(tq, t, d, v < v1, p.c2);
+                    const float w = use_r ? w2.x : w2.y;
+                    // offset of the threshold inside the chunk, back in probability units
+                    const float off = __ull2float_rn(off_sh - base_sh) * 2.220446049250313e-16f;
+                    const float run = warp_incl_scan_f(w, lane);
+                    const unsigned hit = __ballot_sync(0xffffffffu, w > 0.f && run > off);
+                    const unsigned pos = __ballot_sync(0xffffffffu, w > 0.f);
+                    // fp32 rounding inside the chunk can leave the crossing just past its end: then
+                    // the chunk's last entry with positive weight
+                    const int ln = hit ? __ffs(hit) - 1 : (pos ? 31 - __clz(pos) : 0);
+                    if (lane == 0) p.out_tokens[d0 + sq + k] = v0 + t * kVeM + q * 32 + ln;
+                }
+            }
+            __syncthreads();
+        }
+    }
+
+    // ---- release tensor memory; the last CTA out clears the grid-barrier counters
+    tc_fence_before();
+    __syncthreads();
+    if (warp == 1) {
+        tc_fence_after();
+        tmem_dealloc(tmem, p.tmem_cols);
+    }
+    if (tid == 0) {
+        const unsigned int old = atom_add_acq_rel_gpu(p.sync + 1, 1u);
+        if (old == (unsigned)grid - 1u) {
+            atomicExch(p.sync, 0u);
+            atomicExch(p.sync + 1, 0u);
+        }
+    }
+}
+
+template <bool GREEDY, int NP>
+size_t ve_smem_bytes() {
+    return 1024 + (size_t)kVeStages * (kVeWBytes + NP * 128);
+}
+
+struct VeLayout {
+    size_t sync_off, part_off, xg_off, tot_off, total;
+};
+VeLayout ve_layout(int num_seqs, int total_draft) {
+    VeLayout l;
+    const int rows = 2 * total_draft + num_seqs;
+    l.sync_off = 0;
+    l.part_off = 256;
+    l.xg_off = l.part_off + align_up((size_t)(rows > 0 ? rows : 1) * kVeMaxGrid * sizeof(float2), 256);
+    l.tot_off = l.xg_off + align_up((size_t)(total_draft > 0 ? total_draft : 1) * sizeof(float2), 256);
+    l.total = l.tot_off + align_up((size_t)(num_seqs > 0 ? num_seqs : 1) * kVeMaxGrid * sizeof(ulonglong2), 256);
+    return l;
+}
+
+template <bool GREEDY, int NP>
+int ve_launch(const CUtensorMap& wmap, const VeParams& p, int grid, const DeviceInfo& dev, cudaStream_t stream) {
+    static int configured[64] = {};
+    const size_t smem = ve_smem_bytes<GREEDY, NP>();
+    if (dev.device >= 0 && dev.device < 64 && !configured[dev.device]) {
+        if (cudaFuncSetAttribute(verify_epilogue_kernel<GREEDY, NP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+                                 (int)smem) != cudaSuccess)
+            return BP_ERR_CUDA;
+        int per_sm = 0;
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, verify_epilogue_kernel<GREEDY, NP>, kVeThreads,
+                                                          smem) != cudaSuccess ||
+            per_sm < 1)
+            return BP_ERR_UNSUPPORTED;
+        configured[dev.device] = 1;
+    }
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3((unsigned)grid);
+    cfg.blockDim = dim3(kVeThreads);
+    cfg.dynamicSmemBytes = smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;  // every CTA co-resident: the grid barriers need it
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, verify_epilogue_kernel<GREEDY, NP>, wmap, p) == cudaSuccess ? BP_OK
+                                                                                               : BP_ERR_CUDA;
+}
+
+}  // namespace
+
+size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft) {
+    return ve_layout(num_seqs, total_draft).total;
+}
+
+int verify_epilogue_config(int rows, int vocab, int sm_count, int* grid, int* np, int* tiles_per_cta) {
+    const int tiles_total = (vocab + kVeM - 1) / kVeM;
+    const int g = min(min(sm_count, kVeMaxGrid), tiles_total);
+    if (g < 1 || rows < 1 || rows > 64) return BP_ERR_UNSUPPORTED;
+    const int NP = rows <= 32 ? 32 : 64;
+    const int per = (tiles_total + g - 1) / g;
+    if (per > kVeMaxTiles || per * NP > 512) return BP_ERR_UNSUPPORTED;
+    *grid = g;
+    *np = NP;
+    *tiles_per_cta = per;
+    return BP_OK;
+}
+
+int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
+    const bool greedy = a.temperature == 0.f;
+    const int rows_t = a.total_draft + a.num_seqs;
+    const int rows = rows_t + (greedy ? 0 : a.total_draft);
+    int grid = 0, NP = 0, per = 0;
+    int rc = verify_epilogue_config(rows, a.vocab, dev.sm_count, &grid, &NP, &per);
+    if (rc != BP_OK) return rc;
+    const int tiles_total = (a.vocab + kVeM - 1) / kVeM;
+    uint32_t cols = 32;
+    while (cols < (uint32_t)(per * NP)) cols <<= 1;
+
+    CUtensorMap wmap;
+    const cuuint64_t dims[2] = {(cuuint64_t)a.hidden, (cuuint64_t)a.vocab};
+    const cuuint64_t strides[1] = {(cuuint64_t)a.hidden * 2};
+    const cuuint32_t box[2] = {(cuuint32_t)kVeAtom, (cuuint32_t)kVeM};
+    if (encode_tensor_map(&wmap, CU_TENSOR_MAP_DATA_TYPE_BFLOAT16, 2, const_cast<void*>(a.lm_head), dims, strides, box,
+                          CU_TENSOR_MAP_SWIZZLE_128B) != BP_OK)
+        return BP_ERR_CUDA;
+
+    const VeLayout l = ve_layout(a.num_seqs, a.total_draft);
+    uint8_t* ws = static_cast<uint8_t*>(a.scratch);
+    VeParams p;
+    p.h_target = static_cast<const __nv_bfloat16*>(a.h_target);
+    p.h_draft = static_cast<const __nv_bfloat16*>(greedy ? a.h_target : a.h_draft);
+    p.hidden = a.hidden;
+    p.vocab = a.vocab;
+    p.atoms = a.hidden / kVeAtom;
+    p.num_seqs = a.num_seqs;
+    p.total_draft = a.total_draft;
+    p.rows_t = rows_t;
+    p.rows = rows;
+    p.tiles_base = tiles_total / grid;
+    p.tiles_extra = tiles_total % grid;
+    p.tmem_cols = cols;
+    p.c2 = greedy ? 0.f : 1.4426950408889634f / a.temperature;
+    p.tokens = a.tokens;
+    p.cu_draft = a.cu_draft;
+    p.u_accept = a.u_accept;
+    p.u_sample = a.u_sample;
+    p.n_accepted = a.n_accepted;
+    p.out_tokens = a.out_tokens;
+    p.accept_prob = a.accept_prob;
+    p.logits_out = a.logits_out;
+    p.part = reinterpret_cast<float2*>(ws + l.part_off);
+    p.xg = reinterpret_cast<float2*>(ws + l.xg_off);
+    p.tot = reinterpret_cast<ulonglong2*>(ws + l.tot_off);
+    p.sync = reinterpret_cast<unsigned int*>(ws + l.sync_off);
+    p.err = a.err_word;
+    if (greedy) return NP == 32 ? ve_launch<true, 32>(wmap, p, grid, dev, stream)
+                                : ve_launch<true, 64>(wmap, p, grid, dev, stream);
+    return NP == 32 ? ve_launch<false, 32>(wmap, p, grid, dev, stream) : ve_launch<false, 64>(wmap, p, grid, dev, stream);
+}
+
+}  // namespace bp

@@ -43,7 +43,7 @@ def test_exports_match_header(lib):
 
 
 def test_version_and_error_strings(lib):
-    assert lib.bp_abi_version() == 2
+    assert lib.bp_abi_version() == 3
     for code in range(7):
         assert lib.bp_error_string(code).startswith(b"BP_")
     assert lib.bp_error_string(99) == b"unknown bp_status"
@@ -112,6 +112,27 @@ def test_paged_host_validation_needs_no_gpu(lib):
     assert append(page=100) == 1
     assert append(head_dim=4) == 2                            # 8-byte rows: not a multiple of 16 bytes
     assert lib.bp_kv_append(fake, fake, fake, fake, fake, fake, None, 33, 64, 40, 1, 16, 8, 128, 1, None) == 1
+
+
+def test_verify_epilogue_host_validation_needs_no_gpu(lib):
+    vp, f32 = ctypes.c_void_p, ctypes.c_float
+    fake, ws = vp(0x10000), vp(0x20000)
+
+    def call(hidden=2560, vocab=151936, seqs=1, drafts=15, temp=1.0, h_draft=fake, ws_bytes=1 << 20, w=fake):
+        return lib.bp_verify_epilogue(w, fake, h_draft, hidden, vocab, fake, fake, seqs, drafts, f32(temp), fake, fake,
+                                      fake, fake, None, None, ws, ws_bytes, None)
+    need = lib.bp_verify_epilogue_workspace_size(1, 15)
+    assert 256 < need < (1 << 20) and need % 256 == 0
+    assert call(w=None) == 1                      # no LM head
+    assert call(temp=-1.0) == 1                   # negative temperature
+    assert call(h_draft=None) == 1                # T > 0 needs the drafter's states
+    assert call(hidden=100) == 2                  # hidden not a multiple of 64
+    assert call(drafts=40) == 2                   # 40 + 1 + 40 rows > 64
+    assert call(w=vp(0x10008)) == 2               # LM head not 16-byte aligned
+    assert call(ws_bytes=need - 256) == 4         # workspace too small
+    assert call(seqs=0) == 0                      # nothing to do
+    if not __import__("torch").cuda.is_available():
+        assert call(temp=0.0, h_draft=None) == 3  # valid; no device to run on
 
 
 def test_no_cpu_fallback_without_gpu(lib):
