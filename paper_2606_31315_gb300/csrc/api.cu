@@ -302,7 +302,7 @@ int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_
     DeviceInfo dev;
     if ((rc = device_info(&dev)) != BP_OK) return rc;
     int grid, np, per;
-    if ((rc = verify_epilogue_config((int)rows, vocab, dev.sm_count, &grid, &np, &per)) != BP_OK) return rc;
+    if ((rc = verify_epilogue_config((int)rows, vocab, hidden, dev.sm_count, &grid, &np, &per)) != BP_OK) return rc;
     VerifyEpilogueArgs a;
     a.lm_head = lm_head; a.h_target = h_target; a.h_draft = h_draft;
     a.hidden = hidden; a.vocab = vocab; a.num_seqs = num_seqs; a.total_draft = total_draft;

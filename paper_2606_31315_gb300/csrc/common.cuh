@@ -135,7 +135,7 @@ struct VerifyEpilogueArgs {
 };
 size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft);
 // Grid size, padded row count (MMA N) and tiles per CTA; BP_ERR_UNSUPPORTED outside the limits.
-int verify_epilogue_config(int rows, int vocab, int sm_count, int* grid, int* np, int* tiles_per_cta);
+int verify_epilogue_config(int rows, int vocab, int hidden, int sm_count, int* grid, int* np, int* tiles_per_cta);
 int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
 }  // namespace bp

@@ -43,13 +43,18 @@ namespace {
 
 constexpr int kVeM = 128;                        // vocabulary entries per tile: the MMA M, TMEM lanes
 constexpr int kVeAtom = 64;                      // hidden columns per 128-byte swizzle atom
-constexpr int kVeWBytes = kVeM * kVeAtom * 2;    // 16 KB of W per stage
-constexpr int kVeStages = 8;
+constexpr int kVeWBytes = kVeM * kVeAtom * 2;    // 16 KB of W per atom
+constexpr int kVeMaxStages = 8;
 constexpr int kVeLag = 2;                        // state copies kept in flight before a stage is published
 constexpr int kVeThreads = 256;
 constexpr int kVeEpi = 4;                        // first epilogue warp (lane quarter = warp % 4)
 constexpr int kVeMaxTiles = 16;
-constexpr int kVeMaxGrid = 256;
+constexpr int kVeMaxGrid = 160;
+
+// Ring geometry: APS atoms (64 hidden columns each) per stage -- two atoms fetch 256 contiguous
+// bytes of every W row at once, which HBM serves far better than 128 -- and as many stages as
+// fit beside the states (NP rows per atom) in shared memory.
+__host__ __device__ constexpr int ve_stages(int NP, int APS) { return APS == 1 ? 8 : (NP == 32 ? 5 : 4); }
 
 struct VeParams {
     const __nv_bfloat16* h_target;  // [rows_t][hidden]
@@ -189,13 +194,14 @@ __device__ __forceinline__ float2 entry_weights(uint32_t tmem_q, int t, const Dr
     return make_float2(rv, pv);
 }
 
-template <bool GREEDY, int NP>
+template <bool GREEDY, int NP, int APS>
 __global__ void __launch_bounds__(kVeThreads, 1)
     verify_epilogue_kernel(const __grid_constant__ CUtensorMap wmap, const VeParams p) {
+    constexpr int STG = ve_stages(NP, APS);
     extern __shared__ uint8_t smem_raw[];
     uint8_t* sW = reinterpret_cast<uint8_t*>((reinterpret_cast<uintptr_t>(smem_raw) + 1023) & ~uintptr_t(1023));
-    uint8_t* sH = sW + kVeStages * kVeWBytes;  // state rows of each stage: NP rows of 128 bytes
-    __shared__ uint64_t wfull[kVeStages], hfull[kVeStages], empty[kVeStages], acc_full[kVeMaxTiles], mma_done;
+    uint8_t* sH = sW + STG * APS * kVeWBytes;  // state rows of each stage: APS x NP rows of 128 bytes
+    __shared__ uint64_t wfull[kVeMaxStages], hfull[kVeMaxStages], empty[kVeMaxStages], acc_full[kVeMaxTiles], mma_done;
     __shared__ uint32_t tmem_sh;
     __shared__ int ok_sh, own_n, find_sh, sel_sh;
     __shared__ float2 wst[4][64];      // per epilogue warp: statistics of each row over its lanes
@@ -203,7 +209,6 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     __shared__ int own_v[64], own_ct[64], own_cd[64], own_i[64];  // draft tokens held by the slice
     __shared__ int cu_sh[65], k_sh[64];
     __shared__ ulonglong2 wtot[4][64];
-    __shared__ unsigned long long chunk_sh[kVeMaxTiles * 4];
     __shared__ unsigned long long off_sh, base_sh;
     __shared__ int use_r_sh;
 
@@ -213,12 +218,13 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     const int tile0 = c * p.tiles_base + min(c, p.tiles_extra);
     const int v0 = tile0 * kVeM;                        // first vocabulary entry of the slice
     const int v1 = min(p.vocab, v0 + ntile * kVeM);
-    const int J = ntile * p.atoms;                      // ring stages of this CTA
+    const int spt = p.atoms / APS;                   // ring stages per tile
+    const int J = ntile * spt;                          // ring stages of this CTA
     const int S = p.num_seqs;
 
     if (tid == 0) {
         prefetch_tensormap(&wmap);
-        for (int st = 0; st < kVeStages; ++st) {
+        for (int st = 0; st < STG; ++st) {
             mbar_init(&wfull[st], 1);
             mbar_init(&hfull[st], 1);
             mbar_init(&empty[st], 1);
@@ -232,7 +238,6 @@ __global__ void __launch_bounds__(kVeThreads, 1)
         tmem_alloc(&tmem_sh, p.tmem_cols);
         tmem_relinquish();
     }
-    for (int i = tid; i <= S; i += kVeThreads) cu_sh[i] = p.cu_draft[i];
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
@@ -243,36 +248,40 @@ __global__ void __launch_bounds__(kVeThreads, 1)
         if (lane == 0) {
             int issued = 0;
             for (int j = 0; j < J; ++j) {
-                const int st = j % kVeStages;
-                if (j >= kVeStages && !mbar_wait(&empty[st], ((j / kVeStages) - 1) & 1, kWaitBudget)) {
+                const int st = j % STG;
+                if (j >= STG && !mbar_wait(&empty[st], ((j / STG) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
-                const int t = j / p.atoms, a = j - t * p.atoms;
-                mbar_arrive_expect_tx(&wfull[st], kVeWBytes);
-                tma_load_2d(sW + st * kVeWBytes, &wmap, &wfull[st], a * kVeAtom, (tile0 + t) * kVeM);
+                const int t = j / spt, a0 = (j - t * spt) * APS;
+                mbar_arrive_expect_tx(&wfull[st], APS * kVeWBytes);
+#pragma unroll
+                for (int u = 0; u < APS; ++u)
+                    tma_load_2d(sW + (st * APS + u) * kVeWBytes, &wmap, &wfull[st], (a0 + u) * kVeAtom,
+                                (tile0 + t) * kVeM);
                 issued = j + 1;
             }
             if (issued < J)  // wound down early: let the copies still in flight land before exiting
-                for (int j = max(0, issued - kVeStages); j < issued; ++j)
-                    mbar_wait(&wfull[j % kVeStages], (j / kVeStages) & 1, kWaitBudget);
+                for (int j = max(0, issued - STG); j < issued; ++j)
+                    mbar_wait(&wfull[j % STG], (j / STG) & 1, kWaitBudget);
         }
     } else if (warp == 2) {
         // ---- state producer: row n's 16-byte chunk ch of atom a goes to chunk ch ^ (n & 7) of row n
         int j = 0;
         for (; j < J; ++j) {
-            const int st = j % kVeStages;
-            const bool ok = j < kVeStages || mbar_wait(&empty[st], ((j / kVeStages) - 1) & 1, kWaitBudget);
+            const int st = j % STG;
+            const bool ok = j < STG || mbar_wait(&empty[st], ((j / STG) - 1) & 1, kWaitBudget);
             if (!__all_sync(0xffffffffu, ok)) {
                 if (lane == 0) raise_error(p.err, kErrTimeout);
                 break;
             }
-            const int a = j % p.atoms;
-            uint8_t* dst = sH + st * (NP * 128);
+            const int a0 = (j % spt) * APS;
 #pragma unroll
-            for (int it = 0; it < NP * 8 / 32; ++it) {
+            for (int it = 0; it < APS * NP * 8 / 32; ++it) {
                 const int idx = it * 32 + lane;
-                const int n = idx >> 3, ch = idx & 7;
+                const int u = idx / (NP * 8), n = (idx >> 3) % NP, ch = idx & 7;
+                const int a = a0 + u;
+                uint8_t* dst = sH + (st * APS + u) * (NP * 128);
                 const bool valid = n < p.rows;
                 const __nv_bfloat16* row = n < p.rows_t ? p.h_target + (size_t)n * p.hidden
                                                         : p.h_draft + (size_t)(valid ? n - p.rows_t : 0) * p.hidden;
@@ -284,40 +293,47 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 cp_async_wait_group<kVeLag>();
                 fence_proxy_async_smem();  // the MMAs read the states through the async proxy
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&hfull[(j - kVeLag) % kVeStages]);
+                if (lane == 0) mbar_arrive(&hfull[(j - kVeLag) % STG]);
             }
         }
         cp_async_wait_group<0>();
         fence_proxy_async_smem();
         __syncwarp();
         if (lane == 0)
-            for (int jj = max(0, j - kVeLag); jj < j; ++jj) mbar_arrive(&hfull[jj % kVeStages]);
+            for (int jj = max(0, j - kVeLag); jj < j; ++jj) mbar_arrive(&hfull[jj % STG]);
     } else if (warp == 1) {
         // ---- MMA issuer: tile t accumulates into TMEM columns [t * NP, t * NP + NP)
         if (lane == 0) {
             const uint32_t idesc = idesc_bf16_f32(kVeM, NP, false, false);
             for (int j = 0; j < J; ++j) {
-                const int st = j % kVeStages;
-                const uint32_t par = (j / kVeStages) & 1;
+                const int st = j % STG;
+                const uint32_t par = (j / STG) & 1;
                 if (!mbar_wait(&wfull[st], par, kWaitBudget) || !mbar_wait(&hfull[st], par, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
                 tc_fence_after();
-                const int t = j / p.atoms, a = j - t * p.atoms;
-                const uint32_t wa = smem_addr(sW + st * kVeWBytes), ha = smem_addr(sH + st * (NP * 128));
+                const int t = j / spt, a0 = (j - t * spt) * APS;
 #pragma unroll
-                for (int kk = 0; kk < kVeAtom / 16; ++kk)
-                    umma_ss(tmem + (uint32_t)(t * NP), smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
-                            smem_desc(ha + kk * 32, 16, 1024, kSwizzle128B), idesc, (a | kk) ? 1u : 0u);
+                for (int u = 0; u < APS; ++u) {
+                    const uint32_t wa = smem_addr(sW + (st * APS + u) * kVeWBytes);
+                    const uint32_t ha = smem_addr(sH + (st * APS + u) * (NP * 128));
+#pragma unroll
+                    for (int kk = 0; kk < kVeAtom / 16; ++kk)
+                        umma_ss(tmem + (uint32_t)(t * NP), smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                                smem_desc(ha + kk * 32, 16, 1024, kSwizzle128B), idesc, ((a0 + u) | kk) ? 1u : 0u);
+                }
                 umma_commit(&empty[st]);  // the stage is free once these MMAs have read it
-                if (a == p.atoms - 1) umma_commit(&acc_full[t]);
+                if (a0 + APS == p.atoms) umma_commit(&acc_full[t]);
             }
             umma_commit(&mma_done);  // every MMA issued is complete before tensor memory is released
             mbar_wait(&mma_done, 0, kWaitBudget);
         }
     } else if (warp == 3) {
-        // ---- the draft tokens held by this slice (their logits are captured by the epilogue)
+        // ---- sequence offsets (read by every warp after grid barrier 1), then the draft tokens held
+        // by this slice (their logits are captured by the epilogue)
+        for (int i = lane; i <= S; i += 32) cu_sh[i] = p.cu_draft[i];
+        __syncwarp();
         if (!GREEDY) {
             for (int i = lane; i < p.total_draft; i += 32) {
                 const int x = p.tokens[i];
@@ -445,25 +461,41 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     // ================= grid barrier 1: every slice's statistics and draft-token logits are out
     if (!grid_barrier(p.sync, (unsigned)grid, &ok_sh)) raise_error(p.err, kErrTimeout);
 
-    // ---- row statistics over the whole vocabulary, merged in one fixed order in every CTA
-    for (int r = warp; r < p.rows; r += kVeThreads / 32) {
-        float a0 = -INFINITY, a1 = 0.f;
-        int ai = INT_MAX;
-        for (int cc = lane; cc < grid; cc += 32) {
-            const float2 x = __ldcg(&p.part[(size_t)r * grid + cc]);
-            if (GREEDY) amax_merge(a0, ai, x.x, __float_as_int(x.y));
-            else lse_merge(a0, a1, x.x, x.y);
-        }
+    // ---- row statistics over the whole vocabulary, merged in one fixed order in every CTA; a warp
+    // takes rows warp, warp + 8, ... and keeps the loads of four rows in flight at once
+    for (int r0 = warp; r0 < p.rows; r0 += 4 * (kVeThreads / 32)) {
+        float2 x[4][kVeMaxGrid / 32];
 #pragma unroll
-        for (int o = 16; o >= 1; o >>= 1) {
-            const float b0 = __shfl_xor_sync(0xffffffffu, a0, o);
-            if (GREEDY) {
-                amax_merge(a0, ai, b0, __shfl_xor_sync(0xffffffffu, ai, o));
-            } else {
-                lse_merge(a0, a1, b0, __shfl_xor_sync(0xffffffffu, a1, o));
+        for (int b = 0; b < 4; ++b) {
+            const int r = r0 + b * (kVeThreads / 32);
+#pragma unroll
+            for (int m = 0; m < kVeMaxGrid / 32; ++m) {
+                const int cc = m * 32 + lane;
+                const float2 none = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
+                x[b][m] = (r < p.rows && cc < grid) ? __ldcg(&p.part[(size_t)r * grid + cc]) : none;
             }
         }
-        if (lane == 0) rst[r] = GREEDY ? make_float2(a0, __int_as_float(ai)) : make_float2(a0, a1);
+#pragma unroll
+        for (int b = 0; b < 4; ++b) {
+            const int r = r0 + b * (kVeThreads / 32);
+            float a0 = -INFINITY, a1 = 0.f;
+            int ai = INT_MAX;
+#pragma unroll
+            for (int m = 0; m < kVeMaxGrid / 32; ++m) {
+                if (GREEDY) amax_merge(a0, ai, x[b][m].x, __float_as_int(x[b][m].y));
+                else lse_merge(a0, a1, x[b][m].x, x[b][m].y);
+            }
+#pragma unroll
+            for (int o = 16; o >= 1; o >>= 1) {
+                const float b0 = __shfl_xor_sync(0xffffffffu, a0, o);
+                if (GREEDY) {
+                    amax_merge(a0, ai, b0, __shfl_xor_sync(0xffffffffu, ai, o));
+                } else {
+                    lse_merge(a0, a1, b0, __shfl_xor_sync(0xffffffffu, a1, o));
+                }
+            }
+            if (lane == 0 && r < p.rows) rst[r] = GREEDY ? make_float2(a0, __int_as_float(ai)) : make_float2(a0, a1);
+        }
     }
     __syncthreads();
     // ---- ratios and the first rejection of every sequence (identical in every CTA)
@@ -482,7 +514,9 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 } else {
                     const float2 xx = __ldcg(&p.xg[i]);
                     const float2 st = rst[ct], sd = rst[p.rows_t + i];
-                    a = fminf(1.f, ex2(__fsub_rn(__fsub_rn(xx.x, st.x), __fsub_rn(xx.y, sd.x))) * __fdiv_rn(sd.y, st.y));
+                    // a = min(1, p(x)/q(x)) in the log domain: 2^((xt - Mt) - (xd - Md)) * Zd / Zt
+                    const float lr = __fsub_rn(__fsub_rn(xx.x, st.x), __fsub_rn(xx.y, sd.x));
+                    a = fminf(1.f, ex2(lr) * __fdiv_rn(sd.y, st.y));
                 }
                 if (c == 0 && p.accept_prob) p.accept_prob[i] = a;
                 const bool rej = GREEDY ? (a == 0.f) : !(__ldg(p.u_accept + i) < a);
@@ -505,7 +539,9 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     }
 
     if (!GREEDY) {
-        // ---- this slice's mass of each sequence's draw distribution, exact fixed point
+        // ---- this slice's mass of each sequence's draw distribution, exact fixed point; the masses of
+        // its 32-entry chunks are kept (in the ring's shared memory, idle now) for the crossing search
+        ulonglong2* chunk = reinterpret_cast<ulonglong2*>(sW);  // [sequence][tile][lane quarter]
         const int q = warp & 3;
         const uint32_t tq = tmem + ((uint32_t)(q * 32) << 16);
         if (warp >= kVeEpi) {
@@ -521,8 +557,10 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 unsigned long long R = 0, P = 0;
                 for (int t = 0; t < ntile; ++t) {
                     const float2 w = entry_weights<NP>(tq, t, d, v0 + t * kVeM + q * 32 + lane < v1, p.c2);
-                    R += to_fix(warp_sum_f(w.x));
-                    P += to_fix(warp_sum_f(w.y));
+                    const unsigned long long fr = to_fix(warp_sum_f(w.x)), fp = to_fix(warp_sum_f(w.y));
+                    if (lane == 0) chunk[(sq * ntile + t) * 4 + q] = make_ulonglong2(fr, fp);
+                    R += fr;
+                    P += fp;
                 }
                 if (lane == 0) wtot[q][sq] = make_ulonglong2(R, P);
             }
@@ -594,18 +632,13 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 d.Md = d.cd >= 0 ? rst[d.cd].x : 0.f;
                 d.izd = d.cd >= 0 ? __fdiv_rn(1.f, rst[d.cd].y) : 0.f;
                 const bool use_r = use_r_sh != 0;
-                for (int t = 0; t < ntile; ++t) {
-                    const float2 w = entry_weights<NP>(tq, t, d, v0 + t * kVeM + q * 32 + lane < v1, p.c2);
-                    const unsigned long long f = to_fix(warp_sum_f(use_r ? w.x : w.y));
-                    if (lane == 0) chunk_sh[t * 4 + q] = f;
-                }
-                named_sync(1, 128);
                 if (tid == kVeEpi * 32) {
                     const unsigned long long off = off_sh;
                     unsigned long long cum = 0;
                     int sel = -1;
-                    for (int idx = 0; idx < ntile * 4; ++idx) {
-                        const unsigned long long x = chunk_sh[idx];
+                    for (int idx = 0; idx < ntile * 4; ++idx) {  // chunks in entry order: tile, then quarter
+                        const ulonglong2 cx = chunk[sq * ntile * 4 + idx];
+                        const unsigned long long x = use_r ? cx.x : cx.y;
                         if (sel < 0 && x > 0 && cum <= off && off < cum + x) {
                             sel = idx;
                             base_sh = cum;
@@ -657,9 +690,9 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     }
 }
 
-template <bool GREEDY, int NP>
+template <int NP, int APS>
 size_t ve_smem_bytes() {
-    return 1024 + (size_t)kVeStages * (kVeWBytes + NP * 128);
+    return 1024 + (size_t)ve_stages(NP, APS) * APS * (kVeWBytes + NP * 128);
 }
 
 struct VeLayout {
@@ -676,16 +709,16 @@ VeLayout ve_layout(int num_seqs, int total_draft) {
     return l;
 }
 
-template <bool GREEDY, int NP>
+template <bool GREEDY, int NP, int APS>
 int ve_launch(const CUtensorMap& wmap, const VeParams& p, int grid, const DeviceInfo& dev, cudaStream_t stream) {
-    static int configured[64] = {};
-    const size_t smem = ve_smem_bytes<GREEDY, NP>();
+    static int configured[64] = {};  // per instantiation (a template's own static)
+    const size_t smem = ve_smem_bytes<NP, APS>();
     if (dev.device >= 0 && dev.device < 64 && !configured[dev.device]) {
-        if (cudaFuncSetAttribute(verify_epilogue_kernel<GREEDY, NP>, cudaFuncAttributeMaxDynamicSharedMemorySize,
+        if (cudaFuncSetAttribute(verify_epilogue_kernel<GREEDY, NP, APS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
                                  (int)smem) != cudaSuccess)
             return BP_ERR_CUDA;
         int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, verify_epilogue_kernel<GREEDY, NP>, kVeThreads,
+        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, verify_epilogue_kernel<GREEDY, NP, APS>, kVeThreads,
                                                           smem) != cudaSuccess ||
             per_sm < 1)
             return BP_ERR_UNSUPPORTED;
@@ -701,7 +734,7 @@ int ve_launch(const CUtensorMap& wmap, const VeParams& p, int grid, const Device
     attr[0].val.cooperative = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 1;
-    return cudaLaunchKernelEx(&cfg, verify_epilogue_kernel<GREEDY, NP>, wmap, p) == cudaSuccess ? BP_OK
+    return cudaLaunchKernelEx(&cfg, verify_epilogue_kernel<GREEDY, NP, APS>, wmap, p) == cudaSuccess ? BP_OK
                                                                                                : BP_ERR_CUDA;
 }
 
@@ -711,7 +744,8 @@ size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft) {
     return ve_layout(num_seqs, total_draft).total;
 }
 
-int verify_epilogue_config(int rows, int vocab, int sm_count, int* grid, int* np, int* tiles_per_cta) {
+int verify_epilogue_config(int rows, int vocab, int hidden, int sm_count, int* grid, int* np, int* tiles_per_cta) {
+    if (hidden % kVeAtom != 0) return BP_ERR_UNSUPPORTED;
     const int tiles_total = (vocab + kVeM - 1) / kVeM;
     const int g = min(min(sm_count, kVeMaxGrid), tiles_total);
     if (g < 1 || rows < 1 || rows > 64) return BP_ERR_UNSUPPORTED;
@@ -729,7 +763,7 @@ int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, c
     const int rows_t = a.total_draft + a.num_seqs;
     const int rows = rows_t + (greedy ? 0 : a.total_draft);
     int grid = 0, NP = 0, per = 0;
-    int rc = verify_epilogue_config(rows, a.vocab, dev.sm_count, &grid, &NP, &per);
+    int rc = verify_epilogue_config(rows, a.vocab, a.hidden, dev.sm_count, &grid, &NP, &per);
     if (rc != BP_OK) return rc;
     const int tiles_total = (a.vocab + kVeM - 1) / kVeM;
     uint32_t cols = 32;
@@ -772,9 +806,18 @@ int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, c
     p.tot = reinterpret_cast<ulonglong2*>(ws + l.tot_off);
     p.sync = reinterpret_cast<unsigned int*>(ws + l.sync_off);
     p.err = a.err_word;
-    if (greedy) return NP == 32 ? ve_launch<true, 32>(wmap, p, grid, dev, stream)
-                                : ve_launch<true, 64>(wmap, p, grid, dev, stream);
-    return NP == 32 ? ve_launch<false, 32>(wmap, p, grid, dev, stream) : ve_launch<false, 64>(wmap, p, grid, dev, stream);
+    const bool two = p.atoms % 2 == 0;  // two atoms per stage where the hidden size allows
+    if (greedy && NP == 32)
+        return two ? ve_launch<true, 32, 2>(wmap, p, grid, dev, stream)
+                   : ve_launch<true, 32, 1>(wmap, p, grid, dev, stream);
+    if (greedy)
+        return two ? ve_launch<true, 64, 2>(wmap, p, grid, dev, stream)
+                   : ve_launch<true, 64, 1>(wmap, p, grid, dev, stream);
+    if (NP == 32)
+        return two ? ve_launch<false, 32, 2>(wmap, p, grid, dev, stream)
+                   : ve_launch<false, 32, 1>(wmap, p, grid, dev, stream);
+    return two ? ve_launch<false, 64, 2>(wmap, p, grid, dev, stream)
+               : ve_launch<false, 64, 1>(wmap, p, grid, dev, stream);
 }
 
 }  // namespace bp

@@ -246,7 +246,7 @@ def lm_head_weight(vocab: int, hidden: int, logit_std: float, seed: int) -> np.n
 
 
 def lm_head_inputs(w: Workload, temperature: float, hidden: int | None = None, push_prob: float = 0.85,
-                   boost: float = 18.0, weight: np.ndarray | None = None) -> dict:
+                   boost: float = 18.0, weight: np.ndarray | None = None, target_peak: float | None = None) -> dict:
     """LM-head weight, the final hidden states the verify epilogue projects, draft tokens, uniforms.
 
     W [V, H] from lm_head_weight.  Target states [sum (gamma_s + 1), H] ~ N(0, 1).  Draft token x_i
@@ -254,8 +254,11 @@ def lm_head_inputs(w: Workload, temperature: float, hidden: int | None = None, p
     N(0, 1 / logit_std^2) noise (its logits are the target's plus unit-variance noise) plus
     boost * w_x / |w_x|^2, which raises the drafter's logit of x_i by `boost`; with probability
     push_prob the target row's state gets the same push (the target agrees with the draft),
-    otherwise none.  States are rounded to bf16 last.  At T = 0 the drafter's states are not
-    returned (greedy acceptance reads the target rows only).
+    otherwise none.  With target_peak, every target row not pushed toward its draft (the rows of
+    rejected drafts and each sequence's last row) is pushed the same way toward a random token of
+    its own by target_peak, giving it a dominant token as a confident model's rows have.  States are
+    rounded to bf16 last.  At T = 0 the drafter's states are not returned (greedy acceptance reads
+    the target rows only).
     """
     gammas = np.asarray(w.block, dtype=np.int64) - 1
     cu_draft = offsets(gammas)
@@ -275,6 +278,12 @@ def lm_head_inputs(w: Workload, temperature: float, hidden: int | None = None, p
     h_draft = base[trow] + noise + dirs
     h_target = base.copy()
     h_target[trow[push]] += dirs[push]
+    if target_peak is not None:
+        free = np.ones(td + s, dtype=bool)
+        free[trow[push]] = False
+        fav = _rng(w.seed, 57).integers(0, V, size=td + s)
+        wf = bf16_bits_to_f32(W[fav[free]]).astype(np.float64)
+        h_target[free] += wf / np.maximum((wf * wf).sum(axis=1, keepdims=True), 1e-30) * target_peak
     out = dict(w=W, hidden=H, h_target=f32_to_bf16_bits(h_target.astype(np.float32)), draft_tokens=tokens,
                cu_draft=cu_draft, vocab=V, temperature=float(temperature),
                u_accept=_rng(w.seed, 55).random(td, dtype=np.float32),
