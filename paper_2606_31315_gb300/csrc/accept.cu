@@ -91,22 +91,6 @@ __device__ __forceinline__ float4 resid4(float4 p, float4 q) {
 __host__ __device__ inline size_t smem_bytes(int chunk4, bool greedy) { return (size_t)chunk4 * (greedy ? 16 : 32); }
 __host__ __device__ inline int warp_range(int chunk4) { return (chunk4 + kWarps - 1) / kWarps; }
 
-// Lane `lane` of a warp holding the values v[0..31] (per lane) ends with the warp-wide sum of
-// value `lane`: a butterfly that halves the values it carries at every step (31 shuffles).
-__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) {
-        const bool up = (lane & o) != 0;
-#pragma unroll
-        for (int q = 0; q < o; ++q) {
-            const float send = up ? v[q] : v[q + o];
-            const float keep = up ? v[q + o] : v[q];
-            v[q] = keep + __shfl_xor_sync(0xffffffffu, send, o);
-        }
-    }
-    return v[0];
-}
-
 // A warp's range of one row slice -> shared memory: one bulk copy (16-byte aligned rows, lane 0
 // issues it) or plain loads by the warp (padding past the vocabulary reads -inf).
 template <bool VEC>

@@ -60,4 +60,20 @@ __device__ __forceinline__ void amax_merge(float& v, int& i, float v2, int i2) {
     }
 }
 
+// Lane `lane` of a warp holding the values v[0..31] (per lane) ends with the warp-wide sum of
+// value `lane`: a butterfly that halves the values it carries at every step (31 shuffles).
+__device__ __forceinline__ float reduce_scatter32(float (&v)[32], int lane) {
+#pragma unroll
+    for (int o = 16; o >= 1; o >>= 1) {
+        const bool up = (lane & o) != 0;
+#pragma unroll
+        for (int q = 0; q < o; ++q) {
+            const float send = up ? v[q] : v[q + o];
+            const float keep = up ? v[q + o] : v[q];
+            v[q] = keep + __shfl_xor_sync(0xffffffffu, send, o);
+        }
+    }
+    return v[0];
+}
+
 }  // namespace bp

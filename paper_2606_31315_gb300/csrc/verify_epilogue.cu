@@ -169,29 +169,26 @@ __device__ __forceinline__ float2 amax_reduce_scatter32(float (&v)[32], int (&ix
     return make_float2(v[0], __int_as_float(ix[0]));
 }
 
-__device__ __forceinline__ float warp_sum_f(float x) {  // xor butterfly: bit-identical in every lane
-#pragma unroll
-    for (int o = 16; o >= 1; o >>= 1) x += __shfl_xor_sync(0xffffffffu, x, o);
-    return x;
-}
-
 // Weights of this lane's entry in tile t of the slice for one sequence's draw: x.x = r = max(0, p - q)
 // (0 without a draft row), x.y = p.  The crossing search recomputes them with this same code.
 struct DrawRow {
     int ct, cd;        // TMEM columns of the target row and the drafter row (cd < 0: none)
     float Mt, izt, Md, izd;
 };
+__device__ __forceinline__ float2 draw_weights(float lt, float ld, const DrawRow& d, bool in_vocab, float c2) {
+    if (!in_vocab) return make_float2(0.f, 0.f);
+    const float pv = __fmul_rn(ex2(__fsub_rn(__fmul_rn(lt, c2), d.Mt)), d.izt);
+    float rv = 0.f;
+    if (d.cd >= 0) rv = fmaxf(0.f, __fsub_rn(pv, __fmul_rn(ex2(__fsub_rn(__fmul_rn(ld, c2), d.Md)), d.izd)));
+    return make_float2(rv, pv);
+}
 template <int NP>
 __device__ __forceinline__ float2 entry_weights(uint32_t tmem_q, int t, const DrawRow& d, bool in_vocab, float c2) {
     const uint32_t col = (uint32_t)(t * NP);
     const float lt = __uint_as_float(tmem_ld1(tmem_q + col + (uint32_t)d.ct));
     const float ld = d.cd >= 0 ? __uint_as_float(tmem_ld1(tmem_q + col + (uint32_t)d.cd)) : 0.f;
     tmem_ld_wait();
-    if (!in_vocab) return make_float2(0.f, 0.f);
-    const float pv = __fmul_rn(ex2(__fsub_rn(__fmul_rn(lt, c2), d.Mt)), d.izt);
-    float rv = 0.f;
-    if (d.cd >= 0) rv = fmaxf(0.f, __fsub_rn(pv, __fmul_rn(ex2(__fsub_rn(__fmul_rn(ld, c2), d.Md)), d.izd)));
-    return make_float2(rv, pv);
+    return draw_weights(lt, ld, d, in_vocab, c2);
 }
 
 template <bool GREEDY, int NP, int APS>
@@ -207,7 +204,8 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     __shared__ float2 wst[4][64];      // per epilogue warp: statistics of each row over its lanes
     __shared__ float2 rst[64];         // statistics of each row over the whole vocabulary
     __shared__ int own_v[64], own_ct[64], own_cd[64], own_i[64];  // draft tokens held by the slice
-    __shared__ int cu_sh[65], k_sh[64];
+    __shared__ int cu_sh[65], k_sh[64], tok_sh[64];
+    __shared__ float ua_sh[64];
     __shared__ ulonglong2 wtot[4][64];
     __shared__ unsigned long long off_sh, base_sh;
     __shared__ int use_r_sh;
@@ -333,10 +331,14 @@ __global__ void __launch_bounds__(kVeThreads, 1)
         // ---- sequence offsets (read by every warp after grid barrier 1), then the draft tokens held
         // by this slice (their logits are captured by the epilogue)
         for (int i = lane; i <= S; i += 32) cu_sh[i] = p.cu_draft[i];
+        for (int i = lane; i < p.total_draft; i += 32) {  // inputs of the decisions, read before they are due
+            tok_sh[i] = p.tokens[i];
+            ua_sh[i] = GREEDY ? 0.f : p.u_accept[i];
+        }
         __syncwarp();
         if (!GREEDY) {
             for (int i = lane; i < p.total_draft; i += 32) {
-                const int x = p.tokens[i];
+                const int x = tok_sh[i];
                 if (x >= v0 && x < v1) {
                     int lo = 0, hi = S;  // sequence of draft i: cu[lo] <= i < cu[lo + 1]
                     while (hi - lo > 1) {
@@ -355,7 +357,7 @@ __global__ void __launch_bounds__(kVeThreads, 1)
         }
         if (c == 0)
             for (int i = lane; i < p.total_draft; i += 32) {
-                const int x = p.tokens[i];
+                const int x = tok_sh[i];
                 if (x < 0 || x >= p.vocab) raise_error(p.err, kErrDeviceArg);
             }
     } else {
@@ -461,6 +463,7 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     // ================= grid barrier 1: every slice's statistics and draft-token logits are out
     if (!grid_barrier(p.sync, (unsigned)grid, &ok_sh)) raise_error(p.err, kErrTimeout);
 
+    for (int sq = tid; sq < S; sq += kVeThreads) k_sh[sq] = cu_sh[sq + 1] - cu_sh[sq];  // no rejection yet
     // ---- row statistics over the whole vocabulary, merged in one fixed order in every CTA; a warp
     // takes rows warp, warp + 8, ... and keeps the loads of four rows in flight at once
     for (int r0 = warp; r0 < p.rows; r0 += 4 * (kVeThreads / 32)) {
@@ -498,39 +501,38 @@ __global__ void __launch_bounds__(kVeThreads, 1)
         }
     }
     __syncthreads();
-    // ---- ratios and the first rejection of every sequence (identical in every CTA)
-    if (warp == 0) {
-        for (int sq = lane; sq < S; sq += 32) {
-            const int d0 = cu_sh[sq], g = cu_sh[sq + 1] - d0;
-            int k = g;
-            for (int j = 0; j < g; ++j) {
-                const int i = d0 + j, ct = i + sq;
-                const int x = p.tokens[i];
-                float a;
-                if (GREEDY) {
-                    a = (x == __float_as_int(rst[ct].y)) ? 1.f : 0.f;
-                } else if (x < 0 || x >= p.vocab) {
-                    a = 0.f;
-                } else {
-                    const float2 xx = __ldcg(&p.xg[i]);
-                    const float2 st = rst[ct], sd = rst[p.rows_t + i];
-                    // a = min(1, p(x)/q(x)) in the log domain: 2^((xt - Mt) - (xd - Md)) * Zd / Zt
-                    const float lr = __fsub_rn(__fsub_rn(xx.x, st.x), __fsub_rn(xx.y, sd.x));
-                    a = fminf(1.f, ex2(lr) * __fdiv_rn(sd.y, st.y));
-                }
-                if (c == 0 && p.accept_prob) p.accept_prob[i] = a;
-                const bool rej = GREEDY ? (a == 0.f) : !(__ldg(p.u_accept + i) < a);
-                if (rej && k == g) k = j;
-            }
-            k_sh[sq] = k;
+    // ---- ratios of every drafted position (one thread each) and the first rejection of every
+    // sequence (identical in every CTA)
+    for (int i = tid; i < p.total_draft; i += kVeThreads) {
+        int sq = 0, hi = S;  // sequence of draft i: cu[sq] <= i < cu[sq + 1]
+        while (hi - sq > 1) {
+            const int mid = (sq + hi) >> 1;
+            if (cu_sh[mid] <= i) sq = mid; else hi = mid;
         }
+        const int ct = i + sq;
+        const int x = tok_sh[i];
+        float a;
+        if (GREEDY) {
+            a = (x == __float_as_int(rst[ct].y)) ? 1.f : 0.f;
+        } else if (x < 0 || x >= p.vocab) {
+            a = 0.f;
+        } else {
+            const float2 xx = __ldcg(&p.xg[i]);
+            const float2 st = rst[ct], sd = rst[p.rows_t + i];
+            // a = min(1, p(x)/q(x)) in the log domain: 2^((xt - Mt) - (xd - Md)) * Zd / Zt
+            const float lr = __fsub_rn(__fsub_rn(xx.x, st.x), __fsub_rn(xx.y, sd.x));
+            a = fminf(1.f, ex2(lr) * __fdiv_rn(sd.y, st.y));
+        }
+        if (c == 0 && p.accept_prob) p.accept_prob[i] = a;
+        const bool rej = GREEDY ? (a == 0.f) : !(ua_sh[i] < a);
+        if (rej) atomicMin(&k_sh[sq], i - cu_sh[sq]);
     }
     __syncthreads();
     if (c == 0) {  // n_accepted, the accepted drafts, -1 past the emitted slot (T = 0: the emitted argmax)
         for (int sq = warp; sq < S; sq += kVeThreads / 32) {
             const int d0 = cu_sh[sq], g = cu_sh[sq + 1] - d0, k = k_sh[sq], t0 = d0 + sq;
             for (int j = lane; j <= g; j += 32) {
-                if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
+                if (j < k) p.out_tokens[t0 + j] = tok_sh[d0 + j];
                 else if (j > k) p.out_tokens[t0 + j] = -1;
                 else if (GREEDY) p.out_tokens[t0 + j] = __float_as_int(rst[t0 + k].y);
             }
@@ -554,15 +556,36 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 d.izt = __fdiv_rn(1.f, rst[d.ct].y);
                 d.Md = d.cd >= 0 ? rst[d.cd].x : 0.f;
                 d.izd = d.cd >= 0 ? __fdiv_rn(1.f, rst[d.cd].y) : 0.f;
-                unsigned long long R = 0, P = 0;
-                for (int t = 0; t < ntile; ++t) {
-                    const float2 w = entry_weights<NP>(tq, t, d, v0 + t * kVeM + q * 32 + lane < v1, p.c2);
-                    const unsigned long long fr = to_fix(warp_sum_f(w.x)), fp = to_fix(warp_sum_f(w.y));
-                    if (lane == 0) chunk[(sq * ntile + t) * 4 + q] = make_ulonglong2(fr, fp);
-                    R += fr;
-                    P += fp;
+                // every tile's two columns first (one wait), then the weights of this lane's entries
+                uint32_t rt[kVeMaxTiles], rd[kVeMaxTiles];
+#pragma unroll
+                for (int t = 0; t < kVeMaxTiles; ++t) {
+                    if (t < ntile) {
+                        rt[t] = tmem_ld1(tq + (uint32_t)(t * NP + d.ct));
+                        rd[t] = d.cd >= 0 ? tmem_ld1(tq + (uint32_t)(t * NP + d.cd)) : 0u;
+                    }
                 }
-                if (lane == 0) wtot[q][sq] = make_ulonglong2(R, P);
+                tmem_ld_wait();
+                // lane t ends with the r-mass of tile t's chunk, lane 16 + t with its p-mass (31 shuffles)
+                float v[32];
+#pragma unroll
+                for (int t = 0; t < kVeMaxTiles; ++t) {
+                    float2 w = make_float2(0.f, 0.f);
+                    if (t < ntile)
+                        w = draw_weights(__uint_as_float(rt[t]), __uint_as_float(rd[t]), d,
+                                         v0 + t * kVeM + q * 32 + lane < v1, p.c2);
+                    v[t] = w.x;
+                    v[kVeMaxTiles + t] = w.y;
+                }
+                const unsigned long long f = to_fix(reduce_scatter32(v, lane));
+                const int tl = lane & (kVeMaxTiles - 1);
+                unsigned long long* cf = reinterpret_cast<unsigned long long*>(chunk);
+                if (tl < ntile) cf[((sq * ntile + tl) * 4 + q) * 2 + (lane >> 4)] = f;  // .x = r, .y = p
+                unsigned long long tot = tl < ntile ? f : 0ull;  // lanes 0-15 sum r, lanes 16-31 sum p
+#pragma unroll
+                for (int o = kVeMaxTiles / 2; o >= 1; o >>= 1) tot += __shfl_xor_sync(0xffffffffu, tot, o);
+                if (lane == 0) wtot[q][sq].x = tot;
+                if (lane == kVeMaxTiles) wtot[q][sq].y = tot;
             }
             named_sync(1, 128);
             for (int sq = tid - kVeEpi * 32; sq < S; sq += 128) {
@@ -632,20 +655,22 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 d.Md = d.cd >= 0 ? rst[d.cd].x : 0.f;
                 d.izd = d.cd >= 0 ? __fdiv_rn(1.f, rst[d.cd].y) : 0.f;
                 const bool use_r = use_r_sh != 0;
-                if (tid == kVeEpi * 32) {
+                if (warp == kVeEpi) {  // one warp scans the chunk masses in entry order (tile, then quarter)
                     const unsigned long long off = off_sh;
-                    unsigned long long cum = 0;
-                    int sel = -1;
-                    for (int idx = 0; idx < ntile * 4; ++idx) {  // chunks in entry order: tile, then quarter
-                        const ulonglong2 cx = chunk[sq * ntile * 4 + idx];
-                        const unsigned long long x = use_r ? cx.x : cx.y;
-                        if (sel < 0 && x > 0 && cum <= off && off < cum + x) {
-                            sel = idx;
-                            base_sh = cum;
-                        }
-                        cum += x;
+                    const int n = ntile * 4, i0 = 2 * lane;  // lane l holds chunks 2l and 2l + 1
+                    const ulonglong2 c0 = i0 < n ? chunk[sq * n + i0] : make_ulonglong2(0ull, 0ull);
+                    const ulonglong2 c1 = i0 + 1 < n ? chunk[sq * n + i0 + 1] : make_ulonglong2(0ull, 0ull);
+                    const unsigned long long x0 = use_r ? c0.x : c0.y, x1 = use_r ? c1.x : c1.y;
+                    const unsigned long long incl = warp_incl_scan(x0 + x1, lane);
+                    const unsigned long long b0 = incl - x1 - x0, b1 = incl - x1;
+                    const bool h0 = x0 > 0 && b0 <= off && off < b1, h1 = x1 > 0 && b1 <= off && off < incl;
+                    const unsigned hits = __ballot_sync(0xffffffffu, h0 || h1);  // exactly one with exact sums
+                    if (hits == 0u) {
+                        if (lane == 0) sel_sh = -1;
+                    } else if (lane == __ffs(hits) - 1) {
+                        sel_sh = h0 ? i0 : i0 + 1;
+                        base_sh = h0 ? b0 : b1;
                     }
-                    sel_sh = sel;
                 }
                 named_sync(1, 128);
                 const int sel = sel_sh;
