@@ -392,7 +392,8 @@ def run_ours(args):
         "next2_policy_head_32req_151936x2048": row(t_pol_big, big_bytes,
                                                    ["policy_gather_kernel", "policy_tc_kernel (streamed)"]),
         "next1_fused_verify_epilogue_qwen3_4b_t1": dict(
-            row(t_ve, ve_bytes, ["verify_epilogue_kernel<false,32>"]),
+            row(t_ve, ve_bytes, ["verify_epilogue_kernel<false,32,2>"]),
+            traffic=committed_traffic("verify_epilogue_kernel"),
             unfused_us=round(t_unfused * 1e6, 3),
             unfused="cuBLAS bf16 GEMM to logits + fp32 cast + accept_kernel"),
     }

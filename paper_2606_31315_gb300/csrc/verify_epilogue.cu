@@ -220,6 +220,15 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     const int J = ntile * spt;                          // ring stages of this CTA
     const int S = p.num_seqs;
 
+    // stage j of the ring: atoms a0 .. a0 + APS - 1 of tile t, both found from j
+    auto issue_w = [&](int j) {
+        const int st = j % STG, t = j / spt, a0 = (j - t * spt) * APS;
+        mbar_arrive_expect_tx(&wfull[st], APS * kVeWBytes);
+#pragma unroll
+        for (int u = 0; u < APS; ++u)
+            tma_load_2d(sW + (st * APS + u) * kVeWBytes, &wmap, &wfull[st], (a0 + u) * kVeAtom, (tile0 + t) * kVeM);
+    };
+    const int j_first = min(STG, J);  // stages issued before the block-wide set-up completes
     if (tid == 0) {
         prefetch_tensormap(&wmap);
         for (int st = 0; st < STG; ++st) {
@@ -231,6 +240,7 @@ __global__ void __launch_bounds__(kVeThreads, 1)
         mbar_init(&mma_done, 1);
         fence_mbar_init();
         own_n = 0;
+        for (int j = 0; j < j_first; ++j) issue_w(j);  // the W stream starts at once
     }
     if (warp == 1) {
         tmem_alloc(&tmem_sh, p.tmem_cols);
@@ -242,21 +252,16 @@ __global__ void __launch_bounds__(kVeThreads, 1)
     const uint32_t tmem = tmem_sh;
 
     if (warp == 0) {
-        // ---- W producer: the slice's LM-head rows, tile by tile, 64 hidden columns per stage
+        // ---- W producer: the slice's LM-head rows, tile by tile, APS x 64 hidden columns per stage
         if (lane == 0) {
-            int issued = 0;
-            for (int j = 0; j < J; ++j) {
+            int issued = j_first;
+            for (int j = j_first; j < J; ++j) {
                 const int st = j % STG;
-                if (j >= STG && !mbar_wait(&empty[st], ((j / STG) - 1) & 1, kWaitBudget)) {
+                if (!mbar_wait(&empty[st], ((j / STG) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
-                const int t = j / spt, a0 = (j - t * spt) * APS;
-                mbar_arrive_expect_tx(&wfull[st], APS * kVeWBytes);
-#pragma unroll
-                for (int u = 0; u < APS; ++u)
-                    tma_load_2d(sW + (st * APS + u) * kVeWBytes, &wmap, &wfull[st], (a0 + u) * kVeAtom,
-                                (tile0 + t) * kVeM);
+                issue_w(j);
                 issued = j + 1;
             }
             if (issued < J)  // wound down early: let the copies still in flight land before exiting

@@ -1,0 +1,84 @@
+"""One kernel of the hot path on its own, for profilers: seeded synthetic inputs of the benchmark's
+shapes on the device (nothing else allocated), a few warm-up calls, then N calls.
+
+    python -m paper_2606_31315_gb300.profile CASE [--calls N] [--warmup W]
+
+CASE is one of:
+  verify_epilogue_t1  Qwen3-4B LM head (151936 x 2560 bf16) fused with the acceptance, 16 target and
+                      15 drafter states, T = 1
+  verify_epilogue_t0  the same at T = 0 (16 target states)
+  accept_t1           acceptance over 16 x 151936 target and 15 x 151936 draft fp32 logits, T = 1
+  attention           causal verify attention, 1 sequence, 2048 + 16 keys, 32 / 8 heads, D = 128
+"""
+from __future__ import annotations
+
+import argparse
+
+import torch
+
+from . import _binding as bp
+
+V, H, CTX, B, HQ, HKV, D = 151936, 2560, 2048, 16, 32, 8, 128
+
+
+def _verify_epilogue(dev, gen, temperature):
+    td = B - 1
+    w = (torch.randn(V, H, device=dev, generator=gen) * (3.0 / H ** 0.5)).to(torch.bfloat16)
+    h_t = torch.randn(td + 1, H, device=dev, generator=gen).to(torch.bfloat16)
+    h_d = (h_t[:td].float() + torch.randn(td, H, device=dev, generator=gen) / 3).to(torch.bfloat16)
+    tok = torch.randint(0, V, (td,), device=dev, generator=gen, dtype=torch.int32)
+    cu = torch.tensor([0, td], dtype=torch.int32, device=dev)
+    ua, us = torch.rand(td, device=dev, generator=gen), torch.rand(1, device=dev, generator=gen)
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(1, td), dev)
+    return lambda: bp.verify_epilogue(w, h_t, h_d if temperature > 0 else None, tok, cu, temperature, ua, us,
+                                      want_accept_prob=False, ws=ws)
+
+
+def _accept(dev, gen):
+    td = B - 1
+    t = torch.randn(td + 1, V, device=dev, generator=gen) * 3
+    d = t[:td] + torch.randn(td, V, device=dev, generator=gen)
+    tok = torch.randint(0, V, (td,), device=dev, generator=gen, dtype=torch.int32)
+    cu = torch.tensor([0, td], dtype=torch.int32, device=dev)
+    ua, us = torch.rand(td, device=dev, generator=gen), torch.rand(1, device=dev, generator=gen)
+    ws = bp.workspace(bp.spec_accept_workspace_size(1, td, V), dev)
+    return lambda: bp.spec_accept(t, d, tok, cu, 1.0, ua, us, ws=ws)
+
+
+def _attention(dev, gen):
+    q = torch.randn(B, HQ, D, device=dev, generator=gen).to(torch.bfloat16)
+    k = torch.randn(CTX + B, HKV, D, device=dev, generator=gen).to(torch.bfloat16)
+    v = torch.randn(CTX + B, HKV, D, device=dev, generator=gen).to(torch.bfloat16)
+    cu_q = torch.tensor([0, B], dtype=torch.int32, device=dev)
+    cu_kv = torch.tensor([0, CTX + B], dtype=torch.int32, device=dev)
+    ws = bp.workspace(bp.block_attention_workspace_size(1, B, HQ, HKV, D), dev)
+    return lambda: bp.block_attention(q, k, v, cu_q, cu_kv, B, CTX + B, mask=bp.MASK_CAUSAL, ws=ws)
+
+
+CASES = {
+    "verify_epilogue_t1": lambda dev, gen: _verify_epilogue(dev, gen, 1.0),
+    "verify_epilogue_t0": lambda dev, gen: _verify_epilogue(dev, gen, 0.0),
+    "accept_t1": _accept,
+    "attention": _attention,
+}
+
+
+def main(argv=None) -> None:
+    ap = argparse.ArgumentParser(description=__doc__, formatter_class=argparse.RawDescriptionHelpFormatter)
+    ap.add_argument("case", choices=sorted(CASES))
+    ap.add_argument("--calls", type=int, default=3)
+    ap.add_argument("--warmup", type=int, default=2)
+    args = ap.parse_args(argv)
+    dev = torch.device("cuda:0")
+    gen = torch.Generator(device=dev)
+    gen.manual_seed(7)
+    bp.load()
+    call = CASES[args.case](dev, gen)
+    for _ in range(args.warmup + args.calls):
+        call()
+    torch.cuda.synchronize(dev)
+    print(f"{args.case}: {args.warmup} + {args.calls} calls done")
+
+
+if __name__ == "__main__":
+    main()
