@@ -1,8 +1,9 @@
 """BlockPilot fp64 CPU oracle -- test infrastructure only.
 
 A plain, slow restatement of the block-verify hot path (block attention, lossless
-speculative acceptance, block-size policy head, and the LM-head projection that
-feeds the acceptance) written from the paper, in fp64.
+speculative acceptance, block-size policy head, the LM-head projection that
+feeds the acceptance, and Appendix A's acceptance-length model) written from the
+paper, in fp64.
 Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline leg
 may import this package; the product path never does.  It shares no code with the
 CUDA library.  The arithmetic lives in ``bpo.c``; this module only marshals numpy
@@ -60,6 +61,9 @@ def _load():
         u16 = ctypes.POINTER(ctypes.c_uint16)
         lib.bpo_lm_head_logits.argtypes = [u16, u16, ctypes.c_int, ctypes.c_int, ctypes.c_int, dp, dp]
         lib.bpo_lm_head_logits.restype = ctypes.c_int
+        lib.bpo_tau_select.argtypes = [dp, ctypes.c_int, ctypes.c_int, ip, ctypes.c_int, ctypes.c_int,
+                                       ctypes.c_double, ip, dp, ip, dp, dp, dp]
+        lib.bpo_tau_select.restype = ctypes.c_int
         lib.bpo_num_threads.argtypes = []
         lib.bpo_num_threads.restype = ctypes.c_int
         _lib = lib
@@ -199,6 +203,34 @@ def verify_epilogue(w_bits, h_target_bits, h_draft_bits, draft_tokens, cu_draft,
     if with_abs:
         res.update(target_abs=ta, draft_abs=da)
     return res
+
+
+
+def tau_select(gamma, candidates, train_block: int, alpha: float, predicted=None):
+    """Appendix A: tau(b; x) for every candidate b, B*(x), and (given predicted B_hat) the regret.
+
+    gamma: [n, jmax] per-position predictability (jmax == 1: one gamma_x per request, geometric
+    form).  Returns dict(tau [n, C], best [n], regret [n] or None, lips [n], summary [4] =
+    (mean regret, mean |B* - B_hat|, L_tau, L_tau * mean |B* - B_hat|)).
+    """
+    g = np.ascontiguousarray(gamma, dtype=np.float64)
+    if g.ndim == 1:
+        g = g[:, None]
+    cand = _i32(candidates)
+    pred = _i32(predicted)
+    n, jmax = g.shape
+    tau = np.zeros((n, len(cand)), dtype=np.float64)
+    best = np.zeros(n, dtype=np.int32)
+    regret = np.zeros(n, dtype=np.float64) if pred is not None else None
+    lips = np.zeros(n, dtype=np.float64)
+    summary = np.zeros(4, dtype=np.float64)
+    dp, ip = ctypes.c_double, ctypes.c_int32
+    rc = _load().bpo_tau_select(_p(g, dp), n, jmax, _p(cand, ip), len(cand), int(train_block), float(alpha),
+                                _p(pred, ip), _p(tau, dp), _p(best, ip), _p(regret, dp), _p(lips, dp),
+                                _p(summary, dp))
+    if rc != 0:
+        raise ValueError(f"oracle tau_select rejected its arguments (rc={rc})")
+    return dict(tau=tau, best=best, regret=regret, lips=lips, summary=summary)
 
 
 if __name__ == "__main__":  # pragma: no cover

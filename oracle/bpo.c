@@ -14,7 +14,7 @@
  * entries).  Random numbers the method
  * draws (the acceptance uniforms and the resampling uniform) are inputs.
  *
- * Four parts, one per hot-path stage:
+ * Five parts:
  *   bpo_block_attention  -- block attention of a B-token block over a KV cache,
  *                           causal within the block (target verify pass) or
  *                           bidirectional within the block (dLLM drafter pass).
@@ -23,6 +23,9 @@
  *   bpo_lm_head_logits   -- the output projection that turns the final hidden
  *                           states of the verified (and drafted) positions into
  *                           the logits the acceptance reads.
+ *   bpo_tau_select       -- Appendix A's model of the expected acceptance length
+ *                           tau(b; x) per candidate block size, the optimal size
+ *                           B*(x), and the regret of a predicted size.
  *
  * Readings of the paper where it is silent are documented at each function.
  */
@@ -432,6 +435,102 @@ int bpo_lm_head_logits(const uint16_t *w, const uint16_t *h, int rows, int vocab
     }
     free(hd);
     return bad ? BPO_BAD_ARG : BPO_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Expected acceptance length per block size (Appendix A)                    */
+/* ------------------------------------------------------------------------- */
+/*
+ * Appendix A.1 writes the expected number of accepted drafts as a sum of
+ * prefix-survival probabilities, tau(b; x) = sum_{i=1}^{b} prod_{j=1}^{i}
+ * q_j(x, b).  Appendix A.2 factors the conditional acceptance into sample
+ * predictability and block-size retention, q_j(x, b) = gamma_j(x) r(b; B) with
+ * r(b; B) = exp(-alpha (b - B)^2), so that
+ *
+ *   tau(b; x) = sum_{i=1}^{b} r(b; B)^i prod_{j=1}^{i} gamma_j(x),
+ *
+ * and, for a predictability constant over positions (gamma_j = gamma_x), the
+ * finite geometric series tau = rho (1 - rho^b) / (1 - rho), rho = gamma_x r.
+ * B*(x) = argmax over the candidate set of tau(b; x) (lowest index on ties).
+ * Appendix A.3: the regret of a predicted size is R(x) = tau(B*) - tau(B_hat);
+ * with L the largest |tau(b1) - tau(b2)| / |b1 - b2| over the candidates
+ * (adjacent pairs of the ascending candidate list suffice), R(x) <= L |B* -
+ * B_hat|, and so E[R] <= L_tau E|B* - B_hat| with L_tau = max_x L(x).
+ *
+ * gamma [n][jmax] row-major: gamma_j(x) for j = 1..jmax at column j - 1.  With
+ * jmax == 1 the single value is gamma_x and tau uses the geometric form
+ * (rho == 1 gives tau = b).  candidates [nc], strictly increasing, each <= jmax
+ * unless jmax == 1.  predicted (may be NULL): B_hat per request, one of the
+ * candidates.  Outputs: tau [n][nc] (may be NULL), best [n], regret [n] and
+ * lips [n] (may be NULL; need predicted for regret), summary[4] (may be NULL):
+ * mean regret, mean |B* - B_hat|, L_tau, L_tau * mean |B* - B_hat|.
+ */
+static double tau_general(const double *g, int b, double r)
+{
+    double sum = 0.0, prod = 1.0;
+    for (int i = 1; i <= b; ++i) {
+        prod *= g[i - 1] * r; /* prod_{j<=i} gamma_j r */
+        sum += prod;
+    }
+    return sum;
+}
+
+static double tau_geometric(double gx, int b, double r)
+{
+    const double rho = gx * r;
+    if (rho == 1.0) return (double)b;
+    return rho * (1.0 - pow(rho, (double)b)) / (1.0 - rho);
+}
+
+int bpo_tau_select(const double *gamma, int n, int jmax, const int32_t *cand, int nc,
+                   int train_block, double alpha, const int32_t *predicted,
+                   double *tau, int32_t *best, double *regret, double *lips,
+                   double *summary)
+{
+    if (!gamma || !cand || !best || n < 0 || jmax < 1 || nc < 1 || !(alpha >= 0.0)) return BPO_BAD_ARG;
+    for (int c = 0; c < nc; ++c) {
+        if (cand[c] < 1 || (c > 0 && cand[c] <= cand[c - 1])) return BPO_BAD_ARG;
+        if (jmax > 1 && cand[c] > jmax) return BPO_BAD_ARG;
+    }
+    double sum_r = 0.0, sum_d = 0.0, lmax = 0.0;
+    for (int x = 0; x < n; ++x) {
+        const double *g = gamma + (size_t)x * jmax;
+        double t[64];
+        if (nc > 64) return BPO_BAD_ARG;
+        int bi = 0;
+        for (int c = 0; c < nc; ++c) {
+            const double d = (double)(cand[c] - train_block);
+            const double r = exp(-alpha * d * d);
+            t[c] = jmax == 1 ? tau_geometric(g[0], cand[c], r) : tau_general(g, cand[c], r);
+            if (tau) tau[(size_t)x * nc + c] = t[c];
+            if (t[c] > t[bi]) bi = c;
+        }
+        best[x] = cand[bi];
+        double l = 0.0;
+        for (int c = 1; c < nc; ++c) {
+            const double s = fabs(t[c] - t[c - 1]) / (double)(cand[c] - cand[c - 1]);
+            if (s > l) l = s;
+        }
+        if (lips) lips[x] = l;
+        if (l > lmax) lmax = l;
+        if (predicted) {
+            int pi = -1;
+            for (int c = 0; c < nc; ++c)
+                if (cand[c] == predicted[x]) pi = c;
+            if (pi < 0) return BPO_BAD_ARG;
+            const double rx = t[bi] - t[pi];
+            if (regret) regret[x] = rx;
+            sum_r += rx;
+            sum_d += fabs((double)(cand[bi] - cand[pi]));
+        }
+    }
+    if (summary) {
+        summary[0] = n ? sum_r / n : 0.0;
+        summary[1] = n ? sum_d / n : 0.0;
+        summary[2] = lmax;
+        summary[3] = lmax * summary[1];
+    }
+    return BPO_OK;
 }
 
 /* Number of OpenMP threads the oracle's parallel loops use (1 without OpenMP). */

@@ -292,6 +292,24 @@ def lm_head_inputs(w: Workload, temperature: float, hidden: int | None = None, p
     return out
 
 
+def tau_inputs(num_reqs: int, jmax: int = 24, seed: int = 60, train_block: int = 16, alpha: float = 0.001) -> dict:
+    """Per-request predictabilities for Appendix A's acceptance-length model and a predicted block size.
+
+    gamma_x ~ Beta(12, 2) per request (mean 0.86: tau(16) near the paper's 5.92 at B = 16); per
+    position gamma_j = clip(gamma_x + N(0, 0.03^2), 0.05, 0.999), [num_reqs, jmax] fp32.  The
+    predicted size is the candidate nearest to train_block + N(0, 1.5^2) (a predictor that
+    concentrates near the training size).  alpha is the retention constant of the model.
+    """
+    rng = _rng(seed, 61)
+    gx = rng.beta(12.0, 2.0, size=num_reqs).astype(np.float32)
+    noise = _rng(seed, 62).standard_normal((num_reqs, jmax), dtype=np.float32) * np.float32(0.03)
+    gamma = np.clip(gx[:, None] + noise, np.float32(0.05), np.float32(0.999)).astype(np.float32)
+    want = train_block + _rng(seed, 63).standard_normal(num_reqs) * 1.5
+    idx = np.abs(want[:, None] - CANDIDATES[None, :]).argmin(axis=1)
+    return dict(gamma=gamma, candidates=CANDIDATES.copy(), predicted=CANDIDATES[idx].astype(np.int32),
+                train_block=int(train_block), alpha=float(alpha))
+
+
 def as_f64(x: np.ndarray, dtype: str) -> np.ndarray:
     """The exact fp64 values of an f32 array or of bf16 bits."""
     if dtype == "bf16":
