@@ -377,6 +377,29 @@ def run_ours(args):
     ve_bytes = float(w_lm.numel() * 2 + h_all.numel() * 2)
     del w_lm, lg
 
+    # next row: Appendix A's acceptance-length model over 4M requests (24 positions each, the nine
+    # candidate sizes): tau per candidate, B*, regret of a predicted size, the bound's summary
+    n_tau, j_tau = 1 << 22, 24
+    torch.manual_seed(8)  # the Beta sampler draws from the global generator
+    gx = torch.distributions.Beta(torch.tensor(12.0, device=dev), torch.tensor(2.0, device=dev)).sample((n_tau, 1))
+    g_tau = (gx + 0.03 * torch.randn(n_tau, j_tau, device=dev, generator=gen)).clamp_(0.05, 0.999).contiguous()
+    cand_tau = wl.CANDIDATES  # host array
+    pred_tau = t(wl.CANDIDATES)[torch.randint(0, len(wl.CANDIDATES), (n_tau,), device=dev, generator=gen)].contiguous()
+    tau_out = torch.empty(n_tau, len(wl.CANDIDATES), device=dev)
+    best_tau = torch.empty(n_tau, dtype=torch.int32, device=dev)
+    reg_tau = torch.empty(n_tau, device=dev)
+    sum_tau = torch.empty(4, dtype=torch.float64, device=dev)
+    ws_tau = bp.workspace(bp.tau_select_workspace_size(n_tau), dev)
+
+    def tau_model(_c):
+        bp.tau_select(g_tau, cand_tau, 16, 0.001, predicted=pred_tau, tau=tau_out, best=best_tau, regret=reg_tau,
+                      summary=sum_tau, ws=ws_tau, stream=stream)
+
+    t_tau = time_calls(tau_model, n_graph=4, reps=20)
+    tau_bytes = float(g_tau.numel() * 4 + pred_tau.numel() * 4 + tau_out.numel() * 4 + best_tau.numel() * 4
+                      + reg_tau.numel() * 4)
+    del g_tau, tau_out
+
     def row(tsec, nbytes, kernels):
         gbs = nbytes / tsec / 1e9
         return {"us": round(tsec * 1e6, 3), "bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
@@ -396,6 +419,7 @@ def run_ours(args):
             traffic=committed_traffic("verify_epilogue_kernel"),
             unfused_us=round(t_unfused * 1e6, 3),
             unfused="cuBLAS bf16 GEMM to logits + fp32 cast + accept_kernel"),
+        "next4_tau_model_4M_requests": row(t_tau, tau_bytes, ["tau_kernel"]),
     }
     dom_name, dom_t, dom_bytes = ("accept_kernel", t_acc, accept_bytes(w, 1.0))
     traffic = committed_traffic(dom_name)

@@ -17,6 +17,7 @@
  * a shared pool named by a per-sequence block table) and append a block's K/V to it.
  * bp_verify_epilogue fuses the LM head that produces the logits with bp_spec_accept: it takes
  * the final hidden states of the verified and drafted positions instead of their logits.
+ * bp_tau_select evaluates Appendix A's acceptance-length model for a batch of requests.
  *
  * Conventions shared by every entry point
  *   - Pointers to tensors are DEVICE pointers (cudaMalloc / torch allocations), owned by
@@ -259,6 +260,37 @@ BP_API int bp_verify_epilogue(const void* lm_head, const void* h_target, const v
                               float temperature, const float* u_accept, const float* u_sample,
                               int32_t* n_accepted, int32_t* out_tokens, float* accept_prob, float* logits_out,
                               void* workspace, size_t workspace_bytes, void* stream);
+
+/* ---------------------------------------------------------------------------------
+ * Appendix A's model of the expected acceptance length over a batch of requests, the
+ * optimal block size of each request and the regret of a predicted one.  Appendix A.1-A.2:
+ *
+ *   tau(b; x) = sum_{i=1}^{b} r(b; B)^i prod_{j<=i} gamma_j(x),   r(b; B) = exp(-alpha (b - B)^2)
+ *
+ * (gamma_j(x): predictability of request x at drafted position j; B = train_block, the block
+ * size the drafter was trained with); B*(x) = argmax over the candidates of tau(b; x), lowest
+ * index on ties.  Appendix A.3: R(x) = tau(B*) - tau(B_hat) <= L(x) |B* - B_hat| with L(x) the
+ * largest |tau(b1) - tau(b2)| / |b1 - b2| over the candidates, so E[R] <= L_tau E|B* - B_hat|.
+ *
+ *   gamma        [num_reqs][jmax] fp32 device array; jmax == 1: one gamma_x per request
+ *                (constant predictability, the geometric form of Appendix A.2)
+ *   candidates   [num_cand] int32 HOST array (read during the call; the sizes and r(b; B) travel
+ *                to the GPU with the launch), strictly increasing, each in [1, 64] and <= jmax
+ *                when jmax > 1 (else BP_ERR_INVALID_ARG)
+ *   predicted    [num_reqs] int32 device array of predicted sizes, each one of the candidates
+ *                (else BP_ERR_DEVICE_FLAG), or NULL
+ *   tau_out      [num_reqs][num_cand] fp32 out, may be NULL; best_out [num_reqs] int32 out: B*
+ *   regret_out   [num_reqs] fp32 out, may be NULL (needs predicted)
+ *   summary_out  [4] fp64 out, may be NULL: mean R, mean |B* - B_hat| (both 0 without
+ *                predicted), L_tau, L_tau * mean |B* - B_hat| (the bound on mean R)
+ * Limits: jmax <= 64, num_cand <= 32 (else BP_ERR_UNSUPPORTED).  Sums of the summary are formed
+ * in a fixed order: the result does not depend on scheduling.
+ * ------------------------------------------------------------------------------- */
+BP_API size_t bp_tau_select_workspace_size(int num_reqs);
+BP_API int bp_tau_select(const float* gamma, int num_reqs, int jmax, const int32_t* candidates, int num_cand,
+                         int train_block, float alpha, const int32_t* predicted, float* tau_out, int32_t* best_out,
+                         float* regret_out, double* summary_out, void* workspace, size_t workspace_bytes,
+                         void* stream);
 
 /* Reads and clears the sticky device error word of `workspace` (synchronizes `stream`).
  * Returns BP_OK, BP_ERR_TIMEOUT or BP_ERR_DEVICE_FLAG (or BP_ERR_CUDA if the read fails). */

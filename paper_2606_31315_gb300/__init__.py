@@ -22,6 +22,8 @@ from ._binding import (  # noqa: F401
     policy_select_workspace_size,
     spec_accept,
     spec_accept_workspace_size,
+    tau_select,
+    tau_select_workspace_size,
     verify_epilogue,
     verify_epilogue_workspace_size,
     workspace,

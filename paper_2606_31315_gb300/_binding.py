@@ -10,6 +10,7 @@ from __future__ import annotations
 import ctypes
 import os
 
+import numpy as np
 import torch
 
 from . import _build
@@ -77,6 +78,10 @@ def load():
     lib.bp_verify_epilogue.argtypes = [vp, vp, vp, i32, i32, vp, vp, i32, i32, f32, vp, vp, vp, vp, vp, vp, vp, sz,
                                        vp]
     lib.bp_verify_epilogue.restype = i32
+    lib.bp_tau_select_workspace_size.argtypes = [i32]
+    lib.bp_tau_select_workspace_size.restype = sz
+    lib.bp_tau_select.argtypes = [vp, i32, i32, vp, i32, i32, f32, vp, vp, vp, vp, vp, vp, sz, vp]
+    lib.bp_tau_select.restype = i32
     lib.bp_get_status.argtypes = [vp, vp]
     lib.bp_get_status.restype = i32
     _lib = lib
@@ -251,6 +256,40 @@ def verify_epilogue(lm_head, h_target, h_draft, draft_tokens, cu_draft, temperat
                                 ws.numel(), _stream(stream))
     _check(rc, "bp_verify_epilogue")
     return n_accepted, out_tokens, accept_prob
+
+
+# --------------------------------------------------------------------------- acceptance-length model
+def tau_select_workspace_size(num_reqs) -> int:
+    return int(load().bp_tau_select_workspace_size(num_reqs))
+
+
+def tau_select(gamma, candidates, train_block: int, alpha: float, predicted=None, tau=None, best=None, regret=None,
+               summary=None, want_tau=True, ws=None, stream=None):
+    """Appendix A's tau(b; x), B*(x) and regret; see ``bp_tau_select``.  candidates is a host
+    sequence (list, numpy array or CPU tensor).  Returns (tau, best, regret, summary)."""
+    lib = load()
+    for t, n in ((gamma, "gamma"), (predicted, "predicted")):
+        _cuda(t, n)
+    g = gamma if gamma.dim() == 2 else gamma.reshape(-1, 1)
+    n, jmax = g.shape
+    cand = np.ascontiguousarray(candidates.cpu().numpy() if torch.is_tensor(candidates) else candidates,
+                                dtype=np.int32)  # a host array
+    nc = cand.size
+    dev = gamma.device
+    if tau is None and want_tau:
+        tau = torch.empty(n, nc, dtype=torch.float32, device=dev)
+    if best is None:
+        best = torch.empty(n, dtype=torch.int32, device=dev)
+    if regret is None and predicted is not None:
+        regret = torch.empty(n, dtype=torch.float32, device=dev)
+    if summary is None:
+        summary = torch.empty(4, dtype=torch.float64, device=dev)
+    if ws is None:
+        ws = workspace(lib.bp_tau_select_workspace_size(n), dev)
+    rc = lib.bp_tau_select(_ptr(g), n, jmax, cand.ctypes.data, nc, int(train_block), float(alpha), _ptr(predicted),
+                           _ptr(tau), _ptr(best), _ptr(regret), _ptr(summary), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "bp_tau_select")
+    return tau, best, regret, summary
 
 
 # --------------------------------------------------------------------------- policy head

@@ -316,6 +316,37 @@ int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_
     return rc;
 }
 
+size_t bp_tau_select_workspace_size(int num_reqs) {
+    if (num_reqs < 0) return 0;
+    return sizeof(WorkspaceHeader) + tau_scratch_bytes(num_reqs);
+}
+
+int bp_tau_select(const float* gamma, int num_reqs, int jmax, const int32_t* candidates, int num_cand, int train_block,
+                  float alpha, const int32_t* predicted, float* tau_out, int32_t* best_out, float* regret_out,
+                  double* summary_out, void* workspace, size_t workspace_bytes, void* stream) {
+    if (num_reqs < 0 || jmax < 1 || num_cand < 1 || !(alpha >= 0.f) || isinf(alpha)) return BP_ERR_INVALID_ARG;
+    if (num_reqs == 0) return BP_OK;
+    if (!gamma || !candidates || !best_out || (regret_out && !predicted)) return BP_ERR_INVALID_ARG;
+    if (num_cand > 32 || jmax > 64) return BP_ERR_UNSUPPORTED;
+    for (int c = 0; c < num_cand; ++c) {  // strictly increasing sizes within the rows (a host array)
+        const int b = candidates[c];
+        if (b < 1 || b > 64 || (jmax > 1 && b > jmax) || (c > 0 && b <= candidates[c - 1])) return BP_ERR_INVALID_ARG;
+    }
+    int rc = check_workspace(workspace, workspace_bytes, bp_tau_select_workspace_size(num_reqs));
+    if (rc != BP_OK) return rc;
+    DeviceInfo dev;
+    if ((rc = device_info(&dev)) != BP_OK) return rc;
+    TauArgs a;
+    a.gamma = gamma; a.num_reqs = num_reqs; a.jmax = jmax; a.candidates = candidates; a.num_cand = num_cand;
+    a.train_block = train_block; a.alpha = alpha; a.predicted = predicted; a.tau_out = tau_out;
+    a.best_out = best_out; a.regret_out = regret_out; a.summary_out = summary_out;
+    a.scratch = scratch(workspace);
+    a.err_word = err_word(workspace);
+    rc = launch_tau(a, dev, static_cast<cudaStream_t>(stream));
+    if (rc == BP_ERR_CUDA) cudaGetLastError();
+    return rc;
+}
+
 size_t bp_policy_select_workspace_size(int num_reqs, int d_in, int hidden, int num_cand) {
     if (num_reqs < 0 || d_in < 1 || hidden < 1 || num_cand < 1) return 0;
     return sizeof(WorkspaceHeader) + policy_scratch_bytes(num_reqs, d_in, hidden, num_cand);

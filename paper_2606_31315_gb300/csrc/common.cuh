@@ -138,4 +138,21 @@ size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft);
 int verify_epilogue_config(int rows, int vocab, int hidden, int sm_count, int* grid, int* np, int* tiles_per_cta);
 int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
+struct TauArgs {
+    const float* gamma;         // [num_reqs][jmax]
+    int num_reqs, jmax;
+    const int32_t* candidates;  // [num_cand] HOST array, strictly increasing
+    int num_cand, train_block;
+    float alpha;
+    const int32_t* predicted;   // [num_reqs] or null
+    float* tau_out;             // [num_reqs][num_cand] or null
+    int32_t* best_out;          // [num_reqs]
+    float* regret_out;          // [num_reqs] or null
+    double* summary_out;        // [4] or null
+    void* scratch;
+    unsigned int* err_word;
+};
+size_t tau_scratch_bytes(int num_reqs);
+int launch_tau(const TauArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+
 }  // namespace bp

@@ -9,6 +9,8 @@ CASE is one of:
   verify_epilogue_t0  the same at T = 0 (16 target states)
   accept_t1           acceptance over 16 x 151936 target and 15 x 151936 draft fp32 logits, T = 1
   attention           causal verify attention, 1 sequence, 2048 + 16 keys, 32 / 8 heads, D = 128
+  tau                 Appendix A's acceptance-length model over 4M requests (24 positions, nine
+                      candidate sizes, a predicted size each)
 """
 from __future__ import annotations
 
@@ -55,11 +57,22 @@ def _attention(dev, gen):
     return lambda: bp.block_attention(q, k, v, cu_q, cu_kv, B, CTX + B, mask=bp.MASK_CAUSAL, ws=ws)
 
 
+def _tau(dev, gen):
+    n, j = 1 << 22, 24
+    g = (0.86 + 0.05 * torch.randn(n, j, device=dev, generator=gen)).clamp_(0.05, 0.999).contiguous()
+    cand = list(range(8, 25, 2))
+    pred = torch.tensor(cand, dtype=torch.int32, device=dev)[torch.randint(0, len(cand), (n,), device=dev,
+                                                                           generator=gen)].contiguous()
+    ws = bp.workspace(bp.tau_select_workspace_size(n), dev)
+    return lambda: bp.tau_select(g, cand, 16, 0.001, predicted=pred, ws=ws)
+
+
 CASES = {
     "verify_epilogue_t1": lambda dev, gen: _verify_epilogue(dev, gen, 1.0),
     "verify_epilogue_t0": lambda dev, gen: _verify_epilogue(dev, gen, 0.0),
     "accept_t1": _accept,
     "attention": _attention,
+    "tau": _tau,
 }
 
 

@@ -135,6 +135,26 @@ def test_verify_epilogue_host_validation_needs_no_gpu(lib):
         assert call(temp=0.0, h_draft=None) == 3  # valid; no device to run on
 
 
+def test_tau_select_host_validation_needs_no_gpu(lib):
+    vp, f32 = ctypes.c_void_p, ctypes.c_float
+    fake, ws = vp(0x10000), vp(0x20000)
+
+    cands = (ctypes.c_int32 * 9)(*range(8, 25, 2))  # a host array
+
+    def call(n=1000, jmax=24, nc=9, alpha=0.001, pred=fake, regret=fake, best=fake, cand=cands):
+        return lib.bp_tau_select(fake, n, jmax, cand, nc, 16, f32(alpha), pred, fake, best, regret, fake, ws, 1 << 20,
+                                 None)
+    assert lib.bp_tau_select_workspace_size(1000) >= 256 + 4 * 8 * 4
+    assert call(alpha=-1.0) == 1 and call(jmax=0) == 1 and call(best=None) == 1
+    assert call(pred=None) == 1                  # a regret needs predicted sizes
+    assert call(nc=33) == 2 and call(jmax=65) == 2
+    assert call(n=0) == 0
+    if not __import__("torch").cuda.is_available():
+        assert call() == 3                         # valid; no device to run on
+        assert call(jmax=20) == 1                  # candidate 22 beyond 20-position rows
+        assert call(cand=(ctypes.c_int32 * 9)(8, 10, 12, 14, 16, 18, 20, 24, 22)) == 1  # not increasing
+
+
 def test_no_cpu_fallback_without_gpu(lib):
     import torch
 
