@@ -200,18 +200,19 @@ __global__ void __launch_bounds__(kTauThreads) tau_finish_kernel(const double* _
     fin[tid][0] = a;
     fin[tid][1] = b;
     fin[tid][2] = c;
-    __syncthreads();
-    if (tid == 0) {
-        double A = 0.0, Bs = 0.0, C = 0.0;
-        for (int k = 0; k < kTauThreads; ++k) {
-            A += fin[k][0];
-            Bs += fin[k][1];
-            C = fmax(C, fin[k][2]);
+    for (int h = kTauThreads / 2; h >= 1; h >>= 1) {  // a fixed-order tree
+        __syncthreads();
+        if (tid < h) {
+            fin[tid][0] += fin[tid + h][0];
+            fin[tid][1] += fin[tid + h][1];
+            fin[tid][2] = fmax(fin[tid][2], fin[tid + h][2]);
         }
-        summary[0] = A / (double)n;
-        summary[1] = Bs / (double)n;
-        summary[2] = C;
-        summary[3] = C * (Bs / (double)n);
+    }
+    if (tid == 0) {
+        summary[0] = fin[0][0] / (double)n;
+        summary[1] = fin[0][1] / (double)n;
+        summary[2] = fin[0][2];
+        summary[3] = fin[0][2] * (fin[0][1] / (double)n);
     }
 }
 
@@ -287,13 +288,20 @@ int launch_tau(const TauArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
     p.part = reinterpret_cast<double*>(a.scratch);
     p.err = a.err_word;
     // register rows of 24, 32 or 64 prefix products (64 for one gamma per request: sizes up to 64),
-    // 12 or 32 candidate columns
-    const bool few = a.num_cand <= 12;
-    if (a.jmax > 1 && a.jmax <= 24)
-        return few ? tau_launch<24, 12>(a, p, dev, stream) : tau_launch<24, 32>(a, p, dev, stream);
-    if (a.jmax > 1 && a.jmax <= 32)
-        return few ? tau_launch<32, 12>(a, p, dev, stream) : tau_launch<32, 32>(a, p, dev, stream);
-    return few ? tau_launch<64, 12>(a, p, dev, stream) : tau_launch<64, 32>(a, p, dev, stream);
+    // 9, 16 or 32 candidate columns
+    // (9 columns: the nine candidate sizes 8, 10, ..., 24 of the paper's setting; padding columns cost
+    // a multiply-add each)
+    const int nc = a.num_cand;
+    if (a.jmax > 1 && a.jmax <= 24) {
+        if (nc <= 9) return tau_launch<24, 9>(a, p, dev, stream);
+        return nc <= 16 ? tau_launch<24, 16>(a, p, dev, stream) : tau_launch<24, 32>(a, p, dev, stream);
+    }
+    if (a.jmax > 1 && a.jmax <= 32) {
+        if (nc <= 9) return tau_launch<32, 9>(a, p, dev, stream);
+        return nc <= 16 ? tau_launch<32, 16>(a, p, dev, stream) : tau_launch<32, 32>(a, p, dev, stream);
+    }
+    if (nc <= 9) return tau_launch<64, 9>(a, p, dev, stream);
+    return nc <= 16 ? tau_launch<64, 16>(a, p, dev, stream) : tau_launch<64, 32>(a, p, dev, stream);
 }
 
 }  // namespace bp
