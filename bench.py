@@ -419,7 +419,8 @@ def run_ours(args):
             traffic=committed_traffic("verify_epilogue_kernel"),
             unfused_us=round(t_unfused * 1e6, 3),
             unfused="cuBLAS bf16 GEMM to logits + fp32 cast + accept_kernel"),
-        "next4_tau_model_4M_requests": row(t_tau, tau_bytes, ["tau_kernel"]),
+        "next4_tau_model_4M_requests": dict(row(t_tau, tau_bytes, ["tau_kernel<24,9>", "tau_finish_kernel"]),
+                                            traffic=committed_traffic("tau_kernel")),
     }
     dom_name, dom_t, dom_bytes = ("accept_kernel", t_acc, accept_bytes(w, 1.0))
     traffic = committed_traffic(dom_name)
