@@ -2,8 +2,8 @@
 
 A plain, slow restatement of the block-verify hot path (block attention, lossless
 speculative acceptance, block-size policy head, the LM-head projection that
-feeds the acceptance, and Appendix A's acceptance-length model) written from the
-paper, in fp64.
+feeds the acceptance, Appendix A's acceptance-length model, and the commit of the
+decoding loop) written from the paper, in fp64.
 Only the tests, ``__graft_entry__.smoke()`` and the benchmark's CPU-baseline leg
 may import this package; the product path never does.  It shares no code with the
 CUDA library.  The arithmetic lives in ``bpo.c``; this module only marshals numpy
@@ -64,6 +64,8 @@ def _load():
         lib.bpo_tau_select.argtypes = [dp, ctypes.c_int, ctypes.c_int, ip, ctypes.c_int, ctypes.c_int,
                                        ctypes.c_double, ip, dp, ip, dp, dp, dp]
         lib.bpo_tau_select.restype = ctypes.c_int
+        lib.bpo_verify_commit.argtypes = [ip, ip, ip, ip, ctypes.c_int, ctypes.c_int, ip, ip]
+        lib.bpo_verify_commit.restype = ctypes.c_int
         lib.bpo_num_threads.argtypes = []
         lib.bpo_num_threads.restype = ctypes.c_int
         _lib = lib
@@ -231,6 +233,25 @@ def tau_select(gamma, candidates, train_block: int, alpha: float, predicted=None
     if rc != 0:
         raise ValueError(f"oracle tau_select rejected its arguments (rc={rc})")
     return dict(tau=tau, best=best, regret=regret, lips=lips, summary=summary)
+
+
+
+def verify_commit(ctx, n_accepted, out_tokens, cu_draft, capacity: int):
+    """The decoding loop's commit after a verify step: new context lengths (anchor + accepted drafts
+    stay), the next anchors and the next pass's key offsets.  Returns dict(ctx, anchor, cu_kv)."""
+    c = np.array(ctx, dtype=np.int32)
+    n = _i32(n_accepted)
+    out = _i32(out_tokens)
+    cu = _i32(cu_draft)
+    s = len(c)
+    anchor = np.zeros(s, dtype=np.int32)
+    cu_kv = np.zeros(s + 1, dtype=np.int32)
+    ip = ctypes.c_int32
+    rc = _load().bpo_verify_commit(_p(c, ip), _p(n, ip), _p(out, ip), _p(cu, ip), s, int(capacity), _p(anchor, ip),
+                                   _p(cu_kv, ip))
+    if rc != 0:
+        raise ValueError(f"oracle verify_commit rejected its arguments (rc={rc})")
+    return dict(ctx=c, anchor=anchor, cu_kv=cu_kv)
 
 
 if __name__ == "__main__":  # pragma: no cover

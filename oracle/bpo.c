@@ -14,7 +14,7 @@
  * entries).  Random numbers the method
  * draws (the acceptance uniforms and the resampling uniform) are inputs.
  *
- * Five parts:
+ * Six parts:
  *   bpo_block_attention  -- block attention of a B-token block over a KV cache,
  *                           causal within the block (target verify pass) or
  *                           bidirectional within the block (dLLM drafter pass).
@@ -26,6 +26,8 @@
  *   bpo_tau_select       -- Appendix A's model of the expected acceptance length
  *                           tau(b; x) per candidate block size, the optimal size
  *                           B*(x), and the regret of a predicted size.
+ *   bpo_verify_commit    -- the step of the decoding loop after acceptance: what
+ *                           stays in each sequence's KV cache, and the next block.
  *
  * Readings of the paper where it is silent are documented at each function.
  */
@@ -529,6 +531,46 @@ int bpo_tau_select(const double *gamma, int n, int jmax, const int32_t *cand, in
         summary[1] = n ? sum_d / n : 0.0;
         summary[2] = lmax;
         summary[3] = lmax * summary[1];
+    }
+    return BPO_OK;
+}
+
+/* ------------------------------------------------------------------------- */
+/* Commit of a verify step (the decoding loop around Figure 1)               */
+/* ------------------------------------------------------------------------- */
+/*
+ * Section 2.1 / Figure 1 and Section 2.4: every step drafts a block of B_s =
+ * gamma_s + 1 positions (the anchor -- the last token emitted -- and gamma_s
+ * drafts), the target verifies the whole block in one pass (so the K/V rows of
+ * all B_s positions are appended to the cache), keeps the longest accepted
+ * prefix and emits one more token; the block size is fixed for the request.
+ * The rows that stay are those of the anchor and the n_acc accepted drafts:
+ *
+ *   ctx_s  <-  ctx_s + 1 + n_acc_s         (the rejected drafts' rows drop out)
+ *   anchor_s = the token emitted at slot n_acc_s of the step
+ *   cu_kv_next[s+1] - cu_kv_next[s] = ctx_s + B_s  (the next verify pass's keys)
+ *
+ * ctx [S] in/out, n_acc [S], out_tokens [total_draft + S] (slots of sequence s
+ * start at cu_draft[s] + s), cu_draft [S+1]; capacity = rows the cache can hold
+ * per sequence.  Returns BPO_BAD_ARG (and changes nothing) if some n_acc is
+ * outside [0, gamma_s] or the next pass would not fit the capacity.
+ */
+int bpo_verify_commit(int32_t *ctx, const int32_t *n_acc, const int32_t *out_tokens,
+                      const int32_t *cu_draft, int num_seqs, int capacity,
+                      int32_t *anchor_out, int32_t *cu_kv_next)
+{
+    if (!ctx || !n_acc || !out_tokens || !cu_draft || !cu_kv_next || num_seqs < 0) return BPO_BAD_ARG;
+    for (int s = 0; s < num_seqs; ++s) {
+        const int gamma = cu_draft[s + 1] - cu_draft[s];
+        if (n_acc[s] < 0 || n_acc[s] > gamma) return BPO_BAD_ARG;
+        if ((long long)ctx[s] + 1 + n_acc[s] + gamma + 1 > capacity) return BPO_BAD_ARG;
+    }
+    cu_kv_next[0] = 0;
+    for (int s = 0; s < num_seqs; ++s) {
+        const int gamma = cu_draft[s + 1] - cu_draft[s];
+        ctx[s] += 1 + n_acc[s];
+        if (anchor_out) anchor_out[s] = out_tokens[cu_draft[s] + s + n_acc[s]];
+        cu_kv_next[s + 1] = cu_kv_next[s] + ctx[s] + gamma + 1;
     }
     return BPO_OK;
 }
