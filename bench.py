@@ -377,6 +377,48 @@ def run_ours(args):
     ve_bytes = float(w_lm.numel() * 2 + h_all.numel() * 2)
     del w_lm, lg
 
+    # next row: the decoding loop on the device -- each step runs 36 layers (Qwen3-4B) of append-the-block
+    # + paged verify attention, the T=1 acceptance and the commit (lengths back to the accepted prefix,
+    # next offsets on the device); a graph of 8 steps that starts by resetting the lengths, replayed
+    n_layers, g_steps, page_l = 36, 8, 64
+    ctx0, blk = int(w.ctx[0]), int(w.block[0])
+    cap_l = -(-(ctx0 + (g_steps + 1) * blk) // page_l) * page_l
+    pps_l = cap_l // page_l
+    pool_k = [torch.randn(cap_l, w.num_kv_heads, w.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+              for _ in range(n_layers)]
+    pool_v = [torch.randn(cap_l, w.num_kv_heads, w.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+              for _ in range(n_layers)]
+    bt_l = torch.arange(pps_l, dtype=torch.int32, device=dev).view(1, pps_l)
+    kn_l = torch.randn(blk, w.num_kv_heads, w.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+    vn_l = torch.randn(blk, w.num_kv_heads, w.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+    o_l = torch.empty(blk, w.num_q_heads, w.head_dim, dtype=torch.bfloat16, device=dev)
+    cu_q_l = torch.tensor([0, blk], dtype=torch.int32, device=dev)
+    ctx_init = torch.tensor([ctx0], dtype=torch.int32, device=dev)
+    cu_kv_init = torch.tensor([0, ctx0 + blk], dtype=torch.int32, device=dev)
+    ctx_d, cu_kv_d = ctx_init.clone(), cu_kv_init.clone()
+    na_l, ot_l = torch.empty(1, dtype=torch.int32, device=dev), torch.empty(blk, dtype=torch.int32, device=dev)
+    anc_l = torch.empty(1, dtype=torch.int32, device=dev)
+    ws_acc_l = bp.workspace(bp.spec_accept_workspace_size(1, blk - 1, w.vocab), dev)
+    ws_c = bp.workspace(256, dev)
+    c0_ = copies[0]
+
+    def loop_steps(_c):
+        with torch.cuda.stream(stream):
+            ctx_d.copy_(ctx_init)
+            cu_kv_d.copy_(cu_kv_init)
+        for _ in range(g_steps):
+            for l in range(n_layers):
+                bp.kv_append(pool_k[l], pool_v[l], kn_l, vn_l, cu_q_l, cu_kv_d, bt_l, page_l, stream=stream)
+                bp.block_attention_paged(c0_["q"], pool_k[l], pool_v[l], cu_q_l, cu_kv_d, bt_l, page_l, cap_l, blk,
+                                         cap_l, out=o_l, ws=ws_a, stream=stream)
+            bp.spec_accept(c0_["target"], c0_["draft"], c0_["tok"], cu_d, 1.0, c0_["ua"], c0_["us"], n_accepted=na_l,
+                           out_tokens=ot_l, want_accept_prob=False, ws=ws_acc_l, stream=stream)
+            bp.verify_commit(ctx_d, na_l, ot_l, cu_d, cap_l, anchor=anc_l, cu_kv_next=cu_kv_d, ws=ws_c, stream=stream)
+
+    t_loop = time_calls(loop_steps, n_graph=1, reps=10) / g_steps
+    loop_bytes = n_layers * (attention_bytes(w) + 2 * kn_l.numel() * 2 * 2) + accept_bytes(w, 1.0)
+    del pool_k, pool_v
+
     # next row: Appendix A's acceptance-length model over 4M requests (24 positions each, the nine
     # candidate sizes): tau per candidate, B*, regret of a predicted size, the bound's summary
     n_tau, j_tau = 1 << 22, 24
@@ -419,6 +461,11 @@ def run_ours(args):
             traffic=committed_traffic("verify_epilogue_kernel"),
             unfused_us=round(t_unfused * 1e6, 3),
             unfused="cuBLAS bf16 GEMM to logits + fp32 cast + accept_kernel"),
+        "next3_verify_loop_step_qwen3_4b_36_layers": dict(
+            row(t_loop, loop_bytes, ["kv_append_kernel", "attn_bf16_tc_kernel (paged)", "accept_kernel<false,true>",
+                                     "verify_commit_kernel"]),
+            per_step="36 x (append + paged verify attention, 64-row pages) + T=1 acceptance + commit; the "
+                     "context grows from 2048 by the accepted prefix each step; bytes counted at 2048 + 16 keys"),
         "next4_tau_model_4M_requests": dict(row(t_tau, tau_bytes, ["tau_kernel<24,9>", "tau_finish_kernel"]),
                                             traffic=committed_traffic("tau_kernel")),
     }

@@ -18,6 +18,7 @@
  * bp_verify_epilogue fuses the LM head that produces the logits with bp_spec_accept: it takes
  * the final hidden states of the verified and drafted positions instead of their logits.
  * bp_tau_select evaluates Appendix A's acceptance-length model for a batch of requests.
+ * bp_verify_commit rolls the KV lengths back to the accepted prefix on the device, closing the loop.
  *
  * Conventions shared by every entry point
  *   - Pointers to tensors are DEVICE pointers (cudaMalloc / torch allocations), owned by
@@ -291,6 +292,31 @@ BP_API int bp_tau_select(const float* gamma, int num_reqs, int jmax, const int32
                          int train_block, float alpha, const int32_t* predicted, float* tau_out, int32_t* best_out,
                          float* regret_out, double* summary_out, void* workspace, size_t workspace_bytes,
                          void* stream);
+
+/* ---------------------------------------------------------------------------------
+ * Commit of a verify step: the decoding loop's bookkeeping after the acceptance, on the device,
+ * so that a step -- bp_kv_append of the block's K/V, bp_block_attention_paged, bp_spec_accept,
+ * bp_verify_commit -- needs no host round trip and can be captured once in a CUDA graph.  Section
+ * 2.1 / Figure 1: the verify pass appends the rows of all B_s = gamma_s + 1 block positions (the
+ * anchor and the drafts); the rows that stay are the anchor's and the accepted drafts', the
+ * rejected drafts' rows are dropped (the next block overwrites them):
+ *
+ *   ctx_lens[s]   += 1 + n_accepted[s]
+ *   anchor_out[s]  = out_tokens[cu_draft[s] + s + n_accepted[s]]     (the next block's anchor)
+ *   cu_kv_next     = prefix sums of ctx_lens[s] + gamma_s + 1        (the next pass's keys)
+ *
+ *   ctx_lens     [num_seqs] int32 device array, in/out: committed rows per sequence
+ *   n_accepted, out_tokens, cu_draft: as bp_spec_accept writes / reads them
+ *   capacity     rows a sequence's cache can hold (pages_per_seq * page_size)
+ *   anchor_out   [num_seqs] int32 out, may be NULL; cu_kv_next [num_seqs+1] int32 out (may be the
+ *                cu_kv array the next step's append and attention read)
+ *   workspace    at least 256 bytes (the error word)
+ * If some n_accepted is outside [0, gamma_s] or a next pass would exceed capacity, the device error
+ * word is set (BP_ERR_DEVICE_FLAG) and nothing is changed.  One CTA; num_seqs is not limited.
+ * ------------------------------------------------------------------------------- */
+BP_API int bp_verify_commit(int32_t* ctx_lens, const int32_t* n_accepted, const int32_t* out_tokens,
+                            const int32_t* cu_draft, int num_seqs, int capacity, int32_t* anchor_out,
+                            int32_t* cu_kv_next, void* workspace, size_t workspace_bytes, void* stream);
 
 /* Reads and clears the sticky device error word of `workspace` (synchronizes `stream`).
  * Returns BP_OK, BP_ERR_TIMEOUT or BP_ERR_DEVICE_FLAG (or BP_ERR_CUDA if the read fails). */

@@ -24,6 +24,7 @@ from ._binding import (  # noqa: F401
     spec_accept_workspace_size,
     tau_select,
     tau_select_workspace_size,
+    verify_commit,
     verify_epilogue,
     verify_epilogue_workspace_size,
     workspace,

@@ -82,6 +82,8 @@ def load():
     lib.bp_tau_select_workspace_size.restype = sz
     lib.bp_tau_select.argtypes = [vp, i32, i32, vp, i32, i32, f32, vp, vp, vp, vp, vp, vp, sz, vp]
     lib.bp_tau_select.restype = i32
+    lib.bp_verify_commit.argtypes = [vp, vp, vp, vp, i32, i32, vp, vp, vp, sz, vp]
+    lib.bp_verify_commit.restype = i32
     lib.bp_get_status.argtypes = [vp, vp]
     lib.bp_get_status.restype = i32
     _lib = lib
@@ -256,6 +258,27 @@ def verify_epilogue(lm_head, h_target, h_draft, draft_tokens, cu_draft, temperat
                                 ws.numel(), _stream(stream))
     _check(rc, "bp_verify_epilogue")
     return n_accepted, out_tokens, accept_prob
+
+
+# --------------------------------------------------------------------------- decoding-loop commit
+def verify_commit(ctx_lens, n_accepted, out_tokens, cu_draft, capacity: int, anchor=None, cu_kv_next=None, ws=None,
+                  stream=None):
+    """Device-side commit of a verify step; see ``bp_verify_commit``.  ctx_lens is updated in place.
+    Returns (anchor, cu_kv_next)."""
+    lib = load()
+    for t, n in ((ctx_lens, "ctx_lens"), (n_accepted, "n_accepted"), (out_tokens, "out_tokens"),
+                 (cu_draft, "cu_draft"), (anchor, "anchor"), (cu_kv_next, "cu_kv_next")):
+        _cuda(t, n)
+    s = ctx_lens.numel()
+    dev = ctx_lens.device
+    if cu_kv_next is None:
+        cu_kv_next = torch.empty(s + 1, dtype=torch.int32, device=dev)
+    if ws is None:
+        ws = workspace(256, dev)
+    rc = lib.bp_verify_commit(_ptr(ctx_lens), _ptr(n_accepted), _ptr(out_tokens), _ptr(cu_draft), s, int(capacity),
+                              _ptr(anchor), _ptr(cu_kv_next), _ptr(ws), ws.numel(), _stream(stream))
+    _check(rc, "bp_verify_commit")
+    return anchor, cu_kv_next
 
 
 # --------------------------------------------------------------------------- acceptance-length model

@@ -347,6 +347,25 @@ int bp_tau_select(const float* gamma, int num_reqs, int jmax, const int32_t* can
     return rc;
 }
 
+int bp_verify_commit(int32_t* ctx_lens, const int32_t* n_accepted, const int32_t* out_tokens, const int32_t* cu_draft,
+                     int num_seqs, int capacity, int32_t* anchor_out, int32_t* cu_kv_next, void* workspace,
+                     size_t workspace_bytes, void* stream) {
+    if (num_seqs < 0 || capacity < 1) return BP_ERR_INVALID_ARG;
+    if (num_seqs == 0) return BP_OK;
+    if (!ctx_lens || !n_accepted || !out_tokens || !cu_draft || !cu_kv_next) return BP_ERR_INVALID_ARG;
+    int rc = check_workspace(workspace, workspace_bytes, sizeof(WorkspaceHeader));
+    if (rc != BP_OK) return rc;
+    DeviceInfo dev;
+    if ((rc = device_info(&dev)) != BP_OK) return rc;
+    CommitArgs a;
+    a.ctx_lens = ctx_lens; a.n_accepted = n_accepted; a.out_tokens = out_tokens; a.cu_draft = cu_draft;
+    a.num_seqs = num_seqs; a.capacity = capacity; a.anchor_out = anchor_out; a.cu_kv_next = cu_kv_next;
+    a.err_word = err_word(workspace);
+    rc = launch_verify_commit(a, static_cast<cudaStream_t>(stream));
+    if (rc == BP_ERR_CUDA) cudaGetLastError();
+    return rc;
+}
+
 size_t bp_policy_select_workspace_size(int num_reqs, int d_in, int hidden, int num_cand) {
     if (num_reqs < 0 || d_in < 1 || hidden < 1 || num_cand < 1) return 0;
     return sizeof(WorkspaceHeader) + policy_scratch_bytes(num_reqs, d_in, hidden, num_cand);

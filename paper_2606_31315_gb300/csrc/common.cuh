@@ -155,4 +155,16 @@ struct TauArgs {
 size_t tau_scratch_bytes(int num_reqs);
 int launch_tau(const TauArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
+struct CommitArgs {
+    int32_t* ctx_lens;            // [num_seqs] in/out
+    const int32_t* n_accepted;    // [num_seqs]
+    const int32_t* out_tokens;    // [total_draft + num_seqs]
+    const int32_t* cu_draft;      // [num_seqs + 1]
+    int num_seqs, capacity;
+    int32_t* anchor_out;          // [num_seqs] or null
+    int32_t* cu_kv_next;          // [num_seqs + 1]
+    unsigned int* err_word;
+};
+int launch_verify_commit(const CommitArgs& a, cudaStream_t stream);
+
 }  // namespace bp

@@ -155,6 +155,19 @@ def test_tau_select_host_validation_needs_no_gpu(lib):
         assert call(cand=(ctypes.c_int32 * 9)(8, 10, 12, 14, 16, 18, 20, 24, 22)) == 1  # not increasing
 
 
+def test_verify_commit_host_validation_needs_no_gpu(lib):
+    vp = ctypes.c_void_p
+    fake, ws = vp(0x10000), vp(0x20000)
+
+    def call(n=4, cap=4096, ctx=fake, cu_kv=fake, ws_bytes=256):
+        return lib.bp_verify_commit(ctx, fake, fake, fake, n, cap, None, cu_kv, ws, ws_bytes, None)
+    assert call(n=-1) == 1 and call(cap=0) == 1 and call(ctx=None) == 1 and call(cu_kv=None) == 1
+    assert call(ws_bytes=128) == 4
+    assert call(n=0) == 0
+    if not __import__("torch").cuda.is_available():
+        assert call() == 3
+
+
 def test_no_cpu_fallback_without_gpu(lib):
     import torch
 
