@@ -101,11 +101,12 @@ __device__ __forceinline__ void named_arrive(int id, int count) {
 }
 
 // Every CTA of the (co-resident) grid arrives, then waits until `target` arrivals are counted.
-// False in every thread if they were not within the wait budget.
+// False in every thread if they were not within the wait budget.  The CTA barrier orders the block's
+// writes before thread 0's gpu-scope release, and its acquire before the block's later reads (release
+// and acquire are cumulative): no separate fences.
 __device__ bool grid_barrier(unsigned int* count, unsigned int target, int* ok_sh) {
     __syncthreads();
     if (threadIdx.x == 0) {
-        __threadfence();
         red_release_gpu(count, 1u);
         const long long t0 = clock64();
         int ok = 1;
@@ -116,7 +117,6 @@ __device__ bool grid_barrier(unsigned int* count, unsigned int target, int* ok_s
             }
             __nanosleep(64);
         }
-        __threadfence();
         *ok_sh = ok;
     }
     __syncthreads();
