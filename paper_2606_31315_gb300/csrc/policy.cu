@@ -443,26 +443,42 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
             for (int pr = 0; pr < kTcMaxKS; ++pr) sum += v[pr];
             dst[item] = sum;
         }
-        __threadfence();  // this tile's partials before the ticket
+        // the CTA barrier orders every thread's partial before thread 0's release (cumulative); its
+        // acquire makes the other tiles' partials visible to this CTA once it holds the last ticket
         __syncthreads();
         if (tid == 0) last_sh = atomic_add_acq_rel_gpu(p.counters + g, 1) == p.tiles - 1;
         __syncthreads();
         if (last_sh) {
             // every tile has published: logits in tile order, then the argmax per request
             float* logits = hs;  // this CTA's h is no longer needed (ng * C <= npad * rpr floats)
-            for (int item = tid; item < ng * C; item += kTcThreads) {
-                float sum = b2s[item % C];
-                const float* src = p.part + (size_t)g * p.tiles * (kTcMaxN * C) + item;
-                for (int t0 = 0; t0 < p.tiles; t0 += 16) {  // 16 loads in flight, summed in tile order
-                    float v[16];
+            const float* base = p.part + (size_t)g * p.tiles * (kTcMaxN * C);
+            constexpr int kItems = 3;  // items per thread per round: 48 loads in flight
+            for (int i0 = 0; i0 < ng * C; i0 += kItems * kTcThreads) {
+                for (int t0 = 0; t0 < p.tiles; t0 += 16) {
+                    float v[kItems][16];
 #pragma unroll
-                    for (int u = 0; u < 16; ++u) v[u] = t0 + u < p.tiles ? __ldcg(src + (size_t)(t0 + u) * (kTcMaxN * C)) : 0.f;
+                    for (int k = 0; k < kItems; ++k) {
+                        const int item = i0 + tid + k * kTcThreads;
 #pragma unroll
-                    for (int u = 0; u < 16; ++u) sum += v[u];
+                        for (int u = 0; u < 16; ++u)
+                            v[k][u] = item < ng * C && t0 + u < p.tiles
+                                          ? __ldcg(base + (size_t)(t0 + u) * (kTcMaxN * C) + item) : 0.f;
+                    }
+#pragma unroll
+                    for (int k = 0; k < kItems; ++k) {
+                        const int item = i0 + tid + k * kTcThreads;
+                        if (item < ng * C) {
+                            float sum = t0 == 0 ? b2s[item % C] : logits[item];
+#pragma unroll
+                            for (int u = 0; u < 16; ++u) sum += v[k][u];  // tile order
+                            logits[item] = sum;
+                        }
+                    }
                 }
-                logits[item] = sum;
-                if (p.logits_out) p.logits_out[(size_t)n0 * C + item] = sum;
             }
+            if (p.logits_out)  // the same items as above: each thread reads back its own sums
+                for (int item = tid; item < ng * C; item += kTcThreads)
+                    p.logits_out[(size_t)n0 * C + item] = logits[item];
             __syncthreads();
             for (int n = tid; n < ng; n += kTcThreads) {
                 int best = 0;
