@@ -349,9 +349,10 @@ __global__ void __launch_bounds__(kThreads, 2) accept_kernel(const AccParams p) 
             if (xi < 0 || tx == -INFINITY) a = 0.f;
             else if (dx == -INFINITY) a = 1.f;
             else a = fminf(1.f, ex2(__fmaf_rn(tx, c2, -Mt) - __fmaf_rn(dx, c2, -Md)) * (Zd / Zt));
+            // reaches the last ticket holder through the cluster barriers below and the writer's
+            // gpu-scope release at its ticket (both cumulative): no fence of its own
             p.a_ws[d_begin + i] = a;
             if (p.accept_prob) p.accept_prob[d_begin + i] = a;
-            __threadfence();
         }
 
         // ================= pass 2: fixed-point segment sums of r and p, one multiply per entry
