@@ -168,6 +168,10 @@ BP_API int bp_kv_append(void* k_cache, void* v_cache, const void* k_new, const v
  *   accept_prob    [total_draft] fp32 out: a_i for every drafted position; may be NULL
  * Row addresses must be 16-byte aligned for the vectorised path (vocab % 4 == 0 and
  * 16-byte aligned bases); other vocabularies take a scalar path.
+ * Fewer than 48 target rows (total_draft + num_seqs) run as one latency-bound kernel (a
+ * thread-block cluster per row); from 48 rows on, as three throughput kernels (chunk
+ * statistics, decisions, draw).  The rule and the result's bars are the same; the workspace
+ * of the larger problems grows by about 16 bytes per row and 16 KB of vocabulary.
  * ------------------------------------------------------------------------------- */
 BP_API size_t bp_spec_accept_workspace_size(int num_seqs, int total_draft, int vocab);
 BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
@@ -184,9 +188,10 @@ BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits,
  * Same arguments, results and errors as bp_spec_accept, except:
  *   - no workspace: the scratch is a fixed array of BP_NOALLOC_SCRATCH_BYTES inside the
  *     library, held on every GPU that loads the library until the process exits;
- *   - problems whose scratch would exceed it return BP_ERR_WORKSPACE (the requirement is
- *     bp_spec_accept_workspace_size(...) - 256 bytes, about 8 bytes per target row plus 4 per
- *     sequence, so roughly a million target rows fit);
+ *   - the three throughput kernels run only when their scratch fits in the array too; other
+ *     problems of 48 rows or more run on the single kernel;
+ *   - problems whose single-kernel scratch would exceed it return BP_ERR_WORKSPACE (about 8
+ *     bytes per target row plus 4 per sequence, so roughly a million target rows fit);
  *   - device-detected errors are OR-ed into *device_error (a caller-owned device word, may be
  *     NULL to drop them) instead of a workspace: 1 = a wait timed out, 2 = a draft token id
  *     outside [0, vocab);

@@ -618,21 +618,29 @@ int launch_variant(const AccParams& prm0, int rows, const DeviceInfo& dev, cudaS
 
 }  // namespace
 
+// Scratch of the cluster kernel (tickets first: the no-workspace path clears them before each call).
+static size_t cluster_scratch_bytes(int num_seqs, int total_draft) {
+    const size_t rows = (size_t)total_draft + num_seqs;
+    return align_up(sizeof(int) * (size_t)num_seqs, 256) + align_up(sizeof(float) * (size_t)total_draft, 256) +
+           align_up(sizeof(int) * rows, 256);
+}
+
 size_t accept_scratch_bytes(int num_seqs, int total_draft, int vocab) {
     if (vocab < 1 || min_cluster(vocab, false) == 0) return 0;  // slices must fit in shared memory
-    const size_t rows = (size_t)total_draft + num_seqs;
-    size_t b = 0;
-    b += align_up(sizeof(int) * (size_t)num_seqs, 256);    // tickets (first: cleared by the no-workspace path)
-    b += align_up(sizeof(float) * (size_t)total_draft, 256);
-    b += align_up(sizeof(int) * rows, 256);
+    size_t b = cluster_scratch_bytes(num_seqs, total_draft);
+    if (total_draft + num_seqs >= kAcceptBatchRows)  // the throughput kernels' regions follow
+        b += accept_batch_scratch_bytes(num_seqs, total_draft, vocab);
     return b;
 }
 
-int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
+int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream, bool allow_batch) {
     if (accept_scratch_bytes(a.num_seqs, a.total_draft, a.vocab) == 0) return BP_ERR_UNSUPPORTED;
     if (a.num_seqs == 0) return BP_OK;
     const int rows = a.total_draft + a.num_seqs;
     uint8_t* w = static_cast<uint8_t*>(a.scratch);
+    if (allow_batch && rows >= kAcceptBatchRows)  // many rows: the throughput kernels
+        return launch_accept_batch(a, reinterpret_cast<int*>(w),
+                                   w + cluster_scratch_bytes(a.num_seqs, a.total_draft), stream);
     AccParams p;
     p.tickets = reinterpret_cast<int*>(w);
     w += align_up(sizeof(int) * (size_t)a.num_seqs, 256);
@@ -708,7 +716,10 @@ int noalloc_scratch_address(void** out) {
 int launch_accept_noalloc(const AcceptArgs& args, const DeviceInfo& dev, cudaStream_t stream) {
     const size_t need = accept_scratch_bytes(args.num_seqs, args.total_draft, args.vocab);
     if (need == 0) return BP_ERR_UNSUPPORTED;
-    if (need > (size_t)BP_NOALLOC_SCRATCH_BYTES) return BP_ERR_WORKSPACE;  // problem too large for the array
+    // the throughput kernels only when their regions fit too; else the cluster kernel alone
+    const bool allow_batch = need <= (size_t)BP_NOALLOC_SCRATCH_BYTES;
+    if (cluster_scratch_bytes(args.num_seqs, args.total_draft) > (size_t)BP_NOALLOC_SCRATCH_BYTES)
+        return BP_ERR_WORKSPACE;  // problem too large for the array
     void* base = nullptr;
     int rc = noalloc_scratch_address(&base);
     if (rc != BP_OK) return rc;
@@ -719,7 +730,7 @@ int launch_accept_noalloc(const AcceptArgs& args, const DeviceInfo& dev, cudaStr
     }
     AcceptArgs a = args;
     a.scratch = base;
-    return launch_accept(a, dev, stream);
+    return launch_accept(a, dev, stream, allow_batch);
 }
 
 }  // namespace bp

@@ -91,7 +91,12 @@ struct AcceptArgs {
     unsigned int* err_word;
 };
 size_t accept_scratch_bytes(int num_seqs, int total_draft, int vocab);
-int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+// allow_batch = false keeps every call on the cluster kernel (its scratch alone suffices)
+int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream, bool allow_batch = true);
+// From this many target rows on, the acceptance runs as three throughput kernels (accept_batch.cu).
+constexpr int kAcceptBatchRows = 48;
+size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab);
+int launch_accept_batch(const AcceptArgs& a, int* tickets, void* scratch, cudaStream_t stream);
 // Same kernel, scratch taken from the library's own static device array (no workspace).
 int launch_accept_noalloc(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 

@@ -1,5 +1,8 @@
 """GPU parity of bp_spec_accept against the fp64 oracle.
 
+Batches of fewer than 48 target rows run on the cluster kernel, larger ones on the three throughput
+kernels; the edge cases below are taken on both sides of that line (ROWS_SMALL / ROWS_LARGE blocks).
+
 Bars: accept_prob within 1e-5 absolute at every drafted position; n_accepted and the emitted
 tokens bit-exact for every sequence not flagged as a near-tie (|u_i - a_i| < 1e-5 at a tested
 position, or an inverse-CDF threshold within 1e-5 of a cumulative boundary); greedy (T = 0)
@@ -37,9 +40,19 @@ def test_qwen3_4b_full(temp):
     compare_accept(wl.accept_inputs(w, temp), temp)
 
 
-def test_ragged_batch_full():
+BATCH_ROWS = 48  # from this many target rows on, the throughput kernels run
+SMALL_BLOCKS = (16, 1, 3, 9, 8)                   # 37 rows: cluster kernel
+LARGE_BLOCKS = (16, 1, 3, 9, 24, 16, 5, 2, 16)    # 92 rows: throughput kernels
+
+
+def test_block_sets_straddle_the_threshold():
+    assert sum(SMALL_BLOCKS) < BATCH_ROWS <= sum(LARGE_BLOCKS)
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_ragged_batch_full(temp):
     w = wl.get("ragged")
-    flagged, s = compare_accept(wl.accept_inputs(w, 1.0), 1.0)
+    flagged, s = compare_accept(wl.accept_inputs(w, temp), temp)
     # about a quarter of the draws over a 151936-token vocabulary land within 1e-5 of a CDF
     # boundary (most tokens carry less mass than that); those are checked for validity instead
     assert flagged < s // 2
@@ -61,9 +74,11 @@ def test_planted_long_prefixes(temp):
     assert n_acc.max() >= 10
 
 
-@pytest.mark.parametrize("vocab", [5, 1001, 4099, 32000])
-def test_vocab_sizes_and_scalar_path(vocab):
-    w = wl.custom(seed=vocab, ctx=(0,) * 6, block=(16, 1, 3, 9, 24, 16), vocab=vocab)
+@pytest.mark.parametrize("blocks", [SMALL_BLOCKS, LARGE_BLOCKS])
+@pytest.mark.parametrize("vocab", [5, 1001, 4099, 16384, 32000, 50001])
+def test_vocab_sizes_and_scalar_path(vocab, blocks):
+    """Vocabularies below one chunk, exactly one, and ragged last chunks; odd sizes take the scalar loads."""
+    w = wl.custom(seed=vocab, ctx=(0,) * len(blocks), block=blocks, vocab=vocab)
     for temp in (1.0, 0.0):
         compare_accept(wl.accept_inputs(w, temp), temp)
 
@@ -122,8 +137,9 @@ def test_lossless_chi_square_on_gpu():
                    ref=run_oracle_accept(small, 1.0))
 
 
-def test_out_of_range_draft_token_sets_device_flag():
-    w = wl.custom(seed=3, ctx=(0, 0), block=(4, 4), vocab=1000)
+@pytest.mark.parametrize("blocks", [(4, 4), LARGE_BLOCKS])
+def test_out_of_range_draft_token_sets_device_flag(blocks):
+    w = wl.custom(seed=3, ctx=(0,) * len(blocks), block=blocks, vocab=1000)
     inp = wl.accept_inputs(w, 1.0)
     inp["draft_tokens"][2] = 1000  # caught by the kernel's own bounds check, never dereferenced
     status = run_accept(inp, 1.0)[3]
@@ -139,11 +155,12 @@ def test_host_side_validation():
     assert e.value.status == 1  # T > 0 needs draft logits
 
 
+@pytest.mark.parametrize("blocks", [(16, 9, 1, 5), (16, 9, 1, 5) * 3])
 @pytest.mark.parametrize("temp", [1.0, 0.0])
-def test_masked_vocabulary(temp):
+def test_masked_vocabulary(temp, blocks):
     """Logits of -inf (a masked vocabulary: the first 40% and a band in the middle) in every row:
     whole chunks of some lanes hold no finite entry, and the masked tokens must never be drawn."""
-    w = wl.custom(seed=45, ctx=(0,) * 4, block=(16, 9, 1, 5), vocab=151936)
+    w = wl.custom(seed=45, ctx=(0,) * len(blocks), block=blocks, vocab=151936)
     inp = wl.accept_inputs(w, temp)
     v = inp["target_logits"].shape[1]
     masked = np.zeros(v, dtype=bool)
@@ -162,3 +179,30 @@ def test_masked_vocabulary(temp):
     _, out, _, _ = run_accept(inp, temp)
     emitted = out[out >= 0]
     assert not masked[emitted].any()
+
+
+@pytest.mark.parametrize("blocks", [SMALL_BLOCKS, LARGE_BLOCKS])
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_fully_masked_rows(temp, blocks):
+    """Some drafter rows and some target rows with every entry -inf.  Greedy: the argmax of a masked
+    target row is index 0.  T > 0: a masked drafter row has q = 0, so its token is accepted when p > 0
+    and the residual is p itself; no NaN reaches a decision."""
+    w = wl.custom(seed=46, ctx=(0,) * len(blocks), block=blocks, vocab=3000)
+    inp = wl.accept_inputs(w, temp)
+    inp["target_logits"] = inp["target_logits"].copy()
+    inp["draft_logits"] = inp["draft_logits"].copy()
+    cu = inp["cu_draft"]
+    # per sequence with drafts: mask the drafter's first row; every third sequence (the one-row block
+    # among them) also masks its target bonus row (greedy only: at T > 0 a masked target row has no
+    # distribution to draw from)
+    for s in range(len(blocks)):
+        if cu[s + 1] > cu[s]:
+            inp["draft_logits"][cu[s]] = -np.inf
+        if temp == 0.0 and s % 3 == 1:
+            inp["target_logits"][cu[s + 1] + s] = -np.inf
+    compare_accept(inp, temp)
+    n_acc, out, ap, status = run_accept(inp, temp)
+    assert status == 0
+    assert np.all(np.isfinite(ap))
+    if temp == 0.0:
+        assert out[cu[2] + 1] == 0  # sequence 1: one row, masked

@@ -18,6 +18,8 @@ import torch
 import paper_2606_31315_gb300 as bp
 from paper_2606_31315_gb300 import workloads as wl
 
+from _gpu import compare_accept, run_oracle_accept
+
 pytestmark = pytest.mark.gpu
 
 PROB_TOL = 1e-5
@@ -102,3 +104,25 @@ def test_too_large_problem_is_refused(lib):
                                     _p(out), None, None, stream)
     torch.cuda.synchronize()
     assert rc == 4  # BP_ERR_WORKSPACE
+
+
+def test_large_batch_falls_back_to_the_single_kernel(lib):
+    # 200000 sequences of one draft each over a 16-token vocabulary: 400000 target rows.  The
+    # single kernel's scratch (tickets, ratios, row tokens: about 3.2 MB) fits in the fixed array;
+    # the throughput kernels' regions on top of it (chunk and row statistics of 600000 rows,
+    # per-sequence draw masses: about 14 MB more) do not, so the call runs the single kernel.
+    # Checked against the oracle on the first 20000 sequences.
+    s, v = 200_000, 16
+    rng = np.random.default_rng(81)
+    tl = rng.normal(0.0, 2.0, size=(2 * s, v)).astype(np.float32)
+    dl = rng.normal(0.0, 2.0, size=(s, v)).astype(np.float32)
+    inp = dict(target_logits=tl, draft_logits=dl, draft_tokens=rng.integers(0, v, size=s).astype(np.int32),
+               cu_draft=np.arange(s + 1, dtype=np.int32), u_accept=rng.random(s, dtype=np.float32),
+               u_sample=rng.random(s, dtype=np.float32))
+    assert bp.spec_accept_workspace_size(s, s, v) > (8 << 20)  # the throughput kernels' layout is larger
+    g = {k: torch.from_numpy(np.ascontiguousarray(x)).cuda() for k, x in inp.items()}
+    n_acc, out, ap = _noalloc(lib, g, 1.0)
+    m = 20_000
+    small = {k: x[: 2 * m] if k == "target_logits" else x[: m + 1] if k == "cu_draft" else x[:m]
+             for k, x in inp.items()}
+    compare_accept(small, 1.0, gpu=(n_acc[:m], out[: 2 * m], ap[:m], 0), ref=run_oracle_accept(small, 1.0))
