@@ -442,6 +442,44 @@ def run_ours(args):
                       + reg_tau.numel() * 4)
     del g_tau, tau_out
 
+    # a5-a7 at batch scale: the 32-request ragged batch (blocks 2..32: 502 target and 470 drafter rows
+    # over the 151936-token vocabulary), which runs the three throughput kernels.  Same recipe as the
+    # other rows (target ~ N(0, logit_std^2), draft = target + N(0, 1), tokens by Gumbel-max at T = 1,
+    # argmax at T = 0), drawn on the device; 4 rotating copies (2.4 GB) > L2
+    rw = wl.get("ragged")
+    r_g = np.asarray(rw.block) - 1
+    r_cu = t(wl.offsets(r_g))
+    r_s, r_td = rw.num_seqs, int(r_g.sum())
+    r_trow = t((np.arange(r_td) + np.repeat(np.arange(r_s), r_g)).astype(np.int64))
+    r_copies = []
+    for _ in range(4):
+        tg = torch.randn(r_td + r_s, rw.vocab, device=dev, generator=gen) * rw.logit_std
+        dr = tg[r_trow] + torch.randn(r_td, rw.vocab, device=dev, generator=gen)
+        e = torch.empty_like(dr).exponential_(generator=gen)  # -log(E), E ~ Exp(1), is Gumbel noise
+        r_copies.append(dict(target=tg, draft=dr, tok1=torch.argmax(dr - torch.log(e), dim=1).to(torch.int32),
+                             tok0=torch.argmax(dr, dim=1).to(torch.int32),
+                             ua=torch.rand(r_td, device=dev, generator=gen),
+                             us=torch.rand(r_s, device=dev, generator=gen)))
+        del e
+    r_n = torch.empty(r_s, dtype=torch.int32, device=dev)
+    r_o = torch.empty(r_td + r_s, dtype=torch.int32, device=dev)
+    ws_r = bp.workspace(bp.spec_accept_workspace_size(r_s, r_td, rw.vocab), dev)
+
+    def batch_accept(temperature):
+        turn = [0]
+
+        def go(_c):
+            c = r_copies[turn[0] % len(r_copies)]
+            turn[0] += 1
+            bp.spec_accept(c["target"], c["draft"] if temperature > 0 else None, c["tok1"] if temperature > 0 else
+                           c["tok0"], r_cu, temperature, c["ua"], c["us"], n_accepted=r_n, out_tokens=r_o,
+                           want_accept_prob=False, ws=ws_r, stream=stream)
+        return go
+
+    t_racc1 = time_calls(batch_accept(1.0), n_graph=4, reps=10)
+    t_racc0 = time_calls(batch_accept(0.0), n_graph=4, reps=10)
+    del r_copies
+
     def row(tsec, nbytes, kernels):
         gbs = nbytes / tsec / 1e9
         return {"us": round(tsec * 1e6, 3), "bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
@@ -466,6 +504,12 @@ def run_ours(args):
                                      "verify_commit_kernel"]),
             per_step="36 x (append + paged verify attention, 64-row pages) + T=1 acceptance + commit; the "
                      "context grows from 2048 by the accepted prefix each step; bytes counted at 2048 + 16 keys"),
+        "a5_a6_accept_t1_batch_ragged_32req": dict(
+            row(t_racc1, accept_bytes(rw, 1.0), ["batch_stats_kernel<false,true>", "batch_decide_kernel<false>",
+                                                 "batch_draw_kernel<true,2>"]),
+            traffic=committed_traffic("batch_stats_kernel")),
+        "a7_accept_greedy_t0_batch_ragged_32req": row(t_racc0, accept_bytes(rw, 0.0),
+                                                      ["batch_stats_kernel<true,true>", "batch_decide_kernel<true>"]),
         "next4_tau_model_4M_requests": dict(row(t_tau, tau_bytes, ["tau_kernel<24,9>", "tau_finish_kernel"]),
                                             traffic=committed_traffic("tau_kernel")),
     }

@@ -168,10 +168,11 @@ BP_API int bp_kv_append(void* k_cache, void* v_cache, const void* k_new, const v
  *   accept_prob    [total_draft] fp32 out: a_i for every drafted position; may be NULL
  * Row addresses must be 16-byte aligned for the vectorised path (vocab % 4 == 0 and
  * 16-byte aligned bases); other vocabularies take a scalar path.
- * Fewer than 48 target rows (total_draft + num_seqs) run as one latency-bound kernel (a
- * thread-block cluster per row); from 48 rows on, as three throughput kernels (chunk
- * statistics, decisions, draw).  The rule and the result's bars are the same; the workspace
- * of the larger problems grows by about 16 bytes per row and 16 KB of vocabulary.
+ * Small problems run as one latency-bound kernel (a thread-block cluster per row); from 2.5M
+ * logits read at T = 0 ((total_draft + num_seqs) x vocab) and 6.5M at T > 0 ((2 total_draft +
+ * num_seqs) x vocab) on, as three throughput kernels (chunk statistics, decisions, draw).  The
+ * rule and the result's bars are the same; the workspace of the larger problems grows by about
+ * 16 bytes per row and 16K vocabulary entries, plus 4 KB per sequence and 16K entries.
  * ------------------------------------------------------------------------------- */
 BP_API size_t bp_spec_accept_workspace_size(int num_seqs, int total_draft, int vocab);
 BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits, const int32_t* draft_tokens,
@@ -189,7 +190,7 @@ BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits,
  *   - no workspace: the scratch is a fixed array of BP_NOALLOC_SCRATCH_BYTES inside the
  *     library, held on every GPU that loads the library until the process exits;
  *   - the three throughput kernels run only when their scratch fits in the array too; other
- *     problems of 48 rows or more run on the single kernel;
+ *     problems large enough for them run on the single kernel;
  *   - problems whose single-kernel scratch would exceed it return BP_ERR_WORKSPACE (about 8
  *     bytes per target row plus 4 per sequence, so roughly a million target rows fit);
  *   - device-detected errors are OR-ed into *device_error (a caller-owned device word, may be

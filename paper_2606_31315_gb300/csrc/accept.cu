@@ -628,7 +628,7 @@ static size_t cluster_scratch_bytes(int num_seqs, int total_draft) {
 size_t accept_scratch_bytes(int num_seqs, int total_draft, int vocab) {
     if (vocab < 1 || min_cluster(vocab, false) == 0) return 0;  // slices must fit in shared memory
     size_t b = cluster_scratch_bytes(num_seqs, total_draft);
-    if (total_draft + num_seqs >= kAcceptBatchRows)  // the throughput kernels' regions follow
+    if (accept_may_batch(num_seqs, total_draft, vocab))  // the throughput kernels' regions follow
         b += accept_batch_scratch_bytes(num_seqs, total_draft, vocab);
     return b;
 }
@@ -638,8 +638,8 @@ int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t strea
     if (a.num_seqs == 0) return BP_OK;
     const int rows = a.total_draft + a.num_seqs;
     uint8_t* w = static_cast<uint8_t*>(a.scratch);
-    if (allow_batch && rows >= kAcceptBatchRows)  // many rows: the throughput kernels
-        return launch_accept_batch(a, reinterpret_cast<int*>(w),
+    if (allow_batch && accept_use_batch(a.num_seqs, a.total_draft, a.vocab, a.temperature == 0.f))
+        return launch_accept_batch(a, dev.sm_count, reinterpret_cast<int*>(w),
                                    w + cluster_scratch_bytes(a.num_seqs, a.total_draft), stream);
     AccParams p;
     p.tickets = reinterpret_cast<int*>(w);

@@ -10,13 +10,16 @@
 //      (coalesced 16-byte loads) and writes the chunk's (scaled max, sum of 2^(l*log2e/T - max)) --
 //      at T = 0 its (max, lowest index) -- so the whole batch is one HBM-bound pass;
 //   2. decide: one warp per sequence merges its rows' chunk statistics in a fixed order, forms the
-//      ratios a_i, the first rejection k and the outputs (at T = 0 the emitted argmax too);
+//      ratios a_i, the first rejection k and the outputs (at T = 0 the emitted argmax too).  (Taking
+//      the decisions in the statistics kernel, in the CTA that completes a sequence, costs every CTA a
+//      gpu-scope ticket behind its store: measured slower for large batches);
 //   3. draw (T > 0): one CTA per chunk of each sequence's draw row pair (the rejected row, or the bonus
-//      row) forms the chunk's mass of max(0, p_k - q_k) and of p_k in exact 2^-52 fixed point; the
-//      last CTA of the sequence (ticket) finds the chunk, the 128-entry segment and the entry where the
-//      inverse CDF crosses u_s * total, re-reading that one chunk, and writes the emitted token.
-// Only the one draw row pair per sequence is read twice.  The three kernels chain with programmatic
-// dependent launch.
+//      row) forms the chunk's segment masses of max(0, p_k - q_k) and of p_k in exact 2^-52 fixed
+//      point; the last CTA of the sequence (ticket) finds the chunk and the 128-entry segment where the
+//      inverse CDF crosses u_s * total from the stored masses, then the entry from that segment's 128
+//      logits, and writes the emitted token.
+// Only the one draw row pair per sequence is read twice.  The kernels chain with programmatic dependent
+// launch.
 #include <cuda_runtime.h>
 #include <math.h>
 
@@ -48,6 +51,7 @@ struct BatchParams {
     float2* rowstat;   // [rows] row statistics
     int* k_ws;         // [num_seqs] first rejection
     ulonglong2* ctot;  // [num_seqs][chunks] draw masses of r and p (fixed point)
+    unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses (chunks > 1)
     int* tickets;      // [num_seqs], zero between calls
     unsigned int* err;
 };
@@ -67,20 +71,104 @@ __device__ __forceinline__ const float* row_ptr(const BatchParams& p, int r) {
 // groups for one j are 128 consecutive entries (segment (j, warp)) and segments in (j, warp) order
 // are in entry order.
 template <bool VEC>
+__device__ __forceinline__ float4 load4(const float* __restrict__ src, int e, int n) {
+    if (VEC)
+        return e < n ? __ldcs(reinterpret_cast<const float4*>(src + e))
+                     : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
+    return make_float4(e < n ? __ldcs(src + e) : -INFINITY, e + 1 < n ? __ldcs(src + e + 1) : -INFINITY,
+                       e + 2 < n ? __ldcs(src + e + 2) : -INFINITY, e + 3 < n ? __ldcs(src + e + 3) : -INFINITY);
+}
+template <bool VEC>
 __device__ __forceinline__ void load_chunk(const float* __restrict__ src, int n, int tid,
                                            float4 (&v)[kBVec]) {
 #pragma unroll
-    for (int j = 0; j < kBVec; ++j) {
-        const int e = 4 * (tid + j * kBThreads);
-        if (VEC) {
-            v[j] = e < n ? __ldcs(reinterpret_cast<const float4*>(src + e))
-                         : make_float4(-INFINITY, -INFINITY, -INFINITY, -INFINITY);
-        } else {
-            v[j].x = e < n ? __ldcs(src + e) : -INFINITY;
-            v[j].y = e + 1 < n ? __ldcs(src + e + 1) : -INFINITY;
-            v[j].z = e + 2 < n ? __ldcs(src + e + 2) : -INFINITY;
-            v[j].w = e + 3 < n ? __ldcs(src + e + 3) : -INFINITY;
+    for (int j = 0; j < kBVec; ++j) v[j] = load4<VEC>(src, 4 * (tid + j * kBThreads), n);
+}
+
+// Decisions of sequence s, by one warp: its rows' statistics from their chunks', the ratios a_i, the
+// first rejection k and the outputs (at T = 0 the emitted argmax too).
+template <bool GREEDY>
+__device__ __forceinline__ void decide_seq(const BatchParams& p, int s, int lane) {
+    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
+    const int nrows = GREEDY ? g + 1 : 2 * g + 1;  // the target rows, then (T > 0) the drafter's
+    // each lane merges whole rows (two at a time), chunks in order, eight chunks' loads in flight
+    constexpr int RH = 2, CQ = 8;
+    const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
+    for (int rr0 = lane; rr0 < nrows; rr0 += 32 * RH) {
+        int r[RH];
+        float2 acc[RH];
+#pragma unroll
+        for (int h = 0; h < RH; ++h) {
+            const int rr = rr0 + 32 * h;
+            r[h] = rr >= nrows ? -1 : rr <= g ? t0 + rr : p.rows_t + d0 + (rr - g - 1);
+            acc[h] = ident;
         }
+        for (int c0 = 0; c0 < p.chunks; c0 += CQ) {
+            float2 x[RH][CQ];
+#pragma unroll
+            for (int h = 0; h < RH; ++h)
+#pragma unroll
+                for (int q = 0; q < CQ; ++q)
+                    x[h][q] = r[h] >= 0 && c0 + q < p.chunks ? __ldcg(&p.part[(size_t)r[h] * p.chunks + c0 + q])
+                                                             : ident;
+#pragma unroll
+            for (int h = 0; h < RH; ++h)
+#pragma unroll
+                for (int q = 0; q < CQ; ++q) {
+                    if (GREEDY) {
+                        int ai = __float_as_int(acc[h].y);
+                        amax_merge(acc[h].x, ai, x[h][q].x, __float_as_int(x[h][q].y));
+                        acc[h].y = __int_as_float(ai);
+                    } else {
+                        lse_merge(acc[h].x, acc[h].y, x[h][q].x, x[h][q].y);
+                    }
+                }
+        }
+#pragma unroll
+        for (int h = 0; h < RH; ++h) {
+            if (r[h] < 0) continue;
+            float2 a = acc[h];
+            if (GREEDY && __float_as_int(a.y) >= p.vocab) a.y = __int_as_float(0);  // every entry -inf: index 0
+            p.rowstat[r[h]] = a;
+        }
+    }
+    __syncwarp();  // the warp's row statistics are written (and visible to its lanes)
+    int k = g;
+    for (int i0 = 0; i0 < g; i0 += 32) {
+        const int i = i0 + lane;
+        bool rej = false;
+        if (i < g) {
+            const int x = p.tokens[d0 + i];
+            const bool valid = x >= 0 && x < p.vocab;
+            if (!valid) raise_error(p.err, kErrDeviceArg);
+            const float2 st = p.rowstat[t0 + i];
+            float a;
+            if (GREEDY) {
+                a = valid && x == __float_as_int(st.y) ? 1.f : 0.f;
+                rej = a == 0.f;
+            } else {
+                const float tx = valid ? p.target[(size_t)(t0 + i) * p.vocab + x] : -INFINITY;
+                const float dx = valid ? p.draft[(size_t)(d0 + i) * p.vocab + x] : -INFINITY;
+                const float2 sd = p.rowstat[p.rows_t + d0 + i];
+                // a = min(1, p(x)/q(x)) in the log domain (q(x) = 0 < p(x) gives 1, p(x) = 0 gives 0)
+                if (!valid || tx == -INFINITY) a = 0.f;
+                else if (dx == -INFINITY) a = 1.f;
+                else a = fminf(1.f, ex2(__fmaf_rn(tx, p.c2, -st.x) - __fmaf_rn(dx, p.c2, -sd.x)) * (sd.y / st.y));
+                rej = !(p.u_accept[d0 + i] < a);
+            }
+            if (p.accept_prob) p.accept_prob[d0 + i] = a;
+        }
+        const unsigned b = __ballot_sync(0xffffffffu, rej);
+        if (b && k == g) k = i0 + __ffs(b) - 1;
+    }
+    for (int j = lane; j <= g; j += 32) {
+        if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
+        else if (j > k) p.out_tokens[t0 + j] = -1;
+        else if (GREEDY) p.out_tokens[t0 + j] = __float_as_int(p.rowstat[t0 + k].y);
+    }
+    if (lane == 0) {
+        p.n_accepted[s] = k;
+        if (!GREEDY) p.k_ws[s] = k;
     }
 }
 
@@ -149,71 +237,13 @@ __global__ void __launch_bounds__(kBThreads) batch_stats_kernel(const BatchParam
     }
 }
 
-// ---- 2. row statistics, ratios, first rejection and outputs: one warp per sequence
+// ---- 2. decisions: one warp per sequence
 template <bool GREEDY>
 __global__ void __launch_bounds__(kBThreads) batch_decide_kernel(const BatchParams p) {
     griddep_launch_dependents();
     griddep_wait();
-    const int lane = threadIdx.x & 31;
     const int s = blockIdx.x * (kBThreads / 32) + (threadIdx.x >> 5);
-    if (s >= p.num_seqs) return;
-    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
-    const int nrows = GREEDY ? g + 1 : 2 * g + 1;  // the target rows, then (T > 0) the drafter's
-    for (int rr = lane; rr < nrows; rr += 32) {  // each lane merges whole rows, chunks in order
-        const int r = rr <= g ? t0 + rr : p.rows_t + d0 + (rr - g - 1);
-        const float2* pr = p.part + (size_t)r * p.chunks;
-        float a0 = -INFINITY, a1 = GREEDY ? __int_as_float(INT_MAX) : 0.f;
-        for (int c = 0; c < p.chunks; ++c) {
-            const float2 x = pr[c];
-            if (GREEDY) {
-                int ai = __float_as_int(a1);
-                amax_merge(a0, ai, x.x, __float_as_int(x.y));
-                a1 = __int_as_float(ai);
-            } else {
-                lse_merge(a0, a1, x.x, x.y);
-            }
-        }
-        if (GREEDY && __float_as_int(a1) >= p.vocab) a1 = __int_as_float(0);  // every entry -inf: index 0
-        p.rowstat[r] = make_float2(a0, a1);
-    }
-    __syncwarp();  // the warp's row statistics are written (and visible to its lanes)
-    int k = g;
-    for (int i0 = 0; i0 < g; i0 += 32) {
-        const int i = i0 + lane;
-        bool rej = false;
-        if (i < g) {
-            const int x = p.tokens[d0 + i];
-            const bool valid = x >= 0 && x < p.vocab;
-            if (!valid) raise_error(p.err, kErrDeviceArg);
-            const float2 st = p.rowstat[t0 + i];
-            float a;
-            if (GREEDY) {
-                a = valid && x == __float_as_int(st.y) ? 1.f : 0.f;
-                rej = a == 0.f;
-            } else {
-                const float tx = valid ? p.target[(size_t)(t0 + i) * p.vocab + x] : -INFINITY;
-                const float dx = valid ? p.draft[(size_t)(d0 + i) * p.vocab + x] : -INFINITY;
-                const float2 sd = p.rowstat[p.rows_t + d0 + i];
-                // a = min(1, p(x)/q(x)) in the log domain (q(x) = 0 < p(x) gives 1, p(x) = 0 gives 0)
-                if (!valid || tx == -INFINITY) a = 0.f;
-                else if (dx == -INFINITY) a = 1.f;
-                else a = fminf(1.f, ex2(__fmaf_rn(tx, p.c2, -st.x) - __fmaf_rn(dx, p.c2, -sd.x)) * (sd.y / st.y));
-                rej = !(p.u_accept[d0 + i] < a);
-            }
-            if (p.accept_prob) p.accept_prob[d0 + i] = a;
-        }
-        const unsigned b = __ballot_sync(0xffffffffu, rej);
-        if (b && k == g) k = i0 + __ffs(b) - 1;
-    }
-    for (int j = lane; j <= g; j += 32) {
-        if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
-        else if (j > k) p.out_tokens[t0 + j] = -1;
-        else if (GREEDY) p.out_tokens[t0 + j] = __float_as_int(p.rowstat[t0 + k].y);
-    }
-    if (lane == 0) {
-        p.n_accepted[s] = k;
-        if (!GREEDY) p.k_ws[s] = k;
-    }
+    if (s < p.num_seqs) decide_seq<GREEDY>(p, s, threadIdx.x & 31);
 }
 
 // The draw row pair of a sequence and the constants of its weights.
@@ -221,10 +251,14 @@ struct DrawPair {
     int trow, drow;  // drow < 0: a bonus draw from p alone
     float Mt, izt, Md, izd;
 };
-__device__ __forceinline__ DrawPair draw_pair(const BatchParams& p, int s, int t0, int d0, int g, int k) {
+__device__ __forceinline__ DrawPair draw_rows(const BatchParams& p, int t0, int d0, int g, int k) {
     DrawPair d;
     d.trow = t0 + k;
     d.drow = k < g ? p.rows_t + d0 + k : -1;
+    return d;
+}
+// The weights' constants from the rows' statistics (read after the rows' loads are issued).
+__device__ __forceinline__ void draw_consts(const BatchParams& p, DrawPair& d) {
     // a row whose entries are all -inf weighs every entry 0 (M = 0, 1/Z = 0 keep it free of NaN)
     const float2 st = p.rowstat[d.trow];
     const bool tz = st.x == -INFINITY;
@@ -234,7 +268,6 @@ __device__ __forceinline__ DrawPair draw_pair(const BatchParams& p, int s, int t
     const bool dz = sd.x == -INFINITY;
     d.Md = dz ? 0.f : sd.x;
     d.izd = dz ? 0.f : __fdiv_rn(1.f, sd.y);
-    return d;
 }
 // Weights of four entries: (r = max(0, p - q), p) with p = 2^(l*c2 - Mt) / Zt (r = 0 without a draft row).
 __device__ __forceinline__ void weights4(float4 lt, float4 ld, const DrawPair& d, float c2, float4& r, float4& pw) {
@@ -250,32 +283,49 @@ __device__ __forceinline__ void weights4(float4 lt, float4 ld, const DrawPair& d
 }
 __device__ __forceinline__ float sum4f(float4 v) { return (v.x + v.y) + (v.z + v.w); }
 
-// Masses of the 128-entry segments (j, warp) of one chunk of the draw pair, 2^-52 fixed point.
-template <bool VEC>
-__device__ __forceinline__ void chunk_masses(const BatchParams& p, const DrawPair& d, int chunk, int tid,
-                                             unsigned long long (*segR)[kBSegs],
-                                             unsigned long long (*segP)[kBSegs]) {
+// Masses of the 128-entry segments (j, warp) of one chunk of the draw pair, 2^-52 fixed point, into
+// segR / segP; returns the calling thread's one: segment (lane, warp)'s r mass for lanes below 16,
+// segment (lane - 16, warp)'s p mass above.  The chunk's 16-byte groups are loaded in PH phases: one
+// keeps every load in flight (for grids of at most one CTA per SM), two fit 128 registers, i.e. two
+// CTAs per SM (for larger grids).
+template <bool VEC, int PH>
+__device__ __forceinline__ unsigned long long chunk_masses(const BatchParams& p, DrawPair& d, int chunk, int tid,
+                                                           unsigned long long (*segR)[kBSegs],
+                                                           unsigned long long (*segP)[kBSegs]) {
     const int lane = tid & 31, warp = tid >> 5;
     const int v0 = chunk * kBChunk, n = min(kBChunk, p.vocab - v0);
-    float4 lt[kBVec], ld[kBVec];
-    load_chunk<VEC>(row_ptr(p, d.trow) + v0, n, tid, lt);
-    if (d.drow >= 0) load_chunk<VEC>(row_ptr(p, d.drow) + v0, n, tid, ld);
+    const float* tp = row_ptr(p, d.trow) + v0;
+    const float* dp = d.drow >= 0 ? row_ptr(p, d.drow) + v0 : tp;
+    constexpr int JP = kBVec / PH;
     float v[32];  // the lane's r sums of segments j = 0..15, then its p sums
 #pragma unroll
-    for (int j = 0; j < kBVec; ++j) {
-        float4 r, pw;
-        weights4(lt[j], d.drow >= 0 ? ld[j] : lt[j], d, p.c2, r, pw);
-        v[j] = sum4f(r);
-        v[kBVec + j] = sum4f(pw);
+    for (int h = 0; h < PH; ++h) {
+        float4 lt[JP], ld[JP];
+#pragma unroll
+        for (int jj = 0; jj < JP; ++jj) {
+            const int e = 4 * (tid + (h * JP + jj) * kBThreads);
+            lt[jj] = load4<VEC>(tp, e, n);
+            if (d.drow >= 0) ld[jj] = load4<VEC>(dp, e, n);
+        }
+        if (h == 0) draw_consts(p, d);
+#pragma unroll
+        for (int jj = 0; jj < JP; ++jj) {
+            const int j = h * JP + jj;
+            float4 r, pw;
+            weights4(lt[jj], d.drow >= 0 ? ld[jj] : lt[jj], d, p.c2, r, pw);
+            v[j] = sum4f(r);
+            v[kBVec + j] = sum4f(pw);
+        }
     }
     const unsigned long long f = to_fix(reduce_scatter32(v, lane));  // lane j: segment j's r; 16 + j: its p
     if (lane < kBSegs) segR[warp][lane] = f;
     else segP[warp][lane - kBSegs] = f;
+    return f;
 }
 
 // ---- 3. the draw (T > 0): chunk masses, then the last chunk of the sequence finds the entry
-template <bool VEC>
-__global__ void __launch_bounds__(kBThreads) batch_draw_kernel(const BatchParams p) {
+template <bool VEC, int PH>
+__global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchParams p) {
     __shared__ unsigned long long segR[kBThreads / 32][kBSegs], segP[kBThreads / 32][kBSegs];
     __shared__ int last_sh, cstar_sh, jstar_sh, wstar_sh, use_r_sh;
     __shared__ unsigned long long off_sh, base_sh;
@@ -285,19 +335,33 @@ __global__ void __launch_bounds__(kBThreads) batch_draw_kernel(const BatchParams
     const int s = blockIdx.x / p.chunks, chunk = blockIdx.x - s * p.chunks;
     const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
     const int k = p.k_ws[s];
-    const DrawPair d = draw_pair(p, s, t0, d0, g, k);
-    chunk_masses<VEC>(p, d, chunk, tid, segR, segP);
+    DrawPair d = draw_rows(p, t0, d0, g, k);  // its constants are filled in by chunk_masses
+    constexpr int kSeg = kBThreads / 32 * kBSegs;  // 128 segments per chunk
+    static_assert(kBSegs == 16 && 2 * kSeg == kBThreads, "one segment mass per thread");
+    const unsigned long long f = chunk_masses<VEC, PH>(p, d, chunk, tid, segR, segP);
+    if (p.chunks > 1) {  // the segment masses, for the last CTA should the crossing fall in this chunk
+        unsigned long long* segm = p.segm + ((size_t)s * p.chunks + chunk) * 2 * kSeg;
+        segm[(lane < kBSegs ? 0 : kSeg) + warp * kBSegs + (lane & (kBSegs - 1))] = f;  // segR / segP layout
+    }
     __syncthreads();
-    if (tid == 0) {
+    if (warp == 0) {
         unsigned long long R = 0, P = 0;
-        for (int w = 0; w < kBThreads / 32; ++w)
-            for (int j = 0; j < kBSegs; ++j) {
-                R += segR[w][j];
-                P += segP[w][j];
-            }
-        p.ctot[(size_t)s * p.chunks + chunk] = make_ulonglong2(R, P);
-        // release: this chunk's masses before the ticket; acquire: the last sees every chunk's
-        last_sh = ticket_acq_rel(p.tickets + s) == p.chunks - 1;
+#pragma unroll
+        for (int e = 0; e < kSeg / 32; ++e) {
+            R += (&segR[0][0])[lane + 32 * e];
+            P += (&segP[0][0])[lane + 32 * e];
+        }
+#pragma unroll
+        for (int o = 16; o >= 1; o >>= 1) {
+            R += __shfl_xor_sync(0xffffffffu, R, o);
+            P += __shfl_xor_sync(0xffffffffu, P, o);
+        }
+        if (lane == 0) {
+            p.ctot[(size_t)s * p.chunks + chunk] = make_ulonglong2(R, P);
+            // release (cumulative through the barrier): this chunk's total and every thread's segment
+            // mass before the ticket; acquire: the last CTA sees every chunk's
+            last_sh = ticket_acq_rel(p.tickets + s) == p.chunks - 1;
+        }
     }
     __syncthreads();
     if (!last_sh) return;
@@ -354,9 +418,12 @@ __global__ void __launch_bounds__(kBThreads) batch_draw_kernel(const BatchParams
     __syncthreads();
     const int cstar = cstar_sh;
     if (cstar >= 0) {
-        // ---- the crossing chunk's segment masses again (the same arithmetic), then the segment
+        // ---- the crossing chunk's segment masses (stored by its CTA), then the segment
         if (cstar != chunk) {
-            chunk_masses<VEC>(p, d, cstar, tid, segR, segP);
+            const unsigned long long* sm = p.segm + ((size_t)s * p.chunks + cstar) * 2 * kSeg;
+            const unsigned long long x = __ldcg(sm + tid);
+            if (tid < kSeg) (&segR[0][0])[tid] = x;
+            else (&segP[0][0])[tid - kSeg] = x;
             __syncthreads();
         }
         const bool use_r = use_r_sh != 0;
@@ -439,9 +506,10 @@ __global__ void __launch_bounds__(kBThreads) batch_draw_kernel(const BatchParams
 size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
     const size_t chunks = ((size_t)vocab + kBChunk - 1) / kBChunk;
     const size_t rows = 2 * (size_t)total_draft + num_seqs;
+    const size_t segm = chunks > 1 ? (size_t)num_seqs * chunks * 2 * 128 * sizeof(unsigned long long) : 0;
     return align_up(rows * chunks * sizeof(float2), 256) + align_up(rows * sizeof(float2), 256) +
            align_up((size_t)num_seqs * sizeof(int), 256) +
-           align_up((size_t)num_seqs * chunks * sizeof(ulonglong2), 256);
+           align_up((size_t)num_seqs * chunks * sizeof(ulonglong2), 256) + align_up(segm, 256);
 }
 
 namespace {
@@ -461,18 +529,20 @@ int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_
 }
 
 template <bool GREEDY, bool VEC>
-int run_batch(const BatchParams& p, cudaStream_t stream) {
+int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
     int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
     if (rc != BP_OK) return rc;
     rc = launch_pdl(batch_decide_kernel<GREEDY>, (unsigned)((p.num_seqs + kBThreads / 32 - 1) / (kBThreads / 32)), p,
                     stream);
     if (rc != BP_OK || GREEDY) return rc;
-    return launch_pdl(batch_draw_kernel<VEC>, (unsigned)(p.num_seqs * p.chunks), p, stream);
+    const unsigned draw_ctas = (unsigned)(p.num_seqs * p.chunks);
+    return draw_ctas > (unsigned)sm_count ? launch_pdl(batch_draw_kernel<VEC, 2>, draw_ctas, p, stream)
+                                          : launch_pdl(batch_draw_kernel<VEC, 1>, draw_ctas, p, stream);
 }
 }  // namespace
 
-int launch_accept_batch(const AcceptArgs& a, int* tickets, void* scratch, cudaStream_t stream) {
+int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* scratch, cudaStream_t stream) {
     BatchParams p;
     p.target = a.target;
     p.draft = a.draft;
@@ -499,12 +569,14 @@ int launch_accept_batch(const AcceptArgs& a, int* tickets, void* scratch, cudaSt
     p.k_ws = reinterpret_cast<int*>(w);
     w += align_up((size_t)a.num_seqs * sizeof(int), 256);
     p.ctot = reinterpret_cast<ulonglong2*>(w);
+    w += align_up((size_t)a.num_seqs * chunks * sizeof(ulonglong2), 256);
+    p.segm = reinterpret_cast<unsigned long long*>(w);
     p.tickets = tickets;
     p.err = a.err_word;
     const bool vec = (a.vocab % 4 == 0) && (reinterpret_cast<uintptr_t>(a.target) % 16 == 0) &&
                      (greedy || reinterpret_cast<uintptr_t>(a.draft) % 16 == 0);
-    if (greedy) return vec ? run_batch<true, true>(p, stream) : run_batch<true, false>(p, stream);
-    return vec ? run_batch<false, true>(p, stream) : run_batch<false, false>(p, stream);
+    if (greedy) return vec ? run_batch<true, true>(p, sm_count, stream) : run_batch<true, false>(p, sm_count, stream);
+    return vec ? run_batch<false, true>(p, sm_count, stream) : run_batch<false, false>(p, sm_count, stream);
 }
 
 }  // namespace bp

@@ -93,10 +93,21 @@ struct AcceptArgs {
 size_t accept_scratch_bytes(int num_seqs, int total_draft, int vocab);
 // allow_batch = false keeps every call on the cluster kernel (its scratch alone suffices)
 int launch_accept(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream, bool allow_batch = true);
-// From this many target rows on, the acceptance runs as three throughput kernels (accept_batch.cu).
-constexpr int kAcceptBatchRows = 48;
+// The acceptance runs as the throughput kernels of accept_batch.cu from this many logits read on (the
+// per-row cluster kernel below it): target rows x vocab at T = 0, target and drafter rows x vocab at
+// T > 0.  Set at the measured crossover of the two on GB300.
+constexpr long long kAcceptBatchLogitsT0 = 2500000;
+constexpr long long kAcceptBatchLogitsT1 = 6500000;
+inline bool accept_use_batch(int num_seqs, int total_draft, int vocab, bool greedy) {
+    const long long rows = greedy ? (long long)total_draft + num_seqs : 2LL * total_draft + num_seqs;
+    return rows * vocab >= (greedy ? kAcceptBatchLogitsT0 : kAcceptBatchLogitsT1);
+}
+// The workspace is sized for the throughput kernels when either temperature may use them.
+inline bool accept_may_batch(int num_seqs, int total_draft, int vocab) {
+    return accept_use_batch(num_seqs, total_draft, vocab, true) || accept_use_batch(num_seqs, total_draft, vocab, false);
+}
 size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab);
-int launch_accept_batch(const AcceptArgs& a, int* tickets, void* scratch, cudaStream_t stream);
+int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* scratch, cudaStream_t stream);
 // Same kernel, scratch taken from the library's own static device array (no workspace).
 int launch_accept_noalloc(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 

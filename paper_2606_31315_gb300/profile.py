@@ -8,6 +8,9 @@ CASE is one of:
                       15 drafter states, T = 1
   verify_epilogue_t0  the same at T = 0 (16 target states)
   accept_t1           acceptance over 16 x 151936 target and 15 x 151936 draft fp32 logits, T = 1
+  accept_batch_t1     acceptance over a batch of 32 sequences of 16 target rows (512 x 151936 target
+                      and 480 x 151936 draft fp32 logits), T = 1: the three throughput kernels
+  accept_batch_t0     the same batch at T = 0 (target logits only)
   attention           causal verify attention, 1 sequence, 2048 + 16 keys, 32 / 8 heads, D = 128
   tau                 Appendix A's acceptance-length model over 4M requests (24 positions, nine
                       candidate sizes, a predicted size each)
@@ -47,6 +50,18 @@ def _accept(dev, gen):
     return lambda: bp.spec_accept(t, d, tok, cu, 1.0, ua, us, ws=ws)
 
 
+def _accept_batch(dev, gen, temperature):
+    s = 32
+    td = s * (B - 1)
+    t = torch.randn(td + s, V, device=dev, generator=gen) * 3
+    d = torch.randn(td, V, device=dev, generator=gen) * 3 if temperature > 0 else None
+    tok = torch.randint(0, V, (td,), device=dev, generator=gen, dtype=torch.int32)
+    cu = torch.arange(0, td + 1, B - 1, dtype=torch.int32, device=dev)
+    ua, us = torch.rand(td, device=dev, generator=gen), torch.rand(s, device=dev, generator=gen)
+    ws = bp.workspace(bp.spec_accept_workspace_size(s, td, V), dev)
+    return lambda: bp.spec_accept(t, d, tok, cu, temperature, ua, us, ws=ws)
+
+
 def _attention(dev, gen):
     q = torch.randn(B, HQ, D, device=dev, generator=gen).to(torch.bfloat16)
     k = torch.randn(CTX + B, HKV, D, device=dev, generator=gen).to(torch.bfloat16)
@@ -71,6 +86,8 @@ CASES = {
     "verify_epilogue_t1": lambda dev, gen: _verify_epilogue(dev, gen, 1.0),
     "verify_epilogue_t0": lambda dev, gen: _verify_epilogue(dev, gen, 0.0),
     "accept_t1": _accept,
+    "accept_batch_t1": lambda dev, gen: _accept_batch(dev, gen, 1.0),
+    "accept_batch_t0": lambda dev, gen: _accept_batch(dev, gen, 0.0),
     "attention": _attention,
     "tau": _tau,
 }

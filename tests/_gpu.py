@@ -68,6 +68,36 @@ def attention_errors(o_gpu, lse_gpu, a: dict, mask: int, seqs, kv_head: int | No
     return worst, worst_lse
 
 
+# The library's choice between its two acceptance arrangements, mirrored so that tests can take both
+# sides: the throughput kernels from this many logits read on (target rows x vocab at T = 0, target and
+# drafter rows x vocab at T > 0), the per-row cluster kernel below it.
+BATCH_LOGITS_T0, BATCH_LOGITS_T1 = 2_500_000, 6_500_000
+
+
+def accept_uses_batch(blocks, vocab: int, temperature: float) -> bool:
+    s, td = len(blocks), int(np.sum(blocks)) - len(blocks)
+    rows = td + s if temperature == 0 else 2 * td + s
+    return rows * vocab >= (BATCH_LOGITS_T0 if temperature == 0 else BATCH_LOGITS_T1)
+
+
+SMALL_BLOCK_SETS = ((16, 1, 3, 9, 8), (16, 9, 1), (16, 9), (9, 1, 3), (4, 1))
+LARGE_BLOCKS = (16, 1, 3, 9, 24, 16, 5, 2, 16)
+
+
+def blocks_for(vocab: int, temperature: float, batch: bool) -> tuple:
+    """Ragged blocks (1 to 24 positions) whose acceptance at this vocabulary and temperature runs on the
+    throughput kernels (batch) or on the cluster kernel."""
+    if batch:
+        n = 1
+        while not accept_uses_batch(LARGE_BLOCKS * n, vocab, temperature):
+            n += 1
+        return LARGE_BLOCKS * n
+    for b in SMALL_BLOCK_SETS:
+        if not accept_uses_batch(b, vocab, temperature):
+            return b
+    raise ValueError("no small block set for this vocabulary")
+
+
 def run_accept(inp: dict, temperature: float, ws=None):
     g = {key: to_dev(inp[key]) for key in ("target_logits", "draft_tokens", "cu_draft", "u_accept", "u_sample")}
     draft = to_dev(inp["draft_logits"]) if temperature > 0 else None

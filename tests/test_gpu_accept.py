@@ -1,7 +1,7 @@
 """GPU parity of bp_spec_accept against the fp64 oracle.
 
-Batches of fewer than 48 target rows run on the cluster kernel, larger ones on the three throughput
-kernels; the edge cases below are taken on both sides of that line (ROWS_SMALL / ROWS_LARGE blocks).
+Small problems run on the cluster kernel, large ones (by logits read) on the throughput kernels; the
+edge cases below are taken on both sides of that line (blocks_for picks the blocks for either side).
 
 Bars: accept_prob within 1e-5 absolute at every drafted position; n_accepted and the emitted
 tokens bit-exact for every sequence not flagged as a near-tie (|u_i - a_i| < 1e-5 at a tested
@@ -16,7 +16,7 @@ from scipy import stats
 import paper_2606_31315_gb300 as bp
 from paper_2606_31315_gb300 import workloads as wl
 
-from _gpu import compare_accept, run_accept, run_oracle_accept, to_dev
+from _gpu import accept_uses_batch, blocks_for, compare_accept, run_accept, run_oracle_accept, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -40,13 +40,11 @@ def test_qwen3_4b_full(temp):
     compare_accept(wl.accept_inputs(w, temp), temp)
 
 
-BATCH_ROWS = 48  # from this many target rows on, the throughput kernels run
-SMALL_BLOCKS = (16, 1, 3, 9, 8)                   # 37 rows: cluster kernel
-LARGE_BLOCKS = (16, 1, 3, 9, 24, 16, 5, 2, 16)    # 92 rows: throughput kernels
-
-
-def test_block_sets_straddle_the_threshold():
-    assert sum(SMALL_BLOCKS) < BATCH_ROWS <= sum(LARGE_BLOCKS)
+def test_named_workloads_take_the_intended_path():
+    for name, temp, batch in (("qwen3_4b", 1.0, False), ("qwen3_4b", 0.0, False), ("tiny", 1.0, False),
+                              ("ragged", 1.0, True), ("ragged", 0.0, True), ("long_context", 1.0, True)):
+        w = wl.get(name)
+        assert accept_uses_batch(tuple(w.block), w.vocab, temp) == batch, name
 
 
 @pytest.mark.parametrize("temp", [1.0, 0.0])
@@ -74,12 +72,13 @@ def test_planted_long_prefixes(temp):
     assert n_acc.max() >= 10
 
 
-@pytest.mark.parametrize("blocks", [SMALL_BLOCKS, LARGE_BLOCKS])
+@pytest.mark.parametrize("batch", [False, True])
 @pytest.mark.parametrize("vocab", [5, 1001, 4099, 16384, 32000, 50001])
-def test_vocab_sizes_and_scalar_path(vocab, blocks):
+def test_vocab_sizes_and_scalar_path(vocab, batch):
     """Vocabularies below one chunk, exactly one, and ragged last chunks; odd sizes take the scalar loads."""
-    w = wl.custom(seed=vocab, ctx=(0,) * len(blocks), block=blocks, vocab=vocab)
     for temp in (1.0, 0.0):
+        blocks = blocks_for(vocab, temp, batch)
+        w = wl.custom(seed=vocab, ctx=(0,) * len(blocks), block=blocks, vocab=vocab)
         compare_accept(wl.accept_inputs(w, temp), temp)
 
 
@@ -137,8 +136,9 @@ def test_lossless_chi_square_on_gpu():
                    ref=run_oracle_accept(small, 1.0))
 
 
-@pytest.mark.parametrize("blocks", [(4, 4), LARGE_BLOCKS])
-def test_out_of_range_draft_token_sets_device_flag(blocks):
+@pytest.mark.parametrize("batch", [False, True])
+def test_out_of_range_draft_token_sets_device_flag(batch):
+    blocks = blocks_for(1000, 1.0, batch)
     w = wl.custom(seed=3, ctx=(0,) * len(blocks), block=blocks, vocab=1000)
     inp = wl.accept_inputs(w, 1.0)
     inp["draft_tokens"][2] = 1000  # caught by the kernel's own bounds check, never dereferenced
@@ -155,11 +155,12 @@ def test_host_side_validation():
     assert e.value.status == 1  # T > 0 needs draft logits
 
 
-@pytest.mark.parametrize("blocks", [(16, 9, 1, 5), (16, 9, 1, 5) * 3])
+@pytest.mark.parametrize("batch", [False, True])
 @pytest.mark.parametrize("temp", [1.0, 0.0])
-def test_masked_vocabulary(temp, blocks):
+def test_masked_vocabulary(temp, batch):
     """Logits of -inf (a masked vocabulary: the first 40% and a band in the middle) in every row:
     whole chunks of some lanes hold no finite entry, and the masked tokens must never be drawn."""
+    blocks = blocks_for(151936, temp, batch)
     w = wl.custom(seed=45, ctx=(0,) * len(blocks), block=blocks, vocab=151936)
     inp = wl.accept_inputs(w, temp)
     v = inp["target_logits"].shape[1]
@@ -181,12 +182,13 @@ def test_masked_vocabulary(temp, blocks):
     assert not masked[emitted].any()
 
 
-@pytest.mark.parametrize("blocks", [SMALL_BLOCKS, LARGE_BLOCKS])
+@pytest.mark.parametrize("batch", [False, True])
 @pytest.mark.parametrize("temp", [1.0, 0.0])
-def test_fully_masked_rows(temp, blocks):
+def test_fully_masked_rows(temp, batch):
     """Some drafter rows and some target rows with every entry -inf.  Greedy: the argmax of a masked
     target row is index 0.  T > 0: a masked drafter row has q = 0, so its token is accepted when p > 0
     and the residual is p itself; no NaN reaches a decision."""
+    blocks = blocks_for(3000, temp, batch)
     w = wl.custom(seed=46, ctx=(0,) * len(blocks), block=blocks, vocab=3000)
     inp = wl.accept_inputs(w, temp)
     inp["target_logits"] = inp["target_logits"].copy()
