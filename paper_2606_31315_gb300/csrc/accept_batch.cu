@@ -49,7 +49,7 @@ struct BatchParams {
     float* accept_prob;
     float2* part;      // [rows][chunks] chunk statistics (T = 0: value, index bits)
     float2* rowstat;   // [rows] row statistics
-    int* k_ws;         // [num_seqs] first rejection
+    float4* drawrec;   // [num_seqs][2] the draw's rows, weight constants and output slot (T > 0)
     ulonglong2* ctot;  // [num_seqs][chunks] draw masses of r and p (fixed point)
     unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses (chunks > 1)
     int* tickets;      // [num_seqs], zero between calls
@@ -85,12 +85,59 @@ __device__ __forceinline__ void load_chunk(const float* __restrict__ src, int n,
     for (int j = 0; j < kBVec; ++j) v[j] = load4<VEC>(src, 4 * (tid + j * kBThreads), n);
 }
 
+// The draw of a sequence: its row pair, the constants of its weights and the output slot, written by
+// the decisions as two 16-byte words and read back by every draw CTA in one round trip.
+struct DrawPair {
+    int trow, drow;  // drow < 0: a bonus draw from p alone
+    float Mt, izt, Md, izd;
+    int out;         // the emitted token's slot in out_tokens
+};
+__device__ __forceinline__ void store_draw(float4* rec, int trow, int drow, float2 st, float2 sd, int out) {
+    // a row whose entries are all -inf weighs every entry 0 (M = 0, 1/Z = 0 keep it free of NaN)
+    const bool tz = st.x == -INFINITY, dz = drow < 0 || sd.x == -INFINITY;
+    rec[0] = make_float4(__int_as_float(trow), __int_as_float(drow), tz ? 0.f : st.x, tz ? 0.f : __fdiv_rn(1.f, st.y));
+    rec[1] = make_float4(dz ? 0.f : sd.x, dz ? 0.f : __fdiv_rn(1.f, sd.y), __int_as_float(out), 0.f);
+}
+__device__ __forceinline__ DrawPair load_draw(const float4* rec) {
+    const float4 a = __ldcg(rec), b = __ldcg(rec + 1);
+    DrawPair d;
+    d.trow = __float_as_int(a.x);
+    d.drow = __float_as_int(a.y);
+    d.Mt = a.z;
+    d.izt = a.w;
+    d.Md = b.x;
+    d.izd = b.y;
+    d.out = __float_as_int(b.z);
+    return d;
+}
+
 // Decisions of sequence s, by one warp: its rows' statistics from their chunks', the ratios a_i, the
 // first rejection k and the outputs (at T = 0 the emitted argmax too).
 template <bool GREEDY>
 __device__ __forceinline__ void decide_seq(const BatchParams& p, int s, int lane) {
     const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
     const int nrows = GREEDY ? g + 1 : 2 * g + 1;  // the target rows, then (T > 0) the drafter's
+    // the drafted tokens, their two logits and uniforms do not depend on the statistics: the first 32
+    // positions' loads are issued before the merges
+    struct Pick {
+        int x;
+        bool valid;
+        float tx, dx, u;
+    };
+    const auto pick = [&](int i) {
+        Pick q{-1, false, -INFINITY, -INFINITY, 1.f};
+        if (i < g) {
+            q.x = p.tokens[d0 + i];
+            q.valid = q.x >= 0 && q.x < p.vocab;
+            if (!GREEDY && q.valid) {
+                q.tx = p.target[(size_t)(t0 + i) * p.vocab + q.x];
+                q.dx = p.draft[(size_t)(d0 + i) * p.vocab + q.x];
+            }
+            if (!GREEDY) q.u = p.u_accept[d0 + i];
+        }
+        return q;
+    };
+    const Pick first = pick(lane);
     // each lane merges whole rows (two at a time), chunks in order, eight chunks' loads in flight
     constexpr int RH = 2, CQ = 8;
     const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
@@ -136,25 +183,22 @@ __device__ __forceinline__ void decide_seq(const BatchParams& p, int s, int lane
     int k = g;
     for (int i0 = 0; i0 < g; i0 += 32) {
         const int i = i0 + lane;
+        const Pick q = i0 == 0 ? first : pick(i);
         bool rej = false;
         if (i < g) {
-            const int x = p.tokens[d0 + i];
-            const bool valid = x >= 0 && x < p.vocab;
-            if (!valid) raise_error(p.err, kErrDeviceArg);
+            if (!q.valid) raise_error(p.err, kErrDeviceArg);
             const float2 st = p.rowstat[t0 + i];
             float a;
             if (GREEDY) {
-                a = valid && x == __float_as_int(st.y) ? 1.f : 0.f;
+                a = q.valid && q.x == __float_as_int(st.y) ? 1.f : 0.f;
                 rej = a == 0.f;
             } else {
-                const float tx = valid ? p.target[(size_t)(t0 + i) * p.vocab + x] : -INFINITY;
-                const float dx = valid ? p.draft[(size_t)(d0 + i) * p.vocab + x] : -INFINITY;
                 const float2 sd = p.rowstat[p.rows_t + d0 + i];
                 // a = min(1, p(x)/q(x)) in the log domain (q(x) = 0 < p(x) gives 1, p(x) = 0 gives 0)
-                if (!valid || tx == -INFINITY) a = 0.f;
-                else if (dx == -INFINITY) a = 1.f;
-                else a = fminf(1.f, ex2(__fmaf_rn(tx, p.c2, -st.x) - __fmaf_rn(dx, p.c2, -sd.x)) * (sd.y / st.y));
-                rej = !(p.u_accept[d0 + i] < a);
+                if (!q.valid || q.tx == -INFINITY) a = 0.f;
+                else if (q.dx == -INFINITY) a = 1.f;
+                else a = fminf(1.f, ex2(__fmaf_rn(q.tx, p.c2, -st.x) - __fmaf_rn(q.dx, p.c2, -sd.x)) * (sd.y / st.y));
+                rej = !(q.u < a);
             }
             if (p.accept_prob) p.accept_prob[d0 + i] = a;
         }
@@ -168,7 +212,11 @@ __device__ __forceinline__ void decide_seq(const BatchParams& p, int s, int lane
     }
     if (lane == 0) {
         p.n_accepted[s] = k;
-        if (!GREEDY) p.k_ws[s] = k;
+        if (!GREEDY) {
+            const int drow = k < g ? p.rows_t + d0 + k : -1;
+            store_draw(p.drawrec + 2 * s, t0 + k, drow, p.rowstat[t0 + k],
+                       drow >= 0 ? p.rowstat[drow] : make_float2(-INFINITY, 0.f), t0 + k);
+        }
     }
 }
 
@@ -246,29 +294,6 @@ __global__ void __launch_bounds__(kBThreads) batch_decide_kernel(const BatchPara
     if (s < p.num_seqs) decide_seq<GREEDY>(p, s, threadIdx.x & 31);
 }
 
-// The draw row pair of a sequence and the constants of its weights.
-struct DrawPair {
-    int trow, drow;  // drow < 0: a bonus draw from p alone
-    float Mt, izt, Md, izd;
-};
-__device__ __forceinline__ DrawPair draw_rows(const BatchParams& p, int t0, int d0, int g, int k) {
-    DrawPair d;
-    d.trow = t0 + k;
-    d.drow = k < g ? p.rows_t + d0 + k : -1;
-    return d;
-}
-// The weights' constants from the rows' statistics (read after the rows' loads are issued).
-__device__ __forceinline__ void draw_consts(const BatchParams& p, DrawPair& d) {
-    // a row whose entries are all -inf weighs every entry 0 (M = 0, 1/Z = 0 keep it free of NaN)
-    const float2 st = p.rowstat[d.trow];
-    const bool tz = st.x == -INFINITY;
-    d.Mt = tz ? 0.f : st.x;
-    d.izt = tz ? 0.f : __fdiv_rn(1.f, st.y);
-    const float2 sd = d.drow >= 0 ? p.rowstat[d.drow] : make_float2(-INFINITY, 0.f);
-    const bool dz = sd.x == -INFINITY;
-    d.Md = dz ? 0.f : sd.x;
-    d.izd = dz ? 0.f : __fdiv_rn(1.f, sd.y);
-}
 // Weights of four entries: (r = max(0, p - q), p) with p = 2^(l*c2 - Mt) / Zt (r = 0 without a draft row).
 __device__ __forceinline__ void weights4(float4 lt, float4 ld, const DrawPair& d, float c2, float4& r, float4& pw) {
     const auto pt = [&](float l) { return __fmul_rn(ex2(__fmaf_rn(l, c2, -d.Mt)), d.izt); };
@@ -289,7 +314,7 @@ __device__ __forceinline__ float sum4f(float4 v) { return (v.x + v.y) + (v.z + v
 // keeps every load in flight (for grids of at most one CTA per SM), two fit 128 registers, i.e. two
 // CTAs per SM (for larger grids).
 template <bool VEC, int PH>
-__device__ __forceinline__ unsigned long long chunk_masses(const BatchParams& p, DrawPair& d, int chunk, int tid,
+__device__ __forceinline__ unsigned long long chunk_masses(const BatchParams& p, const DrawPair& d, int chunk, int tid,
                                                            unsigned long long (*segR)[kBSegs],
                                                            unsigned long long (*segP)[kBSegs]) {
     const int lane = tid & 31, warp = tid >> 5;
@@ -307,7 +332,6 @@ __device__ __forceinline__ unsigned long long chunk_masses(const BatchParams& p,
             lt[jj] = load4<VEC>(tp, e, n);
             if (d.drow >= 0) ld[jj] = load4<VEC>(dp, e, n);
         }
-        if (h == 0) draw_consts(p, d);
 #pragma unroll
         for (int jj = 0; jj < JP; ++jj) {
             const int j = h * JP + jj;
@@ -333,9 +357,7 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
     griddep_wait();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int s = blockIdx.x / p.chunks, chunk = blockIdx.x - s * p.chunks;
-    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
-    const int k = p.k_ws[s];
-    DrawPair d = draw_rows(p, t0, d0, g, k);  // its constants are filled in by chunk_masses
+    const DrawPair d = load_draw(p.drawrec + 2 * s);
     constexpr int kSeg = kBThreads / 32 * kBSegs;  // 128 segments per chunk
     static_assert(kBSegs == 16 && 2 * kSeg == kBThreads, "one segment mass per thread");
     const unsigned long long f = chunk_masses<VEC, PH>(p, d, chunk, tid, segR, segP);
@@ -407,7 +429,7 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
         if (lane == 0) {
             if (total == 0 || cstar < 0) {  // no positive mass (or unreachable with exact sums): report
                 raise_error(p.err, kErrDeviceArg);
-                p.out_tokens[t0 + k] = 0;
+                p.out_tokens[d.out] = 0;
                 cstar = -1;
             }
             cstar_sh = cstar;
@@ -451,7 +473,7 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
             if (hit == 0u) {
                 if (lane == 0) {  // unreachable with exact sums: report, emit the chunk's first entry
                     raise_error(p.err, kErrDeviceArg);
-                    p.out_tokens[t0 + k] = cstar * kBChunk;
+                    p.out_tokens[d.out] = cstar * kBChunk;
                     jstar_sh = -1;
                 }
             } else if (lane == __ffs(hit) - 1) {
@@ -495,7 +517,7 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
             // segment's last entry with positive weight
             const int tok = any ? __shfl_sync(0xffffffffu, hit, __ffs(any) - 1)
                                 : (pos ? __shfl_sync(0xffffffffu, lastpos, 31 - __clz(pos)) : v0 + e0);
-            if (lane == 0) p.out_tokens[t0 + k] = tok;
+            if (lane == 0) p.out_tokens[d.out] = tok;
         }
     }
     if (tid == 0) p.tickets[s] = 0;  // ready for the next call
@@ -508,7 +530,7 @@ size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
     const size_t rows = 2 * (size_t)total_draft + num_seqs;
     const size_t segm = chunks > 1 ? (size_t)num_seqs * chunks * 2 * 128 * sizeof(unsigned long long) : 0;
     return align_up(rows * chunks * sizeof(float2), 256) + align_up(rows * sizeof(float2), 256) +
-           align_up((size_t)num_seqs * sizeof(int), 256) +
+           align_up((size_t)num_seqs * 2 * sizeof(float4), 256) +
            align_up((size_t)num_seqs * chunks * sizeof(ulonglong2), 256) + align_up(segm, 256);
 }
 
@@ -566,8 +588,8 @@ int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* s
     w += align_up(rows * chunks * sizeof(float2), 256);
     p.rowstat = reinterpret_cast<float2*>(w);
     w += align_up(rows * sizeof(float2), 256);
-    p.k_ws = reinterpret_cast<int*>(w);
-    w += align_up((size_t)a.num_seqs * sizeof(int), 256);
+    p.drawrec = reinterpret_cast<float4*>(w);
+    w += align_up((size_t)a.num_seqs * 2 * sizeof(float4), 256);
     p.ctot = reinterpret_cast<ulonglong2*>(w);
     w += align_up((size_t)a.num_seqs * chunks * sizeof(ulonglong2), 256);
     p.segm = reinterpret_cast<unsigned long long*>(w);
