@@ -20,6 +20,8 @@
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "ptx_sm103.cuh"
 
@@ -152,7 +154,7 @@ constexpr int kTcMaxN = 64;        // requests per group: the MMA N (padded to a
 constexpr int kTcAtom = 64;        // d_in columns per 128-byte swizzle atom
 constexpr int kTcAtomBytes = kTcM * kTcAtom * 2;  // 16 KB of W1 per atom
 constexpr int kTcMaxAtoms = 8;     // atoms per CTA when all of them are loaded at once
-constexpr int kTcStages = 5;       // ring depth when the atoms of a CTA are streamed (large d_in)
+constexpr int kTcStages = 5;       // ring depth at most, when the atoms of a CTA are streamed (large d_in)
 constexpr int kTcMaxKS = 9;        // CTAs per cluster (non-portable above 8)
 constexpr int kTcThreads = 128;    // thread t = tile row t = TMEM lane t
 constexpr uint32_t kTcTmemCols = 64;
@@ -165,6 +167,7 @@ struct PolicyTcParams {
     int num_reqs, d_in, hidden, num_cand;
     int atoms_total, atoms_per_cta, tiles, npad;
     int w_bytes, x_bytes, h_bytes, op_bytes;  // dynamic shared-memory regions
+    int stages, aps;  // ring: its depth and the atoms each stage carries
     const float* b1;
     const __nv_bfloat16* w2;
     const float* b2;
@@ -208,8 +211,9 @@ __global__ void __launch_bounds__(256) policy_gather_kernel(const __nv_bfloat16*
 }
 
 // RING = false: every W1 and x atom of the CTA is loaded at once (x gathered by the CTA itself).
-// RING = true: the atoms stream through a kTcStages-deep ring (W1 and the gathered x by TMA), for
-// any d_in; thread 0 produces, thread 32 issues the MMAs.
+// RING = true: the atoms stream through a ring of p.stages stages (W1 and the gathered x by TMA), for
+// any d_in; thread 0 produces, thread 32 issues the MMAs.  A stage carries p.aps consecutive atoms,
+// so with two each W1 row is fetched as 256 contiguous bytes per stage rather than 128.
 template <bool RING>
 __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_constant__ CUtensorMap w1map,
                                                               const __grid_constant__ CUtensorMap xmap,
@@ -248,10 +252,10 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     if (tid == 0) {
         prefetch_tensormap(&w1map);
         if (RING) prefetch_tensormap(&xmap);
-        const int nb = RING ? kTcStages : na;
+        const int nb = RING ? p.stages : na;
         for (int a = 0; a < nb; ++a) mbar_init(&bar_w[a], 1);
         if (RING)
-            for (int st = 0; st < kTcStages; ++st) mbar_init(&bar_empty[st], 1);
+            for (int st = 0; st < p.stages; ++st) mbar_init(&bar_empty[st], 1);
         mbar_init(&bar_mma, 1);
         fence_mbar_init();
     }
@@ -266,34 +270,42 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     const uint32_t tmem = tmem_sh;
     griddep_wait();  // inputs may come from the previous kernel on the stream
     if (RING) {
-        const uint32_t stage_bytes = (uint32_t)(kTcAtomBytes + npad * 128);
+        const int S = p.stages, A = p.aps;
+        const int nq = (na + A - 1) / A;  // stages this CTA fills; the last may carry fewer atoms
+        const uint32_t atom_bytes = (uint32_t)(kTcAtomBytes + npad * 128);
         if (tid == 0) {  // producer: W1 and x atoms through the ring
-            for (int j = 0; j < na; ++j) {
-                const int st = j % kTcStages;
-                if (j >= kTcStages && !mbar_wait(&bar_empty[st], ((j / kTcStages) - 1) & 1, kWaitBudget)) {
+            for (int q = 0; q < nq; ++q) {
+                const int st = q % S, nat = min(A, na - q * A);
+                if (q >= S && !mbar_wait(&bar_empty[st], ((q / S) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
-                mbar_arrive_expect_tx(&bar_w[st], stage_bytes);
-                tma_load_2d(sW + st * kTcAtomBytes, &w1map, &bar_w[st], (a0 + j) * kTcAtom, m0);
-                tma_load_2d(sX + st * npad * 128, &xmap, &bar_w[st], (a0 + j) * kTcAtom, n0);
+                mbar_arrive_expect_tx(&bar_w[st], atom_bytes * (uint32_t)nat);
+                for (int t = 0; t < nat; ++t) {
+                    const int col = (a0 + q * A + t) * kTcAtom;
+                    tma_load_2d(sW + (st * A + t) * kTcAtomBytes, &w1map, &bar_w[st], col, m0);
+                    tma_load_2d(sX + (st * A + t) * npad * 128, &xmap, &bar_w[st], col, n0);
+                }
             }
         } else if (tid == 32) {  // MMA issuer
             if (na > 0) {
                 const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
                 bool ok = true;
-                for (int j = 0; j < na; ++j) {
-                    const int st = j % kTcStages;
-                    if (!mbar_wait(&bar_w[st], (j / kTcStages) & 1, kWaitBudget)) {
+                for (int q = 0; q < nq; ++q) {
+                    const int st = q % S, nat = min(A, na - q * A);
+                    if (!mbar_wait(&bar_w[st], (q / S) & 1, kWaitBudget)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    const uint32_t wa = smem_addr(sW + st * kTcAtomBytes), xa = smem_addr(sX + st * npad * 128);
+                    for (int t = 0; t < nat; ++t) {
+                        const uint32_t wa = smem_addr(sW + (st * A + t) * kTcAtomBytes);
+                        const uint32_t xa = smem_addr(sX + (st * A + t) * npad * 128);
 #pragma unroll
-                    for (int kk = 0; kk < kTcAtom / 16; ++kk)
-                        umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
-                                smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (j | kk) ? 1u : 0u);
+                        for (int kk = 0; kk < kTcAtom / 16; ++kk)
+                            umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                                    smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (q | t | kk) ? 1u : 0u);
+                    }
                     umma_commit(&bar_empty[st]);  // the stage is free once these MMAs have read it
                 }
                 if (!ok) raise_error(p.err, kErrTimeout);
@@ -509,6 +521,63 @@ size_t tc_x_bytes(int num_reqs, int d_in) {
     return align_up(groups * kTcMaxN * (size_t)d_in * 2, 256);
 }
 
+// Opt-in shared memory and non-portable cluster sizes, once per device.
+int configure_tc(int device) {
+    static std::mutex mu;
+    static bool configured[64] = {};
+    std::lock_guard<std::mutex> lock(mu);
+    if (device >= 0 && device < 64 && configured[device]) return BP_OK;
+    if (cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
+            cudaSuccess ||
+        cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+        return BP_ERR_CUDA;
+    if (device >= 0 && device < 64) configured[device] = true;
+    return BP_OK;
+}
+
+// Clusters of ks streaming CTAs with smem bytes of dynamic shared memory each that the device holds at
+// once (cached per device, cluster size and size).  The occupancy query counts clusters at one CTA per
+// SM (on this GB300 it answers 15 nine-CTA clusters at every size); clusters also share SMs when the
+// shared memory lets several CTAs fit, so its count is scaled by the CTAs per SM (measured: 16 such
+// clusters ran at once at two CTAs per SM, not at one).
+int active_ring_clusters(int device, int ks, int smem) {
+    struct Entry {
+        int device, ks, smem, n;
+    };
+    static std::mutex mu;
+    static Entry cache[64];
+    static int used = 0;
+    std::lock_guard<std::mutex> lock(mu);
+    for (int i = 0; i < used; ++i)
+        if (cache[i].device == device && cache[i].ks == ks && cache[i].smem == smem) return cache[i].n;
+    cudaLaunchConfig_t probe = {};
+    cudaLaunchAttribute pa[1];
+    probe.gridDim = dim3((unsigned)ks, 1, 1);
+    probe.blockDim = dim3(kTcThreads, 1, 1);
+    probe.dynamicSmemBytes = (size_t)smem;
+    pa[0].id = cudaLaunchAttributeClusterDimension;
+    pa[0].val.clusterDim.x = (unsigned)ks;
+    pa[0].val.clusterDim.y = 1;
+    pa[0].val.clusterDim.z = 1;
+    probe.attrs = pa;
+    probe.numAttrs = 1;
+    int n = 0, per_sm = 0, reserved = 0;
+    if (cudaOccupancyMaxActiveClusters(&n, policy_tc_kernel<true>, &probe) != cudaSuccess ||
+        cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, device) != cudaSuccess ||
+        cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, device) != cudaSuccess) {
+        cudaGetLastError();
+        n = 0;
+    }
+    const int ctas_per_sm = per_sm / (smem + reserved);
+    n *= ctas_per_sm > 1 ? ctas_per_sm : 1;
+    if (used < 64) cache[used++] = Entry{device, ks, smem, n};
+    return n;
+}
+
 // Launches the tensor-core path; returns -1 when the shape is outside its limits.
 int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counters, __nv_bfloat16* xg,
            cudaStream_t stream) {
@@ -524,17 +593,43 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     ks = ks > atoms_total ? atoms_total : ks;
     const int per = (atoms_total + ks - 1) / ks;
     const bool ring = per > kTcMaxAtoms;  // too many atoms to hold at once: stream them
-    const int slots = ring ? kTcStages : per;
     const int pd_bytes = kTcM * (npad + 4) * 4;
-    const int w_bytes = slots * kTcAtomBytes > pd_bytes ? slots * kTcAtomBytes : pd_bytes;
-    const int x_bytes = slots * npad * 128;
     const int rpr = (kTcM + ks - 1) / ks;
     int h_bytes = rpr * npad * 4;
     const int lg_bytes = kTcMaxN * a.num_cand * 4;  // the last tile's logits reuse the h region
     h_bytes = h_bytes > lg_bytes ? h_bytes : lg_bytes;
     const int op_bytes = kTcMaxN * a.num_cand * 4;
     const int w2s_bytes = a.num_cand * rpr * 4;
-    const int smem = 1024 + w_bytes + x_bytes + h_bytes + op_bytes + w2s_bytes;
+    const auto smem_for = [&](int slots) {  // atoms held at once
+        const int wb = slots * kTcAtomBytes > pd_bytes ? slots * kTcAtomBytes : pd_bytes;
+        return 1024 + wb + slots * npad * 128 + h_bytes + op_bytes + w2s_bytes;
+    };
+    if (configure_tc(dev.device) != BP_OK) return BP_ERR_CUDA;
+    // ring: the deepest configuration (two atoms per stage, 256-byte row fetches, first) under which
+    // every cluster of the grid is resident at once -- a cluster left for a second wave streams its
+    // tile alone at a fraction of the bandwidth (measured at 32 requests x 151936 -> 2048: 16 tiles of
+    // 9-CTA clusters took 179 us at one CTA per SM, 125 us at two); if none, the deepest that fits
+    int stages = kTcStages, aps = 1;
+    if (ring) {
+        const int tries[7][2] = {{4, 2}, {3, 2}, {2, 2}, {5, 1}, {4, 1}, {3, 1}, {2, 1}};
+        int pick = -1;
+        for (int i = 0; i < 7; ++i) {
+            const int sm = smem_for(tries[i][0] * tries[i][1]);
+            if (sm > kTcMaxSmem) continue;
+            if (pick < 0) pick = i;
+            if (active_ring_clusters(dev.device, ks, sm) >= tiles * groups) {
+                pick = i;
+                break;
+            }
+        }
+        if (pick < 0) return -1;
+        stages = tries[pick][0];
+        aps = tries[pick][1];
+    }
+    const int slots = ring ? stages * aps : per;
+    const int w_bytes = slots * kTcAtomBytes > pd_bytes ? slots * kTcAtomBytes : pd_bytes;
+    const int x_bytes = slots * npad * 128;
+    const int smem = smem_for(slots);
     if (smem > kTcMaxSmem) return -1;
 
     CUtensorMap w1map, xmap;
@@ -552,19 +647,6 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
                               CU_TENSOR_MAP_SWIZZLE_128B) != BP_OK)
             return -1;
     }
-    static int configured[64] = {};
-    if (dev.device >= 0 && dev.device < 64 && !configured[dev.device]) {
-        if (cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
-                cudaSuccess ||
-            cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
-                cudaSuccess ||
-            cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-                cudaSuccess ||
-            cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-                cudaSuccess)
-            return BP_ERR_CUDA;
-        configured[dev.device] = 1;
-    }
     PolicyTcParams p;
     p.feats = static_cast<const __nv_bfloat16*>(a.feats);
     p.row_stride = a.row_stride;
@@ -581,6 +663,8 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     p.x_bytes = x_bytes;
     p.h_bytes = h_bytes;
     p.op_bytes = op_bytes;
+    p.stages = stages;
+    p.aps = aps;
     p.b1 = a.b1;
     p.w2 = static_cast<const __nv_bfloat16*>(a.w2);
     p.b2 = a.b2;

@@ -12,6 +12,9 @@ CASE is one of:
                       and 480 x 151936 draft fp32 logits), T = 1: the three throughput kernels
   accept_batch_t0     the same batch at T = 0 (target logits only)
   attention           causal verify attention, 1 sequence, 2048 + 16 keys, 32 / 8 heads, D = 128
+  policy              policy head, 32 requests, 2560 -> 2048 -> 9 bf16 (W1 loaded at once per CTA)
+  policy_d151936      policy head at the paper's input width, 32 requests, 151936 -> 2048 -> 9 bf16
+                      (W1 622 MB streamed through the ring)
   tau                 Appendix A's acceptance-length model over 4M requests (24 positions, nine
                       candidate sizes, a predicted size each)
 """
@@ -72,6 +75,18 @@ def _attention(dev, gen):
     return lambda: bp.block_attention(q, k, v, cu_q, cu_kv, B, CTX + B, mask=bp.MASK_CAUSAL, ws=ws)
 
 
+def _policy(dev, gen, d_in):
+    n, hidden, c = 32, 2048, 9
+    feats = torch.randn(n, d_in, device=dev, generator=gen).to(torch.bfloat16)
+    w1 = (torch.randn(hidden, d_in, device=dev, generator=gen) / d_in ** 0.5).to(torch.bfloat16)
+    b1 = torch.randn(hidden, device=dev, generator=gen) * 0.1
+    w2 = (torch.randn(c, hidden, device=dev, generator=gen) / hidden ** 0.5).to(torch.bfloat16)
+    b2 = torch.randn(c, device=dev, generator=gen) * 0.1
+    cand = torch.arange(8, 8 + 2 * c, 2, dtype=torch.int32, device=dev)
+    ws = bp.workspace(bp.policy_select_workspace_size(n, d_in, hidden, c), dev)
+    return lambda: bp.policy_select(feats, w1, b1, w2, b2, cand, want_logits=False, ws=ws)
+
+
 def _tau(dev, gen):
     n, j = 1 << 22, 24
     g = (0.86 + 0.05 * torch.randn(n, j, device=dev, generator=gen)).clamp_(0.05, 0.999).contiguous()
@@ -89,6 +104,8 @@ CASES = {
     "accept_batch_t1": lambda dev, gen: _accept_batch(dev, gen, 1.0),
     "accept_batch_t0": lambda dev, gen: _accept_batch(dev, gen, 0.0),
     "attention": _attention,
+    "policy": lambda dev, gen: _policy(dev, gen, 2560),
+    "policy_d151936": lambda dev, gen: _policy(dev, gen, V),
     "tau": _tau,
 }
 
