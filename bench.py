@@ -492,8 +492,9 @@ def run_ours(args):
         "a7_accept_greedy_t0": row(t_acc0, accept_bytes(w, 0.0), ["accept_kernel<true,true>"]),
         "a1_policy_head_32req_2560x2048": row(t_pol, policy_bytes(pin), ["policy_tc_kernel"]),
         "next3_verify_attention_paged_page64": row(t_attn_paged, attention_bytes(w), ["attn_bf16_tc_kernel (paged)"]),
-        "next2_policy_head_32req_151936x2048": row(t_pol_big, big_bytes,
-                                                   ["policy_gather_kernel", "policy_tc_kernel (streamed)"]),
+        "next2_policy_head_32req_151936x2048": dict(
+            row(t_pol_big, big_bytes, ["policy_gather_kernel", "policy_tc_kernel<true,5> (streamed)"]),
+            traffic=committed_traffic("policy_tc_kernel_ring")),
         "next1_fused_verify_epilogue_qwen3_4b_t1": dict(
             row(t_ve, ve_bytes, ["verify_epilogue_kernel<false,32,2>"]),
             traffic=committed_traffic("verify_epilogue_kernel"),

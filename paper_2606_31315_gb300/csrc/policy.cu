@@ -167,7 +167,6 @@ struct PolicyTcParams {
     int num_reqs, d_in, hidden, num_cand;
     int atoms_total, atoms_per_cta, tiles, npad;
     int w_bytes, x_bytes, h_bytes, op_bytes;  // dynamic shared-memory regions
-    int stages, aps;  // ring: its depth and the atoms each stage carries
     const float* b1;
     const __nv_bfloat16* w2;
     const float* b2;
@@ -211,10 +210,12 @@ __global__ void __launch_bounds__(256) policy_gather_kernel(const __nv_bfloat16*
 }
 
 // RING = false: every W1 and x atom of the CTA is loaded at once (x gathered by the CTA itself).
-// RING = true: the atoms stream through a ring of p.stages stages (W1 and the gathered x by TMA), for
-// any d_in; thread 0 produces, thread 32 issues the MMAs.  A stage carries p.aps consecutive atoms,
-// so with two each W1 row is fetched as 256 contiguous bytes per stage rather than 128.
-template <bool RING>
+// RING = true: the atoms stream through a ring of S stages of one atom (W1 and the gathered x by TMA),
+// for any d_in; thread 0 produces, thread 32 issues the MMAs.  S is compile-time: the producer and the
+// issuer are single threads on the critical path of every stage (with S and the atoms per stage as
+// runtime values the same ring ran 127.0 instead of 116.8 us at 32 requests x 151936 -> 2048; two
+// atoms per stage at half the depth, 256-byte row fetches, measured 127.4 us).
+template <bool RING, int S>
 __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_constant__ CUtensorMap w1map,
                                                               const __grid_constant__ CUtensorMap xmap,
                                                               const PolicyTcParams p) {
@@ -252,10 +253,10 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     if (tid == 0) {
         prefetch_tensormap(&w1map);
         if (RING) prefetch_tensormap(&xmap);
-        const int nb = RING ? p.stages : na;
+        const int nb = RING ? S : na;
         for (int a = 0; a < nb; ++a) mbar_init(&bar_w[a], 1);
         if (RING)
-            for (int st = 0; st < p.stages; ++st) mbar_init(&bar_empty[st], 1);
+            for (int st = 0; st < S; ++st) mbar_init(&bar_empty[st], 1);
         mbar_init(&bar_mma, 1);
         fence_mbar_init();
     }
@@ -270,42 +271,35 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
     const uint32_t tmem = tmem_sh;
     griddep_wait();  // inputs may come from the previous kernel on the stream
     if (RING) {
-        const int S = p.stages, A = p.aps;
-        const int nq = (na + A - 1) / A;  // stages this CTA fills; the last may carry fewer atoms
-        const uint32_t atom_bytes = (uint32_t)(kTcAtomBytes + npad * 128);
+        static_assert(!RING || (S >= 2 && S <= kTcStages && S <= kTcMaxAtoms), "ring depth");
+        const uint32_t stage_bytes = (uint32_t)(kTcAtomBytes + npad * 128);
         if (tid == 0) {  // producer: W1 and x atoms through the ring
-            for (int q = 0; q < nq; ++q) {
-                const int st = q % S, nat = min(A, na - q * A);
-                if (q >= S && !mbar_wait(&bar_empty[st], ((q / S) - 1) & 1, kWaitBudget)) {
+            for (int j = 0; j < na; ++j) {
+                const int st = j % S;
+                if (j >= S && !mbar_wait(&bar_empty[st], ((j / S) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
                     break;
                 }
-                mbar_arrive_expect_tx(&bar_w[st], atom_bytes * (uint32_t)nat);
-                for (int t = 0; t < nat; ++t) {
-                    const int col = (a0 + q * A + t) * kTcAtom;
-                    tma_load_2d(sW + (st * A + t) * kTcAtomBytes, &w1map, &bar_w[st], col, m0);
-                    tma_load_2d(sX + (st * A + t) * npad * 128, &xmap, &bar_w[st], col, n0);
-                }
+                mbar_arrive_expect_tx(&bar_w[st], stage_bytes);
+                tma_load_2d(sW + st * kTcAtomBytes, &w1map, &bar_w[st], (a0 + j) * kTcAtom, m0);
+                tma_load_2d(sX + st * npad * 128, &xmap, &bar_w[st], (a0 + j) * kTcAtom, n0);
             }
         } else if (tid == 32) {  // MMA issuer
             if (na > 0) {
                 const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
                 bool ok = true;
-                for (int q = 0; q < nq; ++q) {
-                    const int st = q % S, nat = min(A, na - q * A);
-                    if (!mbar_wait(&bar_w[st], (q / S) & 1, kWaitBudget)) {
+                for (int j = 0; j < na; ++j) {
+                    const int st = j % S;
+                    if (!mbar_wait(&bar_w[st], (j / S) & 1, kWaitBudget)) {
                         ok = false;
                         break;
                     }
                     tc_fence_after();
-                    for (int t = 0; t < nat; ++t) {
-                        const uint32_t wa = smem_addr(sW + (st * A + t) * kTcAtomBytes);
-                        const uint32_t xa = smem_addr(sX + (st * A + t) * npad * 128);
+                    const uint32_t wa = smem_addr(sW + st * kTcAtomBytes), xa = smem_addr(sX + st * npad * 128);
 #pragma unroll
-                        for (int kk = 0; kk < kTcAtom / 16; ++kk)
-                            umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
-                                    smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (q | t | kk) ? 1u : 0u);
-                    }
+                    for (int kk = 0; kk < kTcAtom / 16; ++kk)
+                        umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
+                                smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (j | kk) ? 1u : 0u);
                     umma_commit(&bar_empty[st]);  // the stage is free once these MMAs have read it
                 }
                 if (!ok) raise_error(p.err, kErrTimeout);
@@ -521,20 +515,27 @@ size_t tc_x_bytes(int num_reqs, int d_in) {
     return align_up(groups * kTcMaxN * (size_t)d_in * 2, 256);
 }
 
+// The instantiations: the one-shot kernel, then the rings, deepest first (the order of preference).
+using TcFn = void (*)(CUtensorMap, CUtensorMap, PolicyTcParams);
+struct TcKernel {
+    TcFn fn;
+    int stages;
+};
+constexpr int kTcRings = 4;
+const TcKernel kTcKernels[1 + kTcRings] = {{policy_tc_kernel<false, 1>, 0}, {policy_tc_kernel<true, 5>, 5},
+                                           {policy_tc_kernel<true, 4>, 4}, {policy_tc_kernel<true, 3>, 3},
+                                           {policy_tc_kernel<true, 2>, 2}};
+
 // Opt-in shared memory and non-portable cluster sizes, once per device.
 int configure_tc(int device) {
     static std::mutex mu;
     static bool configured[64] = {};
     std::lock_guard<std::mutex> lock(mu);
     if (device >= 0 && device < 64 && configured[device]) return BP_OK;
-    if (cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(policy_tc_kernel<false>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) !=
-            cudaSuccess ||
-        cudaFuncSetAttribute(policy_tc_kernel<true>, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
-        return BP_ERR_CUDA;
+    for (const TcKernel k : kTcKernels)
+        if (cudaFuncSetAttribute(k.fn, cudaFuncAttributeMaxDynamicSharedMemorySize, kTcMaxSmem) != cudaSuccess ||
+            cudaFuncSetAttribute(k.fn, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess)
+            return BP_ERR_CUDA;
     if (device >= 0 && device < 64) configured[device] = true;
     return BP_OK;
 }
@@ -566,7 +567,7 @@ int active_ring_clusters(int device, int ks, int smem) {
     probe.attrs = pa;
     probe.numAttrs = 1;
     int n = 0, per_sm = 0, reserved = 0;
-    if (cudaOccupancyMaxActiveClusters(&n, policy_tc_kernel<true>, &probe) != cudaSuccess ||
+    if (cudaOccupancyMaxActiveClusters(&n, kTcKernels[1].fn, &probe) != cudaSuccess ||
         cudaDeviceGetAttribute(&per_sm, cudaDevAttrMaxSharedMemoryPerMultiprocessor, device) != cudaSuccess ||
         cudaDeviceGetAttribute(&reserved, cudaDevAttrReservedSharedMemoryPerBlock, device) != cudaSuccess) {
         cudaGetLastError();
@@ -605,28 +606,24 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
         return 1024 + wb + slots * npad * 128 + h_bytes + op_bytes + w2s_bytes;
     };
     if (configure_tc(dev.device) != BP_OK) return BP_ERR_CUDA;
-    // ring: the deepest configuration (two atoms per stage, 256-byte row fetches, first) under which
-    // every cluster of the grid is resident at once -- a cluster left for a second wave streams its
-    // tile alone at a fraction of the bandwidth (measured at 32 requests x 151936 -> 2048: 16 tiles of
-    // 9-CTA clusters took 179 us at one CTA per SM, 125 us at two); if none, the deepest that fits
-    int stages = kTcStages, aps = 1;
+    // ring: the deepest under which every cluster of the grid is resident at once -- a cluster left for
+    // a second wave streams its tile alone at a fraction of the bandwidth (measured at 64 requests x
+    // 151936 -> 2048: 16 tiles of 9-CTA clusters took 200 us with the 5-stage ring at one CTA per SM);
+    // if none, the deepest that fits
+    int kernel = 0;  // index into kTcKernels
     if (ring) {
-        const int tries[7][2] = {{4, 2}, {3, 2}, {2, 2}, {5, 1}, {4, 1}, {3, 1}, {2, 1}};
-        int pick = -1;
-        for (int i = 0; i < 7; ++i) {
-            const int sm = smem_for(tries[i][0] * tries[i][1]);
+        for (int i = 1; i <= kTcRings; ++i) {
+            const int sm = smem_for(kTcKernels[i].stages);
             if (sm > kTcMaxSmem) continue;
-            if (pick < 0) pick = i;
+            if (kernel == 0) kernel = i;
             if (active_ring_clusters(dev.device, ks, sm) >= tiles * groups) {
-                pick = i;
+                kernel = i;
                 break;
             }
         }
-        if (pick < 0) return -1;
-        stages = tries[pick][0];
-        aps = tries[pick][1];
+        if (kernel == 0) return -1;
     }
-    const int slots = ring ? stages * aps : per;
+    const int slots = ring ? kTcKernels[kernel].stages : per;
     const int w_bytes = slots * kTcAtomBytes > pd_bytes ? slots * kTcAtomBytes : pd_bytes;
     const int x_bytes = slots * npad * 128;
     const int smem = smem_for(slots);
@@ -663,8 +660,6 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     p.x_bytes = x_bytes;
     p.h_bytes = h_bytes;
     p.op_bytes = op_bytes;
-    p.stages = stages;
-    p.aps = aps;
     p.b1 = a.b1;
     p.w2 = static_cast<const __nv_bfloat16*>(a.w2);
     p.b2 = a.b2;
@@ -704,8 +699,7 @@ int run_tc(const PolicyArgs& a, const DeviceInfo& dev, float* part, int* counter
     attr[1] = pdl[0];
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    const cudaError_t e = ring ? cudaLaunchKernelEx(&cfg, policy_tc_kernel<true>, w1map, xmap, p)
-                               : cudaLaunchKernelEx(&cfg, policy_tc_kernel<false>, w1map, xmap, p);
+    const cudaError_t e = cudaLaunchKernelEx(&cfg, kTcKernels[kernel].fn, w1map, xmap, p);
     return e == cudaSuccess ? BP_OK : BP_ERR_CUDA;
 }
 

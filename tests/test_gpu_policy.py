@@ -80,6 +80,6 @@ def test_d_in_tail_and_two_request_groups(d_in):
     # d_in is not a multiple of 64 (the last atom is zero-filled), 70 requests span two groups of 64
     # (the second only partly filled) and hidden = 300 leaves the last W1 tile partial.  Split over
     # 9 CTAs per tile, d_in = 4104 (65 atoms, 8 per CTA) is loaded at once; d_in = 5160 (81 atoms, 9
-    # per CTA) streams through the ring, two atoms per stage, so every CTA ends on a half-filled stage.
+    # per CTA) streams through the ring and wraps around it.
     w = wl.custom(seed=7, policy=dict(num_reqs=70, d_in=d_in, hidden=300, wdtype="bf16", feat_std=1.0))
     _compare(wl.policy_inputs(w))
