@@ -58,6 +58,29 @@ def test_workspace_sizes(lib):
     assert lib.bp_spec_accept_workspace_size(-1, 0, 10) == 0
 
 
+def _align(x, a=256):
+    return (x + a - 1) // a * a
+
+
+@pytest.mark.parametrize("s,td,vocab", [(1, 15, 151936), (1, 16, 151936), (4, 60, 32000), (5, 75, 32000),
+                                        (2, 23, 151936), (3, 23, 151936), (1, 0, 5), (32, 470, 151936),
+                                        (200000, 200000, 16), (9, 100, 16385)])
+def test_acceptance_workspace_follows_the_path_choice(lib, s, td, vocab):
+    """The workspace carries the throughput kernels' regions (chunk and row statistics, draw records,
+    chunk totals, segment masses) exactly when either temperature takes those kernels: this pins the
+    tests' mirror of the library's choice (accept_uses_batch) to the library, on the CPU."""
+    from _gpu import accept_uses_batch
+
+    blocks = (td + 1,) + (1,) * (s - 1)
+    cluster = 256 + _align(4 * s) + _align(4 * td) + _align(4 * (td + s))
+    chunks = -(-vocab // 16384)
+    rows = 2 * td + s
+    batch = (_align(rows * chunks * 8) + _align(rows * 8) + _align(s * 32) + _align(s * chunks * 16)
+             + _align(s * chunks * 256 * 8 if chunks > 1 else 0))
+    may = accept_uses_batch(blocks, vocab, 0.0) or accept_uses_batch(blocks, vocab, 1.0)
+    assert bp.spec_accept_workspace_size(s, td, vocab) == cluster + (batch if may else 0)
+
+
 def test_host_validation_needs_no_gpu(lib):
     vp = ctypes.c_void_p
     fake = vp(0x10000)
