@@ -480,6 +480,25 @@ def run_ours(args):
     t_racc0 = time_calls(batch_accept(0.0), n_graph=4, reps=10)
     del r_copies
 
+    # a3 at the drafter's own configuration: 16 sequences of 4096 context keys and a 16-position block of
+    # mask-token queries, bidirectional within the block (269 MB of K/V, larger than L2), drawn on the device
+    dw = wl.get("drafter_bidir")
+    d_kv = np.asarray(dw.ctx) + np.asarray(dw.block)
+    d_cu_q, d_cu_kv = t(wl.offsets(dw.block)), t(wl.offsets(d_kv))
+    d_q = torch.randn(int(np.sum(dw.block)), dw.num_q_heads, dw.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+    d_k = torch.randn(int(d_kv.sum()), dw.num_kv_heads, dw.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+    d_v = torch.randn(int(d_kv.sum()), dw.num_kv_heads, dw.head_dim, device=dev, generator=gen).to(torch.bfloat16)
+    d_o = torch.empty_like(d_q)
+    ws_d = bp.workspace(bp.block_attention_workspace_size(dw.num_seqs, int(max(dw.block)), dw.num_q_heads,
+                                                          dw.num_kv_heads, dw.head_dim), dev)
+
+    def drafter_attn(_c):
+        bp.block_attention(d_q, d_k, d_v, d_cu_q, d_cu_kv, int(max(dw.block)), int(d_kv.max()), mask=bp.MASK_BIDIR,
+                           out=d_o, ws=ws_d, stream=stream)
+
+    t_drafter = time_calls(drafter_attn, n_graph=4, reps=10)
+    del d_q, d_k, d_v, d_o
+
     def row(tsec, nbytes, kernels):
         gbs = nbytes / tsec / 1e9
         return {"us": round(tsec * 1e6, 3), "bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
@@ -488,6 +507,7 @@ def run_ours(args):
     rows = {
         "a2_a4_verify_attention_causal": row(t_attn, attention_bytes(w), ["attn_bf16_tc_kernel"]),
         "a3_drafter_attention_bidir": row(t_bidir, attention_bytes(w), ["attn_bf16_tc_kernel"]),
+        "a3_drafter_attention_bidir_16x4112": row(t_drafter, attention_bytes(dw), ["attn_bf16_tc_kernel"]),
         "a5_a6_accept_t1": row(t_acc, accept_bytes(w, 1.0), ["accept_kernel<false,true>"]),
         "a7_accept_greedy_t0": row(t_acc0, accept_bytes(w, 0.0), ["accept_kernel<true,true>"]),
         "a1_policy_head_32req_2560x2048": row(t_pol, policy_bytes(pin), ["policy_tc_kernel"]),
