@@ -25,6 +25,8 @@
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "ptx_sm103.cuh"
 
@@ -717,12 +719,17 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     p.err = a.err_word;
     if (!q_tma) qmap = kmap;  // unused by the kernel
 
-    // once per device: opt in to the shared-memory size and non-portable clusters, and record how
-    // many clusters of each size (1..16) the GPU can keep resident at once (queried outside any
-    // graph capture; the answer reflects how the SMs are grouped into GPCs)
-    static int configured_device = -1;
-    static int max_active[kMaxCluster + 1];
-    if (configured_device != dev.device) {
+    // once per device (under a lock: calls may come from several host threads): opt in to the
+    // shared-memory size and non-portable clusters, and record how many clusters of each size (1..16)
+    // the GPU can keep resident at once (queried outside any graph capture; the answer reflects how
+    // the SMs are grouped into GPCs)
+    static std::mutex cfg_mu;
+    static bool configured[64] = {};
+    static int max_active_dev[64][kMaxCluster + 1];
+    if (dev.device < 0 || dev.device >= 64) return BP_ERR_UNSUPPORTED;
+    int max_active[kMaxCluster + 1];
+    std::unique_lock<std::mutex> cfg_lock(cfg_mu);
+    if (!configured[dev.device]) {
         for (auto kern : {attn_bf16_tc_kernel<false, false>, attn_bf16_tc_kernel<true, false>,
                           attn_bf16_tc_kernel<false, true>, attn_bf16_tc_kernel<true, true>})
             if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) != cudaSuccess ||
@@ -748,10 +755,12 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
                 cudaGetLastError();
                 n_clusters = 0;
             }
-            max_active[cs] = n_clusters;
+            max_active_dev[dev.device][cs] = n_clusters;
         }
-        configured_device = dev.device;
+        configured[dev.device] = true;
     }
+    for (int c = 0; c <= kMaxCluster; ++c) max_active[c] = max_active_dev[dev.device][c];
+    cfg_lock.unlock();
     // cluster size: the largest split of each unit's keys for which every unit's cluster is resident
     // in the same wave (a unit left for a second wave would double the time)
     // (the tiles of the longest unit per CTA set the time: minimise them, then prefer the smallest

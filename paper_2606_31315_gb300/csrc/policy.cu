@@ -711,10 +711,12 @@ int run(const PolicyArgs& a, cudaStream_t stream) {
     const int group = max_group < kGroup ? max_group : kGroup;
     const int rows_per_block = (kThreads1 / 32) * kRowsPerWarp;
     const unsigned blocks = (unsigned)((a.hidden + rows_per_block - 1) / rows_per_block);
-    static int configured = -1;
+    static std::mutex cfg_mu;
+    static bool configured[64] = {};
     int dev = 0;
-    cudaGetDevice(&dev);
-    if (configured != dev) {
+    if (cudaGetDevice(&dev) != cudaSuccess || dev < 0 || dev >= 64) return BP_ERR_CUDA;
+    std::lock_guard<std::mutex> cfg_lock(cfg_mu);  // once per device, from any host thread
+    if (!configured[dev]) {
         if (cudaFuncSetAttribute(policy_hidden_kernel<T>, cudaFuncAttributeMaxDynamicSharedMemorySize, kSmemBudget) !=
                 cudaSuccess ||
             cudaFuncSetAttribute(policy_hidden_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -722,7 +724,7 @@ int run(const PolicyArgs& a, cudaStream_t stream) {
             cudaFuncSetAttribute(policy_out_kernel<T>, cudaFuncAttributePreferredSharedMemoryCarveout,
                                  cudaSharedmemCarveoutMaxShared) != cudaSuccess)
             return BP_ERR_CUDA;
-        configured = dev;
+        configured[dev] = true;
     }
     cudaLaunchAttribute attr[1];
     attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;

@@ -17,6 +17,8 @@
 #include <cuda_runtime.h>
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 
 namespace bp {
@@ -232,13 +234,18 @@ size_t tau_smem_bytes(int JM, int NCB, int jmax, int nc) {
 
 template <int JM, int NCB>
 int tau_launch(const TauArgs& a, const TauParams& p, const DeviceInfo& dev, cudaStream_t stream) {
+    static std::mutex cfg_mu;
     static int configured[64] = {};
     if (dev.device < 0 || dev.device >= 64) return BP_ERR_UNSUPPORTED;
-    if (!configured[dev.device]) {
-        const int most = (int)tau_smem_bytes(JM, NCB, kTauMaxJ, kTauMaxCand);
-        if (cudaFuncSetAttribute(tau_kernel<JM, NCB>, cudaFuncAttributeMaxDynamicSharedMemorySize, most) != cudaSuccess)
-            return BP_ERR_CUDA;
-        configured[dev.device] = 1;
+    {
+        std::lock_guard<std::mutex> cfg_lock(cfg_mu);  // once per device, from any host thread
+        if (!configured[dev.device]) {
+            const int most = (int)tau_smem_bytes(JM, NCB, kTauMaxJ, kTauMaxCand);
+            if (cudaFuncSetAttribute(tau_kernel<JM, NCB>, cudaFuncAttributeMaxDynamicSharedMemorySize, most) !=
+                cudaSuccess)
+                return BP_ERR_CUDA;
+            configured[dev.device] = 1;
+        }
     }
     // the table: r_c = exp(-alpha (b_c - B)^2) and its powers as running products
     TauTable<JM, NCB> tab;

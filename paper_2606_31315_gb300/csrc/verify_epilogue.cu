@@ -34,6 +34,8 @@
 #include <limits.h>
 #include <math.h>
 
+#include <mutex>
+
 #include "common.cuh"
 #include "ptx_sm103.cuh"
 #include "softmax_math.cuh"
@@ -741,18 +743,22 @@ VeLayout ve_layout(int num_seqs, int total_draft) {
 
 template <bool GREEDY, int NP, int APS>
 int ve_launch(const CUtensorMap& wmap, const VeParams& p, int grid, const DeviceInfo& dev, cudaStream_t stream) {
-    static int configured[64] = {};  // per instantiation (a template's own static)
+    static std::mutex cfg_mu;        // per instantiation (a template's own statics)
+    static int configured[64] = {};
     const size_t smem = ve_smem_bytes<NP, APS>();
-    if (dev.device >= 0 && dev.device < 64 && !configured[dev.device]) {
-        if (cudaFuncSetAttribute(verify_epilogue_kernel<GREEDY, NP, APS>, cudaFuncAttributeMaxDynamicSharedMemorySize,
-                                 (int)smem) != cudaSuccess)
-            return BP_ERR_CUDA;
-        int per_sm = 0;
-        if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, verify_epilogue_kernel<GREEDY, NP, APS>, kVeThreads,
-                                                          smem) != cudaSuccess ||
-            per_sm < 1)
-            return BP_ERR_UNSUPPORTED;
-        configured[dev.device] = 1;
+    if (dev.device >= 0 && dev.device < 64) {
+        std::lock_guard<std::mutex> cfg_lock(cfg_mu);  // once per device, from any host thread
+        if (!configured[dev.device]) {
+            if (cudaFuncSetAttribute(verify_epilogue_kernel<GREEDY, NP, APS>,
+                                     cudaFuncAttributeMaxDynamicSharedMemorySize, (int)smem) != cudaSuccess)
+                return BP_ERR_CUDA;
+            int per_sm = 0;
+            if (cudaOccupancyMaxActiveBlocksPerMultiprocessor(&per_sm, verify_epilogue_kernel<GREEDY, NP, APS>,
+                                                              kVeThreads, smem) != cudaSuccess ||
+                per_sm < 1)
+                return BP_ERR_UNSUPPORTED;
+            configured[dev.device] = 1;
+        }
     }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3((unsigned)grid);
