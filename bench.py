@@ -504,6 +504,65 @@ def run_ours(args):
         return {"us": round(tsec * 1e6, 3), "bytes": nbytes, "gbs": round(gbs, 1), "frac": round(gbs / peak, 4),
                 "kernels": kernels}
 
+    def batch_step(wname):
+        """A whole verify step of a batch workload: causal verify attention, then the T=1 acceptance, on
+        2 rotating input copies drawn on the device (each step's inputs exceed L2); verified tokens/s,
+        requests/s and the step's fraction of the HBM roofline."""
+        sw = wl.get(wname)
+        blocks = np.asarray(sw.block)
+        kv = np.asarray(sw.ctx) + blocks
+        gam = blocks - 1
+        ns, ntd = sw.num_seqs, int(gam.sum())
+        cu_q_b, cu_kv_b, cu_d_b = t(wl.offsets(blocks)), t(wl.offsets(kv)), t(wl.offsets(gam))
+        trow = t((np.arange(ntd) + np.repeat(np.arange(ns), gam)).astype(np.int64))
+        hd, hq, hkv = sw.head_dim, sw.num_q_heads, sw.num_kv_heads
+        cs = []
+        for _ in range(2):
+            c = dict(q=torch.randn(int(blocks.sum()), hq, hd, device=dev, generator=gen).to(torch.bfloat16),
+                     k=torch.randn(int(kv.sum()), hkv, hd, device=dev, generator=gen).to(torch.bfloat16),
+                     v=torch.randn(int(kv.sum()), hkv, hd, device=dev, generator=gen).to(torch.bfloat16),
+                     target=torch.randn(ntd + ns, sw.vocab, device=dev, generator=gen) * sw.logit_std,
+                     ua=torch.rand(ntd, device=dev, generator=gen), us=torch.rand(ns, device=dev, generator=gen))
+            c["o"] = torch.empty_like(c["q"])
+            c["draft"] = c["target"][trow] + torch.randn(ntd, sw.vocab, device=dev, generator=gen)
+            ex = torch.empty_like(c["draft"]).exponential_(generator=gen)  # -log(E), E ~ Exp(1): Gumbel
+            c["tok"] = torch.argmax(c["draft"] - torch.log(ex), dim=1).to(torch.int32)
+            del ex
+            cs.append(c)
+        ws_at = bp.workspace(bp.block_attention_workspace_size(ns, int(blocks.max()), hq, hkv, hd), dev)
+        ws_ac = bp.workspace(bp.spec_accept_workspace_size(ns, ntd, sw.vocab), dev)
+        n_b = torch.empty(ns, dtype=torch.int32, device=dev)
+        o_b = torch.empty(ntd + ns, dtype=torch.int32, device=dev)
+        turn = [0]
+
+        def go(_c):
+            c = cs[turn[0] % len(cs)]
+            turn[0] += 1
+            bp.block_attention(c["q"], c["k"], c["v"], cu_q_b, cu_kv_b, int(blocks.max()), int(kv.max()), out=c["o"],
+                               ws=ws_at, stream=stream)
+            bp.spec_accept(c["target"], c["draft"], c["tok"], cu_d_b, 1.0, c["ua"], c["us"], n_accepted=n_b,
+                           out_tokens=o_b, want_accept_prob=False, ws=ws_ac, stream=stream)
+
+        tsec = time_calls(go, n_graph=4, reps=5)
+        nbytes = attention_bytes(sw) + accept_bytes(sw, 1.0)
+        tokens = int(blocks.sum())
+        del cs
+        out = row(tsec, nbytes, ["attn_bf16_tc_kernel", "batch_stats_kernel", "batch_decide_kernel",
+                                 "batch_draw_kernel"])
+        out.update(verified_tokens_per_s=round(tokens / tsec, 1), requests_per_s=round(ns / tsec, 1),
+                   roofline_tokens_per_s=round(tokens / (nbytes / (peak * 1e9)), 1),
+                   workload=f"{ns} sequences, {tokens} block positions, contexts {min(sw.ctx)}-{max(sw.ctx)}, "
+                            f"vocab {sw.vocab}, T=1")
+        return out
+
+    steps_rows = {}
+    for key, wname in (("c3_step_ragged_32req_attention_accept_t1", "ragged"),
+                       ("c5_step_long_context_8x32768_attention_accept_t1", "long_context")):
+        try:  # a row that fails reports its error; the rest of the line stands
+            steps_rows[key] = batch_step(wname)
+        except Exception as exc:  # noqa: BLE001
+            steps_rows[key] = {"error": f"{type(exc).__name__}: {exc}"}
+
     rows = {
         "a2_a4_verify_attention_causal": row(t_attn, attention_bytes(w), ["attn_bf16_tc_kernel"]),
         "a3_drafter_attention_bidir": row(t_bidir, attention_bytes(w), ["attn_bf16_tc_kernel"]),
@@ -531,6 +590,7 @@ def run_ours(args):
             traffic=committed_traffic("batch_stats_kernel")),
         "a7_accept_greedy_t0_batch_ragged_32req": row(t_racc0, accept_bytes(rw, 0.0),
                                                       ["batch_stats_kernel<true,true>", "batch_decide_kernel<true>"]),
+        **steps_rows,
         "next4_tau_model_4M_requests": dict(row(t_tau, tau_bytes, ["tau_kernel<24,9>", "tau_finish_kernel"]),
                                             traffic=committed_traffic("tau_kernel")),
     }
