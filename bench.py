@@ -615,7 +615,9 @@ def run_ours(args):
                    "graph": f"CUDA graph of {COPIES} steps"},
         "hbm_roofline": {"step_bytes": step_bytes, "achieved_gbs": round(step_bytes / (elapsed / args.steps) / 1e9, 1),
                          "peak": peak, "frac": round(step_bytes / (elapsed / args.steps) / 1e9 / peak, 4),
-                         "roofline_tokens_per_s": round(tokens_per_step / (step_bytes / (peak * 1e9)), 1)},
+                         "roofline_tokens_per_s": round(tokens_per_step / (step_bytes / (peak * 1e9)), 1),
+                         "requests_per_s": round(job_throughput(w.num_seqs, args.steps, elapsed, world), 1),
+                         "roofline_requests_per_s": round(w.num_seqs / (step_bytes / (peak * 1e9)), 1)},
         "roofline": roofline,
         "rows": rows,
         "e2e": e2e,
