@@ -70,3 +70,23 @@ def test_reference_arm_runs_on_rank_0_only():
                           "--warmup", "0"], env=env, capture_output=True, text=True, timeout=300, cwd=ROOT)
     assert res.returncode == 0, res.stderr
     assert res.stdout.strip() == ""
+
+
+def test_reference_arm_prints_the_contract_line():
+    # rank 0 alone (no torchrun): the fp64 oracle timed on the host cores, one JSON line with the same
+    # metric, unit and config as the CUDA arm, the cpu_baseline describing this run, and an e2e of its own
+    res = subprocess.run([sys.executable, os.path.join(ROOT, "bench.py"), "--impl", "reference", "--steps", "1",
+                          "--warmup", "0"], capture_output=True, text=True, timeout=600, cwd=ROOT,
+                         env={k: v for k, v in os.environ.items() if k not in ("RANK", "WORLD_SIZE", "LOCAL_RANK")})
+    assert res.returncode == 0, res.stderr
+    lines = [ln for ln in res.stdout.splitlines() if ln.startswith("{")]
+    assert len(lines) == 1
+    d = json.loads(lines[0])
+    import bench
+
+    assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == "tokens/s"
+    assert d["higher_is_better"] is True and d["n_gpus"] == 1 and d["steps"] == 1 and d["value"] > 0
+    assert d["config"]["workload"].startswith("qwen3_4b")
+    cb = d["cpu_baseline"]
+    assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
+    assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
