@@ -217,3 +217,13 @@ def test_product_package_never_imports_the_oracle():
                         assert not (node.module or "").startswith("oracle"), path
             if f.endswith((".cu", ".cuh", ".h")):
                 assert "bpo_" not in open(path).read(), path
+
+
+def test_build_compiles_every_source():
+    """build() (the only build step on a fresh machine) compiles every CUDA source and tracks every
+    header of csrc/: a file left off the lists would silently be missing from the library."""
+    csrc = os.path.join(ROOT, "paper_2606_31315_gb300", "csrc")
+    on_disk = sorted(f for f in os.listdir(csrc) if f.endswith(".cu"))
+    headers = sorted(f for f in os.listdir(csrc) if f.endswith(".cuh"))
+    assert sorted(_build.SOURCES) == on_disk
+    assert sorted(_build.HEADERS) == headers
