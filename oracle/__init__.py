@@ -68,6 +68,8 @@ def _load():
         lib.bpo_verify_commit.restype = ctypes.c_int
         lib.bpo_num_threads.argtypes = []
         lib.bpo_num_threads.restype = ctypes.c_int
+        lib.bpo_set_num_threads.argtypes = [ctypes.c_int]
+        lib.bpo_set_num_threads.restype = None
         _lib = lib
     return _lib
 
@@ -87,6 +89,11 @@ def _p(a, ctype):
 def num_threads() -> int:
     """OpenMP threads the oracle's parallel loops use."""
     return int(_load().bpo_num_threads())
+
+
+def set_num_threads(n: int) -> None:
+    """Thread count of the oracle's parallel loops from now on (timing only; results do not change)."""
+    _load().bpo_set_num_threads(int(n))
 
 
 def block_attention(q, k, v, cu_q, cu_kv, num_kv_heads: int, mask: int, scale: float | None = None):

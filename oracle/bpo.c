@@ -579,6 +579,9 @@ int bpo_verify_commit(int32_t *ctx, const int32_t *n_acc, const int32_t *out_tok
 #ifdef _OPENMP
 #include <omp.h>
 int bpo_num_threads(void) { return omp_get_max_threads(); }
+/* Sets the thread count of the following parallel loops (n >= 1); no effect on any result. */
+void bpo_set_num_threads(int n) { if (n >= 1) omp_set_num_threads(n); }
 #else
 int bpo_num_threads(void) { return 1; }
+void bpo_set_num_threads(int n) { (void)n; }
 #endif

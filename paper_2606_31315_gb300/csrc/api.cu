@@ -93,8 +93,10 @@ const char* bp_error_string(int status) {
 
 size_t bp_block_attention_workspace_size(int num_seqs, int max_q_len, int num_q_heads, int num_kv_heads,
                                          int head_dim) {
-    (void)num_seqs; (void)max_q_len; (void)num_q_heads; (void)num_kv_heads; (void)head_dim;
-    return sizeof(WorkspaceHeader);
+    (void)num_seqs; (void)head_dim;
+    if (max_q_len < 1 || num_q_heads < 1 || num_kv_heads < 1 || num_q_heads % num_kv_heads != 0)
+        return sizeof(WorkspaceHeader);
+    return sizeof(WorkspaceHeader) + attention_flat_scratch_bytes(max_q_len, num_q_heads / num_kv_heads);
 }
 
 int bp_block_attention(const void* q, const void* k, const void* v, void* o, float* lse, const int32_t* cu_q,
@@ -115,9 +117,9 @@ int bp_block_attention(const void* q, const void* k, const void* v, void* o, flo
     if (dtype == BP_F32 && head_dim > 128) return BP_ERR_UNSUPPORTED;
     if (dtype == BP_BF16 && (!aligned(q, 16) || !aligned(k, 16) || !aligned(v, 16) || !aligned(o, 16)))
         return BP_ERR_INVALID_ARG;
-    int rc = check_workspace(workspace, workspace_bytes,
-                             bp_block_attention_workspace_size(num_seqs, max_q_len, num_q_heads, num_kv_heads,
-                                                               head_dim));
+    // the header is the minimum; a workspace of bp_block_attention_workspace_size bytes also holds the
+    // flat split's partial slots (a smaller one keeps the cluster split)
+    int rc = check_workspace(workspace, workspace_bytes, sizeof(WorkspaceHeader));
     if (rc != BP_OK) return rc;
     DeviceInfo dev;
     if ((rc = device_info(&dev)) != BP_OK) return rc;
@@ -131,6 +133,8 @@ int bp_block_attention(const void* q, const void* k, const void* v, void* o, flo
     a.err_word = err_word(workspace);
     a.block_table = nullptr;
     a.pages_per_seq = a.page_size = a.num_pages = 0;
+    a.scratch = scratch(workspace);
+    a.scratch_bytes = workspace_bytes - sizeof(WorkspaceHeader);
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     rc = dtype == BP_BF16 ? launch_attention_bf16(a, dev, st) : launch_attention_f32(a, st);
     if (rc == BP_ERR_CUDA) cudaGetLastError();
@@ -163,9 +167,9 @@ int bp_block_attention_paged(const void* q, const void* k_cache, const void* v_c
     if (max_q_len > 64) return BP_ERR_UNSUPPORTED;
     if (dtype != BP_BF16 || head_dim != 128) return BP_ERR_UNSUPPORTED;  // tensor-core path only
     if (!aligned(q, 16) || !aligned(k_cache, 16) || !aligned(v_cache, 16) || !aligned(o, 16)) return BP_ERR_INVALID_ARG;
-    int rc = check_workspace(workspace, workspace_bytes,
-                             bp_block_attention_workspace_size(num_seqs, max_q_len, num_q_heads, num_kv_heads,
-                                                               head_dim));
+    // the header is the minimum; a workspace of bp_block_attention_workspace_size bytes also holds the
+    // flat split's partial slots (a smaller one keeps the cluster split)
+    int rc = check_workspace(workspace, workspace_bytes, sizeof(WorkspaceHeader));
     if (rc != BP_OK) return rc;
     DeviceInfo dev;
     if ((rc = device_info(&dev)) != BP_OK) return rc;
@@ -181,6 +185,8 @@ int bp_block_attention_paged(const void* q, const void* k_cache, const void* v_c
     a.pages_per_seq = pages_per_seq;
     a.page_size = page_size;
     a.num_pages = num_pages;
+    a.scratch = scratch(workspace);
+    a.scratch_bytes = workspace_bytes - sizeof(WorkspaceHeader);
     rc = launch_attention_bf16(a, dev, static_cast<cudaStream_t>(stream));
     if (rc == BP_ERR_CUDA) cudaGetLastError();
     return rc;

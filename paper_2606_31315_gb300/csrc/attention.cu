@@ -25,6 +25,10 @@
 #include <cooperative_groups.h>
 #include <cuda_bf16.h>
 
+#include <stdlib.h>
+#include <string.h>
+
+#include <algorithm>
 #include <mutex>
 
 #include "common.cuh"
@@ -65,6 +69,12 @@ struct AttnParams {
     // at row j & (page size - 1); NULL block_table = contiguous K/V rows from cu_kv[s]
     const int32_t* block_table;
     int pages_per_seq, page_shift;
+    // flat split: partial (O, m, l) slots in the workspace, two per CTA, slot_rows rows each; and one
+    // work entry per CTA for the merge: (sequence, query tile, first tile, all tiles) of the cut unit
+    // whose first tile the CTA holds, or sequence -1
+    float* part;
+    int4* work;
+    int slot_rows;
     unsigned int* err;
 };
 constexpr int kMaxSub = kTileN / 16;  // sub-boxes per K/V tile at the smallest page size (16 keys)
@@ -88,13 +98,99 @@ __device__ __forceinline__ uint32_t cluster_size() {
     return r;
 }
 
+__device__ __forceinline__ int cdiv(int a, int b) { return (a + b - 1) / b; }
+
+// One stretch of consecutive 128-key tiles of one work unit (sequence s, KV head h, 128-row query
+// tile mt), processed by one CTA.
+struct Seg {
+    int s, h, mt;
+    int q0, B, kv0, n;  // the sequence's first query row, block size, first key row, key count
+    int jt0, nt;        // first tile of the stretch within the unit, tiles in it
+    int whole;          // flat split: the stretch is the whole unit (the CTA writes the output)
+    int slot;           // flat split, part of a unit: the CTA's partial slot (0 first stretch, 1 last)
+};
+
+// Flat split: key tiles of every sequence over its 128-row query tiles, counted once for all KV heads
+// (a group of CTAs, one per KV head, streams the same tiles of every head at the same time); a
+// sequence without block rows has none.
+__device__ __forceinline__ int flat_seq_tiles(int B, int n, int G) {
+    return B > 0 ? cdiv(B * G, kM) * cdiv(n, kTileN) : 0;
+}
+
+// Flat split: the prefix sums of the sequences' tile counts into pre[0..S] (S <= kMaxOrderedSeqs), by one
+// warp: each lane sums 8 consecutive sequences, then an exclusive scan of the lane sums.
+__device__ __forceinline__ void flat_prefix(const AttnParams& p, int32_t* pre, int lane) {
+    constexpr int kPer = (kMaxOrderedSeqs + 31) / 32;
+    int loc[kPer];
+    int run = 0;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+        const int s = lane * kPer + k;
+        if (s < p.num_seqs) {
+            const int B = __ldg(p.cu_q + s + 1) - __ldg(p.cu_q + s);
+            const int n = __ldg(p.cu_kv + s + 1) - __ldg(p.cu_kv + s);
+            run += flat_seq_tiles(B, n, p.group);
+        }
+        loc[k] = run;
+    }
+    int incl = run;
+#pragma unroll
+    for (int o = 1; o < 32; o <<= 1) {
+        const int y = __shfl_up_sync(0xffffffffu, incl, o);
+        if (lane >= o) incl += y;
+    }
+    const int excl = incl - run;
+#pragma unroll
+    for (int k = 0; k < kPer; ++k) {
+        const int s = lane * kPer + k;
+        if (s < p.num_seqs) pre[s + 1] = excl + loc[k];
+    }
+    if (lane == 0) pre[0] = 0;
+}
+
+// Flat split: the stretch that starts at global tile t of a CTA (KV head h) whose range ends at t_end
+// (pre: the sequences' tile prefix sums; a single sequence needs none).  first: the CTA's first stretch.
+__device__ __forceinline__ Seg flat_seg(const AttnParams& p, const int32_t* pre, int t, int t_end, int h, bool first) {
+    Seg g;
+    int s = 0;
+    if (p.num_seqs > 1) {  // the last sequence whose tiles start at or before t
+        int lo = 0, hi = p.num_seqs;
+        while (hi - lo > 1) {
+            const int mid = (lo + hi) >> 1;
+            if (pre[mid] <= t) lo = mid; else hi = mid;
+        }
+        s = lo;
+    }
+    const int base = p.num_seqs > 1 ? pre[s] : 0;
+    g.s = s;
+    g.q0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_q + s);
+    g.B = p.num_seqs == 1 ? p.total_q : __ldg(p.cu_q + s + 1) - g.q0;
+    g.kv0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_kv + s);
+    g.n = p.num_seqs == 1 ? p.total_kv : __ldg(p.cu_kv + s + 1) - g.kv0;
+    const int ntu = cdiv(g.n, kTileN);
+    const int local = t - base;
+    g.mt = local / ntu;
+    g.jt0 = local - g.mt * ntu;
+    g.h = h;
+    g.nt = min(ntu - g.jt0, t_end - t);
+    g.whole = g.jt0 == 0 && g.nt == ntu;
+    g.slot = first ? 0 : 1;
+    return g;
+}
+
 // PAGED: K/V rows come from pages named by p.block_table (the contiguous instantiation carries no
 // paging code at all).
 // SPREAD (units of at most 64 query rows, group size dividing 16): logical row r sits at TMEM lane
 // (r / 16) * 32 + r % 16, so the 64 rows fill 16 lanes of each of the four TMEM sub-partitions and
 // all four softmax warps (and their SMSPs' exp2 units) work; the two half-warps take the two
 // 64-column halves of a row (tcgen05 16x32bx2 accesses), combining row statistics by shuffle.
-template <bool PAGED, bool SPREAD>
+// FLAT: the flat split.  The key tiles of all units, in order, are cut into gridDim.x equal ranges,
+// one per CTA (no clusters); a CTA works through the stretches of its range one after another with
+// one pipeline (K/V ring, S double buffer, O accumulator) and writes a unit it covers whole straight
+// to the output, a partial stretch to its workspace slot for attn_combine_kernel.  Otherwise the
+// cluster split: a unit per cluster, its tiles cut into CS ranges, partials merged through
+// distributed shared memory.
+template <bool PAGED, bool SPREAD, bool FLAT>
 __global__ void __launch_bounds__(kThreads, 1)
     attn_bf16_tc_kernel(const __grid_constant__ CUtensorMap qmap, const __grid_constant__ CUtensorMap kmap,
                         const __grid_constant__ CUtensorMap vmap, const AttnParams p) {
@@ -104,10 +200,11 @@ __global__ void __launch_bounds__(kThreads, 1)
     uint8_t* sKV = smem + kQBytes;  // stage s: K at s*64KB, V at s*64KB + 32KB
 
     __shared__ uint64_t bar_kv_full[kStages], bar_kv_empty[kStages];
-    __shared__ uint64_t bar_s_full[2], bar_p_full[2], bar_pv_done[2], bar_o_done, bar_q_full;
+    __shared__ uint64_t bar_s_full[2], bar_p_full[2], bar_pv_done[2], bar_o_done, bar_q_full, bar_q_empty;
     __shared__ uint32_t tmem_base_sh;
     __shared__ int unit_seq_sh;
-    __shared__ int32_t cu_kv_sh[kMaxOrderedSeqs + 1];
+    // cluster split: the sequences' key offsets (longest-first order); flat split: their tile prefix sums
+    __shared__ int32_t seq_sh[kMaxOrderedSeqs + 1];
 
     const int tid = threadIdx.x;
     const int warp = tid >> 5, lane = tid & 31;
@@ -118,83 +215,106 @@ __global__ void __launch_bounds__(kThreads, 1)
     }
     griddep_launch_dependents();
     if (p.num_seqs > 1) griddep_wait();  // the sequence offsets are read from global memory
-    const uint32_t CS = cluster_size();
-    const uint32_t crank = cluster_rank();
-    const int unit_rank = blockIdx.x / CS;
     const int G = p.group;
-    const int units_per_seq = p.num_kv_heads * p.m_tiles;
-    const int seq_rank = unit_rank / units_per_seq;
-    const int h = (unit_rank / p.m_tiles) % p.num_kv_heads;
-    const int mt = unit_rank % p.m_tiles;
+    const uint32_t CS = FLAT ? 1u : cluster_size();
+    const uint32_t crank = FLAT ? 0u : cluster_rank();
 
-    // ---- which sequence: the seq_rank-th longest (ties by index) for small batches
-    int s;
-    if (p.num_seqs == 1) {
-        s = 0;
-    } else if (p.num_seqs <= kMaxOrderedSeqs) {
-        for (int t = tid; t <= p.num_seqs; t += kThreads) cu_kv_sh[t] = p.cu_kv[t];
-        __syncthreads();
-        for (int t = tid; t < p.num_seqs; t += kThreads) {
-            const int len = cu_kv_sh[t + 1] - cu_kv_sh[t];
-            int rank = 0;
-            for (int u = 0; u < p.num_seqs; ++u) {
-                const int lu = cu_kv_sh[u + 1] - cu_kv_sh[u];
-                rank += (lu > len) || (lu == len && u < t);
-            }
-            if (rank == seq_rank) unit_seq_sh = t;
+    // ---- work assignment.  Flat split: global tiles [t_lo, t_hi).  Cluster split: one stretch, `one`.
+    int t_lo = 0, t_hi = 0, T = 0;
+    Seg one{};
+    if (FLAT) {
+        if (p.num_seqs > 1) {
+            if (warp == 0) flat_prefix(p, seq_sh, lane);
+            __syncthreads();
+            T = seq_sh[p.num_seqs];
+        } else {
+            T = flat_seq_tiles(p.total_q, p.total_kv, G);
         }
-        __syncthreads();
-        s = unit_seq_sh;
+        // CTAs come in groups of one per KV head; group j has tiles [t_lo, t_hi) of every head
+        const int ngroups = gridDim.x / p.num_kv_heads, grp = blockIdx.x / p.num_kv_heads;
+        t_lo = (int)((long long)grp * T / ngroups);
+        t_hi = (int)((long long)(grp + 1) * T / ngroups);
     } else {
-        s = seq_rank;
+        const int unit_rank = blockIdx.x / CS;
+        const int units_per_seq = p.num_kv_heads * p.m_tiles;
+        const int seq_rank = unit_rank / units_per_seq;
+        one.h = (unit_rank / p.m_tiles) % p.num_kv_heads;
+        one.mt = unit_rank % p.m_tiles;
+        // which sequence: the seq_rank-th longest (ties by index) for small batches
+        int s;
+        if (p.num_seqs == 1) {
+            s = 0;
+        } else if (p.num_seqs <= kMaxOrderedSeqs) {
+            for (int t = tid; t <= p.num_seqs; t += kThreads) seq_sh[t] = p.cu_kv[t];
+            __syncthreads();
+            for (int t = tid; t < p.num_seqs; t += kThreads) {
+                const int len = seq_sh[t + 1] - seq_sh[t];
+                int rank = 0;
+                for (int u = 0; u < p.num_seqs; ++u) {
+                    const int lu = seq_sh[u + 1] - seq_sh[u];
+                    rank += (lu > len) || (lu == len && u < t);
+                }
+                if (rank == seq_rank) unit_seq_sh = t;
+            }
+            __syncthreads();
+            s = unit_seq_sh;
+        } else {
+            s = seq_rank;
+        }
+        one.s = s;
+        // a single sequence starts at offset 0 (cu_*[0] = 0) and spans the whole tensors: no loads
+        one.q0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_q + s);
+        one.B = p.num_seqs == 1 ? p.total_q : __ldg(p.cu_q + s + 1) - one.q0;
+        one.kv0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_kv + s);
+        one.n = p.num_seqs == 1 ? p.total_kv : __ldg(p.cu_kv + s + 1) - one.kv0;
+        if (one.B * G - one.mt * kM <= 0) {  // uniform across the cluster: every CTA decodes the same unit
+            griddep_wait();  // this grid must not complete before the one it depends on
+            return;
+        }
+        const int tiles = cdiv(one.n, kTileN);
+        one.jt0 = (int)((long long)crank * tiles / CS);
+        one.nt = (int)((long long)(crank + 1) * tiles / CS) - one.jt0;
+        one.whole = 0;
+        one.slot = 0;
     }
-    // a single sequence starts at offset 0 (cu_*[0] = 0) and spans the whole tensors: no loads
-    const int q0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_q + s);
-    const int B = p.num_seqs == 1 ? p.total_q : __ldg(p.cu_q + s + 1) - q0;
-    const int kv0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_kv + s);
-    const int n = p.num_seqs == 1 ? p.total_kv : __ldg(p.cu_kv + s + 1) - kv0;
-    const int L = n - B;
-    const int rows = B * G;
-    const int row0 = mt * kM;
-    const int m_valid = min(kM, rows - row0);
-    if (m_valid <= 0) {  // uniform across the cluster: every CTA decodes the same unit
-        griddep_wait();  // this grid must not complete before the one it depends on
-        return;
-    }
-
-    const int tiles = (n + kTileN - 1) / kTileN;
-    const int t_begin = (int)((long long)crank * tiles / CS);
-    const int t_end = (int)((long long)(crank + 1) * tiles / CS);
-    const int nt = t_end - t_begin;
+    // The stretches of this CTA, in order: `first` is the CTA's first one; t advances past each.
+    auto seg_at = [&](int t, bool first) -> Seg {
+        return FLAT ? flat_seg(p, seq_sh, t, t_hi, (int)(blockIdx.x % p.num_kv_heads), first) : one;
+    };
+    const int t_begin = FLAT ? t_lo : 0;
+    const int t_end = FLAT ? t_hi : 1;
+    auto seg_len = [&](const Seg& g) { return FLAT ? g.nt : 1; };
 
     // ---- Q tile -> shared memory, SWIZZLE_128B K-major (two 64-column halves).  With a TMA map the
-    // 128/G block positions x G heads box lands exactly as rows r = i*G + j; otherwise plain loads.
-    if (!p.q_tma) {
+    // 128/G block positions x G heads box lands exactly as rows r = i*G + j; otherwise (cluster split
+    // only) plain loads.
+    if (!FLAT && !p.q_tma) {
         griddep_wait();
+        const int row0 = one.mt * kM, m_valid = min(kM, one.B * G - row0);
         for (int idx = tid; idx < kM * 16; idx += kThreads) {
             const int r = idx >> 4, ch = idx & 15;
             uint4 val = make_uint4(0, 0, 0, 0);
             if (r < m_valid) {
                 const int lr = row0 + r;
                 const int i = lr / G, j = lr % G;
-                val = *reinterpret_cast<const uint4*>(p.q + ((size_t)(q0 + i) * p.num_q_heads + h * G + j) * kD +
-                                                      ch * 8);
+                val = *reinterpret_cast<const uint4*>(p.q + ((size_t)(one.q0 + i) * p.num_q_heads + one.h * G + j) *
+                                                      kD + ch * 8);
             }
             const int half = ch >> 3, c8 = ch & 7;
             *reinterpret_cast<uint4*>(sQ + half * kHalf + r * 128 + ((c8 ^ (r & 7)) << 4)) = val;
         }
         fence_proxy_async_smem();
     }
-    // paged cache: the pool rows of tile j's sub-boxes (sub_rows keys each); keys past the end of
-    // the sequence read the rows of its last page (finite values the mask then drops)
+    // paged cache: the pool rows of a tile's sub-boxes (sub_rows keys each); keys past the end of the
+    // sequence read the rows of its last page (finite values the mask then drops)
     constexpr bool paged = PAGED;
     const int sub_rows = paged ? min(kTileN, 1 << p.page_shift) : kTileN;
     const int nsub = kTileN / sub_rows;
-    auto tile_rows = [&](int j, int (&row)[kMaxSub]) {
+    auto tile_rows = [&](const Seg& g, int jl, int (&row)[kMaxSub]) {
         if (!paged) return;
-        const int32_t* bt = p.block_table + (size_t)s * p.pages_per_seq;
-        const int last_page = max(0, (n - 1) >> p.page_shift);
-        const int key0 = (t_begin + j) * kTileN;
+        const int32_t* bt = p.block_table + (size_t)g.s * p.pages_per_seq;
+        const int last_page = max(0, (g.n - 1) >> p.page_shift);
+        const int key0 = (g.jt0 + jl) * kTileN;
 #pragma unroll
         for (int sb = 0; sb < kMaxSub; ++sb)
             if (sb < nsub) {
@@ -203,29 +323,47 @@ __global__ void __launch_bounds__(kThreads, 1)
                 row[sb] = __ldg(bt + pi) * (1 << p.page_shift) + (key & ((1 << p.page_shift) - 1));
             }
     };
-    // K/V tile j of this CTA's range -> ring stage j % kStages (producer thread only)
-    auto issue_kv = [&](int j, const int (&row)[kMaxSub]) {
-        const int st = j % kStages;
+    // K/V tile jl of stretch g -> ring stage J % kStages (J counts the CTA's tiles; producer thread only)
+    auto issue_kv = [&](int J, const Seg& g, int jl, const int (&row)[kMaxSub]) {
+        const int st = J % kStages;
         uint8_t* sK = sKV + st * kStageBytes;
         uint8_t* sV = sK + kKVBytes;
         mbar_arrive_expect_tx(&bar_kv_full[st], kStageBytes);
         if (!paged) {
-            const int key = kv0 + (t_begin + j) * kTileN;
-            tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, h, key);
-            tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, h, key);
-            tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, h, key);
-            tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, h, key);
+            const int key = g.kv0 + (g.jt0 + jl) * kTileN;
+            tma_load_3d(sK, &kmap, &bar_kv_full[st], 0, g.h, key);
+            tma_load_3d(sK + kHalf, &kmap, &bar_kv_full[st], 64, g.h, key);
+            tma_load_3d(sV, &vmap, &bar_kv_full[st], 0, g.h, key);
+            tma_load_3d(sV + kHalf, &vmap, &bar_kv_full[st], 64, g.h, key);
         } else {
 #pragma unroll
             for (int sb = 0; sb < kMaxSub; ++sb) {  // sub-box sb lands at row sb * sub_rows of the tile
                 if (sb < nsub) {
                     const int off = sb * sub_rows * 128;
-                    tma_load_3d(sK + off, &kmap, &bar_kv_full[st], 0, h, row[sb]);
-                    tma_load_3d(sK + kHalf + off, &kmap, &bar_kv_full[st], 64, h, row[sb]);
-                    tma_load_3d(sV + off, &vmap, &bar_kv_full[st], 0, h, row[sb]);
-                    tma_load_3d(sV + kHalf + off, &vmap, &bar_kv_full[st], 64, h, row[sb]);
+                    tma_load_3d(sK + off, &kmap, &bar_kv_full[st], 0, g.h, row[sb]);
+                    tma_load_3d(sK + kHalf + off, &kmap, &bar_kv_full[st], 64, g.h, row[sb]);
+                    tma_load_3d(sV + off, &vmap, &bar_kv_full[st], 0, g.h, row[sb]);
+                    tma_load_3d(sV + kHalf + off, &vmap, &bar_kv_full[st], 64, g.h, row[sb]);
                 }
             }
+        }
+    };
+    // the Q tile of stretch g (producer thread only)
+    auto issue_q = [&](const Seg& g) {
+        const int row0 = g.mt * kM;
+        if (SPREAD) {  // four boxes of 16 rows, at shared-memory rows 0, 32, 64, 96
+            mbar_arrive_expect_tx(&bar_q_full, kQBytes / 2);
+#pragma unroll
+            for (int qq = 0; qq < 4; ++qq) {
+                const int qrow = g.q0 + (row0 + 16 * qq) / G;
+                tma_load_3d(sQ + qq * 32 * 128, &qmap, &bar_q_full, 0, g.h * G, qrow);
+                tma_load_3d(sQ + kHalf + qq * 32 * 128, &qmap, &bar_q_full, 64, g.h * G, qrow);
+            }
+        } else {
+            mbar_arrive_expect_tx(&bar_q_full, kQBytes);
+            const int qrow = g.q0 + row0 / G;
+            tma_load_3d(sQ, &qmap, &bar_q_full, 0, g.h * G, qrow);
+            tma_load_3d(sQ + kHalf, &qmap, &bar_q_full, 64, g.h * G, qrow);
         }
     };
     if (tid == 0) {
@@ -240,6 +378,7 @@ __global__ void __launch_bounds__(kThreads, 1)
         }
         mbar_init(&bar_o_done, 1);
         mbar_init(&bar_q_full, 1);
+        mbar_init(&bar_q_empty, 1);
         fence_mbar_init();
     }
     if (warp == 1) {  // tensor memory is allocated (and released) by warp 1, in parallel
@@ -252,89 +391,99 @@ __global__ void __launch_bounds__(kThreads, 1)
     const uint32_t tmem = tmem_base_sh;
     // inputs may be produced by the previous kernel on the stream: wait for it before any global access
     griddep_wait();
-    if (tid == 0 && nt > 0) {  // the producer starts the Q load and fills the K/V ring
-        if (SPREAD) {  // four boxes of 16 rows, at shared-memory rows 0, 32, 64, 96
-            mbar_arrive_expect_tx(&bar_q_full, kQBytes / 2);
-#pragma unroll
-            for (int qq = 0; qq < 4; ++qq) {
-                const int qrow = q0 + (row0 + 16 * qq) / G;
-                tma_load_3d(sQ + qq * 32 * 128, &qmap, &bar_q_full, 0, h * G, qrow);
-                tma_load_3d(sQ + kHalf + qq * 32 * 128, &qmap, &bar_q_full, 64, h * G, qrow);
-            }
-        } else if (p.q_tma) {
-            mbar_arrive_expect_tx(&bar_q_full, kQBytes);
-            const int qrow = q0 + row0 / G;
-            tma_load_3d(sQ, &qmap, &bar_q_full, 0, h * G, qrow);
-            tma_load_3d(sQ + kHalf, &qmap, &bar_q_full, 64, h * G, qrow);
-        }
-        int rows0[kStages][kMaxSub];  // the first tiles' page lookups, all in flight together
-#pragma unroll
-        for (int j = 0; j < kStages; ++j)
-            if (j < nt) tile_rows(j, rows0[j]);
-#pragma unroll
-        for (int j = 0; j < kStages; ++j)
-            if (j < nt) issue_kv(j, rows0[j]);
-    }
 
     if (warp == 0) {
-        // ================= TMA producer
-        if (lane == 0 && nt > 0) {
-            int issued = min(nt, kStages);  // the prologue issued the first tiles
-            for (int j = kStages; j < nt; ++j) {
-                int rows[kMaxSub];
-                tile_rows(j, rows);  // page lookups in flight while the stage drains
-                if (!mbar_wait(&bar_kv_empty[j % kStages], ((j / kStages) - 1) & 1, kWaitBudget)) {
-                    raise_error(p.err, kErrTimeout);
-                    break;
+        // ================= TMA producer: the Q tile of each stretch, the K/V tiles through the ring
+        if (lane == 0) {
+            int J = 0, nq = 0;
+            bool ok = true;
+            for (int t = t_begin; t < t_end && ok;) {
+                const Seg g = seg_at(t, t == t_begin);
+                t += seg_len(g);
+                if (g.nt == 0) continue;
+                for (int jl = 0; jl < g.nt; ++jl, ++J) {
+                    int rows[kMaxSub];
+                    tile_rows(g, jl, rows);  // page lookups in flight while the stage drains
+                    if (J >= kStages &&
+                        !mbar_wait(&bar_kv_empty[J % kStages], ((J / kStages) - 1) & 1, kWaitBudget)) {
+                        ok = false;
+                        break;
+                    }
+                    issue_kv(J, g, jl, rows);
+                    if (jl == 0 && p.q_tma) {
+                        // the stretch's Q, once the MMAs of the previous stretch no longer read the buffer
+                        if (nq > 0 && !mbar_wait(&bar_q_empty, (nq - 1) & 1, kWaitBudget)) {
+                            ++J;
+                            ok = false;
+                            break;
+                        }
+                        issue_q(g);
+                        ++nq;
+                    }
                 }
-                issue_kv(j, rows);
-                ++issued;
             }
+            if (!ok) raise_error(p.err, kErrTimeout);
             // no copy may still be in flight when the CTA leaves
-            for (int j = max(0, issued - kStages); j < issued; ++j)
+            for (int j = max(0, J - kStages); j < J; ++j)
                 if (!mbar_wait(&bar_kv_full[j % kStages], (j / kStages) & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
-            if (p.q_tma && !mbar_wait(&bar_q_full, 0, kWaitBudget)) raise_error(p.err, kErrTimeout);
+            if (nq > 0 && !mbar_wait(&bar_q_full, (nq - 1) & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
         }
     } else if (warp == 1) {
         // ================= MMA issuer
-        if (lane == 0 && nt > 0) {
+        if (lane == 0) {
             const uint32_t id_s = idesc_bf16_f32(kM, kTileN, false, false);
             const uint32_t id_o = idesc_bf16_f32(kM, kD, false, true);
             const uint32_t q_addr = smem_addr(sQ);
-            bool ok = !p.q_tma || mbar_wait(&bar_q_full, 0, kWaitBudget);
-            auto issue_pv = [&](int j) {
-                const int sb = j & 1, st = j % kStages;
-                if (!mbar_wait(&bar_p_full[sb], (j >> 1) & 1, kWaitBudget)) return false;
+            int J = 0, nq = 0;
+            bool ok = true;
+            auto issue_pv = [&](int Jx, bool first) {
+                const int sb = Jx & 1, st = Jx % kStages;
+                if (!mbar_wait(&bar_p_full[sb], (Jx >> 1) & 1, kWaitBudget)) return false;
                 tc_fence_after();
                 const uint32_t v_addr = smem_addr(sKV + st * kStageBytes + kKVBytes);
                 for (int kk = 0; kk < kTileN / 16; ++kk) {
                     const uint64_t bdesc = smem_desc(v_addr + kk * 2048, kHalf, 1024, kSwizzle128B);
-                    umma_ts(tmem + kColO, tmem + col_s(sb) + kk * 8, bdesc, id_o, (j > 0 || kk > 0) ? 1u : 0u);
+                    umma_ts(tmem + kColO, tmem + col_s(sb) + kk * 8, bdesc, id_o, (!first || kk > 0) ? 1u : 0u);
                 }
                 umma_commit(&bar_pv_done[sb]);
                 umma_commit(&bar_kv_empty[st]);
                 return true;
             };
-            for (int j = 0; j < nt && ok; ++j) {
-                const int sb = j & 1, st = j % kStages;
-                if (!mbar_wait(&bar_kv_full[st], (j / kStages) & 1, kWaitBudget)) { ok = false; break; }
-                if (j >= 2 && !mbar_wait(&bar_pv_done[sb], ((j - 2) >> 1) & 1, kWaitBudget)) { ok = false; break; }
-                tc_fence_after();
-                const uint32_t k_addr = smem_addr(sKV + st * kStageBytes);
-                for (int kk = 0; kk < kD / 16; ++kk) {
-                    const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
-                    const uint64_t adesc = smem_desc(q_addr + off, 16, 1024, kSwizzle128B);
-                    const uint64_t bdesc = smem_desc(k_addr + off, 16, 1024, kSwizzle128B);
-                    umma_ss(tmem + col_s(sb), adesc, bdesc, id_s, kk > 0 ? 1u : 0u);
+            for (int t = t_begin; t < t_end && ok;) {
+                const Seg g = seg_at(t, t == t_begin);
+                t += seg_len(g);
+                if (g.nt == 0) continue;
+                if (p.q_tma && !mbar_wait(&bar_q_full, nq & 1, kWaitBudget)) {
+                    ok = false;
+                    break;
                 }
-                umma_commit(&bar_s_full[sb]);
-                if (j >= 1 && !issue_pv(j - 1)) { ok = false; break; }
+                for (int jl = 0; jl < g.nt; ++jl, ++J) {
+                    const int sb = J & 1, st = J % kStages;
+                    if (!mbar_wait(&bar_kv_full[st], (J / kStages) & 1, kWaitBudget)) { ok = false; break; }
+                    if (J >= 2 && !mbar_wait(&bar_pv_done[sb], ((J - 2) >> 1) & 1, kWaitBudget)) { ok = false; break; }
+                    tc_fence_after();
+                    const uint32_t k_addr = smem_addr(sKV + st * kStageBytes);
+                    for (int kk = 0; kk < kD / 16; ++kk) {
+                        const uint32_t off = (kk >> 2) * kHalf + (kk & 3) * 32;
+                        const uint64_t adesc = smem_desc(q_addr + off, 16, 1024, kSwizzle128B);
+                        const uint64_t bdesc = smem_desc(k_addr + off, 16, 1024, kSwizzle128B);
+                        umma_ss(tmem + col_s(sb), adesc, bdesc, id_s, kk > 0 ? 1u : 0u);
+                    }
+                    umma_commit(&bar_s_full[sb]);
+                    if (jl == g.nt - 1) umma_commit(&bar_q_empty);  // the last read of this stretch's Q
+                    if (jl >= 1 && !issue_pv(J - 1, jl == 1)) { ++J; ok = false; break; }
+                }
+                if (!ok) break;
+                if (!issue_pv(J - 1, g.nt == 1)) { ok = false; break; }
+                umma_commit(&bar_o_done);
+                ++nq;
             }
-            if (ok && !issue_pv(nt - 1)) ok = false;
             if (!ok) raise_error(p.err, kErrTimeout);
-            umma_commit(&bar_o_done);
-            // no MMA may still be writing tensor memory when it is released
-            if (!mbar_wait(&bar_o_done, 0, kWaitBudget)) raise_error(p.err, kErrTimeout);
+            if (J > 0) {
+                // no MMA may still be writing tensor memory when it is released
+                umma_commit(&bar_o_done);
+                if (!mbar_wait(&bar_o_done, nq & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
+            }
         }
     }
 
@@ -346,243 +495,377 @@ __global__ void __launch_bounds__(kThreads, 1)
     const int half = SPREAD ? (lane >> 4) : 0;
     const int r = SPREAD ? quad * 16 + (lane & 15) : quad * 32 + lane;
     const bool is_softmax = warp >= 2;
-    const bool row_active = is_softmax && r < m_valid;
-    const bool warp_active = is_softmax && ((SPREAD ? quad * 16 : quad * 32) < m_valid);
     const uint32_t lane_base = static_cast<uint32_t>(quad * 32) << 16;
-    const int limit = row_active ? (p.causal ? L + (row0 + r) / G + 1 : n) : 0;
+    const float kLn2 = 0.6931471805599453f;
     float m_run = -INFINITY, l_run = 0.f;  // SPREAD: l_run is this half's share of the row sum
     float o_acc[kOCols];
     bool failed = false;
+    bool row_active = false;  // the cluster split's merge below needs the (one) stretch's values
+    int m_valid = 0;
+
+    // normalised output row r of stretch g (and its log-sum-exp)
+    auto write_row = [&](const Seg& g) {
+        const int lr = g.mt * kM + r;
+        const int i = lr / G, jh = lr % G;
+        const size_t orow = (size_t)(g.q0 + i) * p.num_q_heads + g.h * G + jh;
+        const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
+        __nv_bfloat16* dst = p.o + orow * kD + half * kOCols;
+#pragma unroll
+        for (int c = 0; c < kOCols / 8; ++c) {
+            uint4 w;
+            w.x = pack_bf16x2(o_acc[c * 8 + 0] * inv, o_acc[c * 8 + 1] * inv);
+            w.y = pack_bf16x2(o_acc[c * 8 + 2] * inv, o_acc[c * 8 + 3] * inv);
+            w.z = pack_bf16x2(o_acc[c * 8 + 4] * inv, o_acc[c * 8 + 5] * inv);
+            w.w = pack_bf16x2(o_acc[c * 8 + 6] * inv, o_acc[c * 8 + 7] * inv);
+            *reinterpret_cast<uint4*>(dst + c * 8) = w;
+        }
+        if (p.lse && half == 0) p.lse[orow] = (m_run + __log2f(l_run)) * kLn2;
+    };
 
     if (is_softmax) {
-        for (int j = 0; j < nt; ++j) {
-            const int sb = j & 1;
-            if (!__all_sync(0xffffffffu, mbar_wait(&bar_s_full[sb], (j >> 1) & 1, kWaitBudget))) {
-                failed = true;
-                break;
-            }
-            tc_fence_after();
-            if (warp_active) {
-                const int nvalid = limit - (t_begin + j) * kTileN;
-                float x[kCols];
-#pragma unroll
-                for (int c = 0; c < kCols / 32; ++c) {
-                    uint32_t v[32];
-                    if (SPREAD) tmem_ld16x2_32<kTileN / 2>(tmem + lane_base + col_s(sb) + c * 32, v);
-                    else tmem_ld32(tmem + lane_base + col_s(sb) + c * 32, v);
-                    tmem_ld_wait();
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        const int kidx = half * (kTileN / 2) + c * 32 + e;
-                        x[c * 32 + e] = (kidx < nvalid) ? __uint_as_float(v[e]) * p.scale_log2 : -INFINITY;
-                    }
+        int J = 0, nq = 0;
+        int4 entry = make_int4(-1, 0, 0, 0);  // flat split: this CTA's work entry for the merge
+        for (int t = t_begin; t < t_end && !failed;) {
+            const Seg g = seg_at(t, t == t_begin);
+            if (FLAT && !g.whole && g.jt0 == 0) entry = make_int4(g.s, g.mt, t, T);  // a cut unit that starts here
+            t += seg_len(g);
+            const int row0 = g.mt * kM;
+            m_valid = min(kM, g.B * G - row0);
+            row_active = r < m_valid;
+            const bool warp_active = (SPREAD ? quad * 16 : quad * 32) < m_valid;
+            const int L = g.n - g.B;
+            const int limit = row_active ? (p.causal ? L + (row0 + r) / G + 1 : g.n) : 0;
+            m_run = -INFINITY;
+            l_run = 0.f;
+            for (int jl = 0; jl < g.nt; ++jl, ++J) {
+                const int sb = J & 1;
+                if (!__all_sync(0xffffffffu, mbar_wait(&bar_s_full[sb], (J >> 1) & 1, kWaitBudget))) {
+                    failed = true;
+                    break;
                 }
-                float mt_ = -INFINITY;
+                tc_fence_after();
+                if (warp_active) {
+                    const int nvalid = limit - (g.jt0 + jl) * kTileN;
+                    float x[kCols];
 #pragma unroll
-                for (int e = 0; e < kCols; ++e) mt_ = fmaxf(mt_, x[e]);
-                if (SPREAD) mt_ = fmaxf(mt_, __shfl_xor_sync(0xffffffffu, mt_, 16));
-                const float m_new = fmaxf(m_run, mt_);
-                const bool need = m_new > m_run + 8.f;
-                const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
-                // rescale the TMEM accumulator of rows whose max grew (warp-uniform TMEM access)
-                if (__any_sync(0xffffffffu, need && j > 0 && m_run != -INFINITY)) {
-                    if (!__all_sync(0xffffffffu,
-                                    mbar_wait(&bar_pv_done[(j - 1) & 1], ((j - 1) >> 1) & 1, kWaitBudget))) {
-                        failed = true;
-                    } else {
-                        tc_fence_after();
+                    for (int c = 0; c < kCols / 32; ++c) {
+                        uint32_t v[32];
+                        if (SPREAD) tmem_ld16x2_32<kTileN / 2>(tmem + lane_base + col_s(sb) + c * 32, v);
+                        else tmem_ld32(tmem + lane_base + col_s(sb) + c * 32, v);
+                        tmem_ld_wait();
 #pragma unroll
-                        for (int c = 0; c < kOCols / 32; ++c) {
-                            uint32_t v[32];
-                            if (SPREAD) tmem_ld16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
-                            else tmem_ld32(tmem + lane_base + kColO + c * 32, v);
-                            tmem_ld_wait();
-                            if (SPREAD) {
+                        for (int e = 0; e < 32; ++e) {
+                            const int kidx = half * (kTileN / 2) + c * 32 + e;
+                            x[c * 32 + e] = (kidx < nvalid) ? __uint_as_float(v[e]) * p.scale_log2 : -INFINITY;
+                        }
+                    }
+                    float mt_ = -INFINITY;
 #pragma unroll
-                                for (int e = 0; e < 32; ++e) v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-                                tmem_st16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
-                            } else {
-                                uint32_t w0[16], w1[16];
+                    for (int e = 0; e < kCols; ++e) mt_ = fmaxf(mt_, x[e]);
+                    if (SPREAD) mt_ = fmaxf(mt_, __shfl_xor_sync(0xffffffffu, mt_, 16));
+                    const float m_new = fmaxf(m_run, mt_);
+                    const bool need = m_new > m_run + 8.f;
+                    const float alpha = need ? fast_exp2(m_run - m_new) : 1.f;
+                    // rescale the TMEM accumulator of rows whose max grew (warp-uniform TMEM access)
+                    if (__any_sync(0xffffffffu, need && jl > 0 && m_run != -INFINITY)) {
+                        if (!__all_sync(0xffffffffu,
+                                        mbar_wait(&bar_pv_done[(J - 1) & 1], ((J - 1) >> 1) & 1, kWaitBudget))) {
+                            failed = true;
+                        } else {
+                            tc_fence_after();
 #pragma unroll
-                                for (int e = 0; e < 16; ++e) {
-                                    w0[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
-                                    w1[e] = __float_as_uint(__uint_as_float(v[16 + e]) * alpha);
+                            for (int c = 0; c < kOCols / 32; ++c) {
+                                uint32_t v[32];
+                                if (SPREAD) tmem_ld16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
+                                else tmem_ld32(tmem + lane_base + kColO + c * 32, v);
+                                tmem_ld_wait();
+                                if (SPREAD) {
+#pragma unroll
+                                    for (int e = 0; e < 32; ++e)
+                                        v[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+                                    tmem_st16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
+                                } else {
+                                    uint32_t w0[16], w1[16];
+#pragma unroll
+                                    for (int e = 0; e < 16; ++e) {
+                                        w0[e] = __float_as_uint(__uint_as_float(v[e]) * alpha);
+                                        w1[e] = __float_as_uint(__uint_as_float(v[16 + e]) * alpha);
+                                    }
+                                    tmem_st16(tmem + lane_base + kColO + c * 32, w0);
+                                    tmem_st16(tmem + lane_base + kColO + c * 32 + 16, w1);
                                 }
-                                tmem_st16(tmem + lane_base + kColO + c * 32, w0);
-                                tmem_st16(tmem + lane_base + kColO + c * 32 + 16, w1);
                             }
                         }
                     }
-                }
-                if (need) {
-                    l_run *= alpha;
-                    m_run = m_new;
-                }
-                float lsum = 0.f;
-                const bool any = m_run != -INFINITY;
-                if (SPREAD) {  // this half's 64 keys -> 32 packed P columns (the other half 32 further)
-                    uint32_t pk[32];
-#pragma unroll
-                    for (int e = 0; e < 32; ++e) {
-                        const float a = any ? fast_exp2(x[2 * e] - m_run) : 0.f;
-                        const float b = any ? fast_exp2(x[2 * e + 1] - m_run) : 0.f;
-                        lsum += a + b;
-                        pk[e] = pack_bf16x2(a, b);
+                    if (need) {
+                        l_run *= alpha;
+                        m_run = m_new;
                     }
-                    tmem_st16x2_32<kTileN / 4>(tmem + lane_base + col_s(sb), pk);
-                } else {
+                    float lsum = 0.f;
+                    const bool any = m_run != -INFINITY;
+                    if (SPREAD) {  // this half's 64 keys -> 32 packed P columns (the other half 32 further)
+                        uint32_t pk[32];
 #pragma unroll
-                    for (int c = 0; c < 4; ++c) {
-                        uint32_t pk[16];
-#pragma unroll
-                        for (int e = 0; e < 16; ++e) {
-                            const float a = any ? fast_exp2(x[c * 32 + 2 * e] - m_run) : 0.f;
-                            const float b = any ? fast_exp2(x[c * 32 + 2 * e + 1] - m_run) : 0.f;
+                        for (int e = 0; e < 32; ++e) {
+                            const float a = any ? fast_exp2(x[2 * e] - m_run) : 0.f;
+                            const float b = any ? fast_exp2(x[2 * e + 1] - m_run) : 0.f;
                             lsum += a + b;
                             pk[e] = pack_bf16x2(a, b);
                         }
-                        tmem_st16(tmem + lane_base + col_s(sb) + c * 16, pk);
+                        tmem_st16x2_32<kTileN / 4>(tmem + lane_base + col_s(sb), pk);
+                    } else {
+#pragma unroll
+                        for (int c = 0; c < 4; ++c) {
+                            uint32_t pk[16];
+#pragma unroll
+                            for (int e = 0; e < 16; ++e) {
+                                const float a = any ? fast_exp2(x[c * 32 + 2 * e] - m_run) : 0.f;
+                                const float b = any ? fast_exp2(x[c * 32 + 2 * e + 1] - m_run) : 0.f;
+                                lsum += a + b;
+                                pk[e] = pack_bf16x2(a, b);
+                            }
+                            tmem_st16(tmem + lane_base + col_s(sb) + c * 16, pk);
+                        }
                     }
+                    l_run += lsum;
+                    tmem_st_wait();
                 }
-                l_run += lsum;
-                tmem_st_wait();
+                tc_fence_before();
+                mbar_arrive(&bar_p_full[sb]);
+                if (failed) break;
             }
-            tc_fence_before();
-            mbar_arrive(&bar_p_full[sb]);
-            if (failed) break;
+            // the stretch's accumulator
+            if (g.nt > 0 && !failed && !__all_sync(0xffffffffu, mbar_wait(&bar_o_done, nq & 1, kWaitBudget)))
+                failed = true;
+            failed = __any_sync(0xffffffffu, failed);
+            tc_fence_after();
+            if (warp_active && g.nt > 0 && !failed) {
+#pragma unroll
+                for (int c = 0; c < kOCols / 32; ++c) {
+                    uint32_t v[32];
+                    if (SPREAD) tmem_ld16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
+                    else tmem_ld32(tmem + lane_base + kColO + c * 32, v);
+                    tmem_ld_wait();
+#pragma unroll
+                    for (int e = 0; e < 32; ++e) o_acc[c * 32 + e] = __uint_as_float(v[e]);
+                }
+            } else {
+#pragma unroll
+                for (int e = 0; e < kOCols; ++e) o_acc[e] = 0.f;
+                if (g.nt == 0 || failed) {
+                    m_run = -INFINITY;
+                    l_run = 0.f;
+                }
+            }
+            if (SPREAD) l_run += __shfl_xor_sync(0xffffffffu, l_run, 16);  // the whole row's sum
+            if (g.nt > 0) ++nq;
+            if (FLAT && !g.whole && m_valid > p.slot_rows) {  // a block longer than max_q_len: rows past the slot are dropped
+                if (r == 0 && warp == 2) raise_error(p.err, kErrDeviceArg);
+                row_active = row_active && r < p.slot_rows;
+            }
+            if (FLAT && !failed && row_active) {
+                if (g.whole) {
+                    write_row(g);
+                } else {  // the partial (O, m, l) of this stretch's rows, for attn_combine_kernel
+                    float* slot = p.part + (size_t)(2 * blockIdx.x + g.slot) * p.slot_rows * (kD + 2);
+                    float* orow = slot + (size_t)r * kD + half * kOCols;
+#pragma unroll
+                    for (int c = 0; c < kOCols / 4; ++c)
+                        *reinterpret_cast<float4*>(orow + c * 4) =
+                            make_float4(o_acc[c * 4], o_acc[c * 4 + 1], o_acc[c * 4 + 2], o_acc[c * 4 + 3]);
+                    if (half == 0)
+                        *reinterpret_cast<float2*>(slot + (size_t)p.slot_rows * kD + 2 * r) = make_float2(m_run, l_run);
+                }
+            }
         }
-        // final accumulator
-        if (nt > 0 && !failed && !__all_sync(0xffffffffu, mbar_wait(&bar_o_done, 0, kWaitBudget))) failed = true;
-        failed = __any_sync(0xffffffffu, failed);
         if (failed) raise_error(p.err, kErrTimeout);
-        tc_fence_after();
-        if (warp_active && nt > 0 && !failed) {
-#pragma unroll
-            for (int c = 0; c < kOCols / 32; ++c) {
-                uint32_t v[32];
-                if (SPREAD) tmem_ld16x2_32<kD / 2>(tmem + lane_base + kColO + c * 32, v);
-                else tmem_ld32(tmem + lane_base + kColO + c * 32, v);
-                tmem_ld_wait();
-#pragma unroll
-                for (int e = 0; e < 32; ++e) o_acc[c * 32 + e] = __uint_as_float(v[e]);
-            }
-        } else {
-#pragma unroll
-            for (int e = 0; e < kOCols; ++e) o_acc[e] = 0.f;
-            if (nt == 0 || failed) {
-                m_run = -INFINITY;
-                l_run = 0.f;
-            }
-        }
-        if (SPREAD) l_run += __shfl_xor_sync(0xffffffffu, l_run, 16);  // the whole row's sum
+        if (FLAT && tid == 64) p.work[blockIdx.x] = entry;
     }
 
-    const float kLn2 = 0.6931471805599453f;
-    if (CS == 1) {
-        if (row_active) {
-            const int lr = row0 + r;
-            const int i = lr / G, jh = lr % G;
-            const size_t orow = (size_t)(q0 + i) * p.num_q_heads + h * G + jh;
-            const float inv = l_run > 0.f ? 1.f / l_run : 0.f;
-            __nv_bfloat16* dst = p.o + orow * kD + half * kOCols;
+    if (!FLAT) {
+        if (CS == 1) {
+            if (row_active) write_row(one);
+        } else {
+            // ---- merge of the CS partial (m, l, O) triples through distributed shared memory.  After the
+            // first cluster barrier every K/V ring is idle (all of its TMA loads were consumed); each CTA
+            // leaves its partial there and pulls the rows it owns from all peers:
+            //   opart  [kM rows][kD] fp32 partial O (16-byte chunks swizzled by row)
+            //   row_ml [kM] (m, l) of each row's partial
+            //   ml_st, w_st, inv_st  the peers' (m, l) of the owned rows, their weights, 1/L
+            m_valid = min(kM, one.B * G - one.mt * kM);
+            const int row0 = one.mt * kM;
+            cg::cluster_group cluster = cg::this_cluster();
+            float* opart = reinterpret_cast<float*>(sKV);
+            float2* row_ml = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float));
+            if (is_softmax) {
+                if (row_active) {
 #pragma unroll
-            for (int c = 0; c < kOCols / 8; ++c) {
-                uint4 w;
-                w.x = pack_bf16x2(o_acc[c * 8 + 0] * inv, o_acc[c * 8 + 1] * inv);
-                w.y = pack_bf16x2(o_acc[c * 8 + 2] * inv, o_acc[c * 8 + 3] * inv);
-                w.z = pack_bf16x2(o_acc[c * 8 + 4] * inv, o_acc[c * 8 + 5] * inv);
-                w.w = pack_bf16x2(o_acc[c * 8 + 6] * inv, o_acc[c * 8 + 7] * inv);
-                *reinterpret_cast<uint4*>(dst + c * 8) = w;
+                    for (int c = 0; c < kOCols / 4; ++c) {
+                        const int pc = (half * (kOCols / 4) + c) ^ (r & 31);
+                        *reinterpret_cast<float4*>(opart + r * kD + pc * 4) =
+                            make_float4(o_acc[c * 4], o_acc[c * 4 + 1], o_acc[c * 4 + 2], o_acc[c * 4 + 3]);
+                    }
+                }
+                if (half == 0) row_ml[r] = make_float2(m_run, l_run);
             }
-            if (p.lse && half == 0) p.lse[orow] = (m_run + __log2f(l_run)) * kLn2;
-        }
-    } else {
-        // ---- merge of the CS partial (m, l, O) triples through distributed shared memory.  After the
-        // first cluster barrier every K/V ring is idle (all of its TMA loads were consumed); each CTA
-        // leaves its partial there and pulls the rows it owns from all peers:
-        //   opart  [kM rows][kD] fp32 partial O (16-byte chunks swizzled by row)
-        //   row_ml [kM] (m, l) of each row's partial
-        //   ml_st, w_st, inv_st  the peers' (m, l) of the owned rows, their weights, 1/L
-        cg::cluster_group cluster = cg::this_cluster();
-        float* opart = reinterpret_cast<float*>(sKV);
-        float2* row_ml = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float));
-        if (is_softmax) {
-            if (row_active) {
-#pragma unroll
-                for (int c = 0; c < kOCols / 4; ++c) {
-                    const int pc = (half * (kOCols / 4) + c) ^ (r & 31);
-                    *reinterpret_cast<float4*>(opart + r * kD + pc * 4) =
-                        make_float4(o_acc[c * 4], o_acc[c * 4 + 1], o_acc[c * 4 + 2], o_acc[c * 4 + 3]);
+            cluster.sync();
+            const int per = (m_valid + (int)CS - 1) / (int)CS;
+            const int rbeg = (int)crank * per;
+            const int nmy = max(0, min(m_valid, rbeg + per) - rbeg);
+            // one round of remote loads for the peers' (m, l) of the owned rows, then the weights
+            float2* ml_st = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float) + kM * sizeof(float2));
+            float* w_st = reinterpret_cast<float*>(ml_st + kMaxCluster * kM);
+            float* inv_st = w_st + kMaxCluster * kM;
+            for (int idx = tid; idx < (int)CS * nmy; idx += kThreads) {
+                const int pr = idx / nmy, rr = idx % nmy;
+                ml_st[pr * nmy + rr] = *cluster.map_shared_rank(&row_ml[rbeg + rr], pr);
+            }
+            __syncthreads();
+            for (int rr = tid; rr < nmy; rr += kThreads) {
+                float M = -INFINITY;
+                for (uint32_t pr = 0; pr < CS; ++pr) M = fmaxf(M, ml_st[pr * nmy + rr].x);
+                float Lsum = 0.f;
+                for (uint32_t pr = 0; pr < CS; ++pr) {
+                    const float2 ml = ml_st[pr * nmy + rr];
+                    const float w = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - M);
+                    w_st[pr * nmy + rr] = w;
+                    Lsum += w * ml.y;
+                }
+                inv_st[rr] = Lsum > 0.f ? 1.f / Lsum : 0.f;
+                if (p.lse) {
+                    const int lr = row0 + rbeg + rr;
+                    p.lse[(size_t)(one.q0 + lr / G) * p.num_q_heads + one.h * G + lr % G] =
+                        (M + __log2f(Lsum)) * kLn2;
                 }
             }
-            if (half == 0) row_ml[r] = make_float2(m_run, l_run);
-        }
-        cluster.sync();
-        const int per = (m_valid + (int)CS - 1) / (int)CS;
-        const int rbeg = (int)crank * per;
-        const int nmy = max(0, min(m_valid, rbeg + per) - rbeg);
-        // one round of remote loads for the peers' (m, l) of the owned rows, then the weights
-        float2* ml_st = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float) + kM * sizeof(float2));
-        float* w_st = reinterpret_cast<float*>(ml_st + kMaxCluster * kM);
-        float* inv_st = w_st + kMaxCluster * kM;
-        for (int idx = tid; idx < (int)CS * nmy; idx += kThreads) {
-            const int pr = idx / nmy, rr = idx % nmy;
-            ml_st[pr * nmy + rr] = *cluster.map_shared_rank(&row_ml[rbeg + rr], pr);
-        }
-        __syncthreads();
-        for (int rr = tid; rr < nmy; rr += kThreads) {
-            float M = -INFINITY;
-            for (uint32_t pr = 0; pr < CS; ++pr) M = fmaxf(M, ml_st[pr * nmy + rr].x);
-            float Lsum = 0.f;
-            for (uint32_t pr = 0; pr < CS; ++pr) {
-                const float2 ml = ml_st[pr * nmy + rr];
-                const float w = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - M);
-                w_st[pr * nmy + rr] = w;
-                Lsum += w * ml.y;
-            }
-            inv_st[rr] = Lsum > 0.f ? 1.f / Lsum : 0.f;
-            if (p.lse) {
-                const int lr = row0 + rbeg + rr;
-                p.lse[(size_t)(q0 + lr / G) * p.num_q_heads + h * G + lr % G] = (M + __log2f(Lsum)) * kLn2;
-            }
-        }
-        __syncthreads();
-        // the owned rows: every peer's 16-byte chunk requested at once
-        for (int item = tid; item < nmy * (kD / 4); item += kThreads) {
-            const int rr = item / (kD / 4);
-            const int c = item % (kD / 4);
-            const int row = rbeg + rr;
-            const float* src = opart + row * kD + ((c ^ (row & 31)) * 4);
-            float4 v[kMaxCluster];
+            __syncthreads();
+            // the owned rows: every peer's 16-byte chunk requested at once
+            for (int item = tid; item < nmy * (kD / 4); item += kThreads) {
+                const int rr = item / (kD / 4);
+                const int c = item % (kD / 4);
+                const int row = rbeg + rr;
+                const float* src = opart + row * kD + ((c ^ (row & 31)) * 4);
+                float4 v[kMaxCluster];
 #pragma unroll
-            for (int pr = 0; pr < kMaxCluster; ++pr)
-                if (pr < (int)CS) v[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(src), pr);
-            float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int pr = 0; pr < kMaxCluster; ++pr)
+                    if (pr < (int)CS) v[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(src), pr);
+                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
-            for (int pr = 0; pr < kMaxCluster; ++pr) {
-                if (pr < (int)CS) {
-                    const float w = w_st[pr * nmy + rr];
-                    acc.x += w * v[pr].x;
-                    acc.y += w * v[pr].y;
-                    acc.z += w * v[pr].z;
-                    acc.w += w * v[pr].w;
+                for (int pr = 0; pr < kMaxCluster; ++pr) {
+                    if (pr < (int)CS) {
+                        const float w = w_st[pr * nmy + rr];
+                        acc.x += w * v[pr].x;
+                        acc.y += w * v[pr].y;
+                        acc.z += w * v[pr].z;
+                        acc.w += w * v[pr].w;
+                    }
                 }
+                const float inv = inv_st[rr];
+                const int lr = row0 + row;
+                const size_t orow = (size_t)(one.q0 + lr / G) * p.num_q_heads + one.h * G + lr % G;
+                uint2 w2;
+                w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+                w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+                *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
             }
-            const float inv = inv_st[rr];
-            const int lr = row0 + row;
-            const size_t orow = (size_t)(q0 + lr / G) * p.num_q_heads + h * G + lr % G;
-            uint2 w2;
-            w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-            w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-            *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
+            cluster.sync();  // no CTA leaves while peers may still read its shared memory
         }
-        cluster.sync();  // no CTA leaves while peers may still read its shared memory
     }
 
     tc_fence_before();
     __syncthreads();
     tc_fence_after();
     if (warp == 1) tmem_dealloc(tmem, kTmemCols);
+}
+
+// Flat split, second kernel: the units whose tiles were cut between CTA groups.  The CTA of the main
+// kernel that holds a cut unit's first tile names it in its work entry; CTA (c, r) here takes work entry
+// c and its rows [r * kCombRows, (r + 1) * kCombRows).  Thread (row, 16-byte chunk) merges the partial
+// (O, m, l) of the unit's CTAs in order -- O = sum_j 2^(m_j - M) O_j / sum_j 2^(m_j - M) l_j, M the
+// largest m_j, as a running merge over batches of kCombBatch partials whose loads are all in flight --
+// and writes the bf16 output chunk (and the row's log-sum-exp).
+constexpr int kCombRows = 16;
+constexpr int kCombThreads = kCombRows * kD / 4;  // 512: one 16-byte chunk of a row each
+constexpr int kCombBatch = 8;
+__global__ void __launch_bounds__(kCombThreads) attn_combine_kernel(const AttnParams p, int grid_main) {
+    __shared__ int32_t gstart[kAttnFlatMaxGrid + 1];  // the CTA groups' ranges: group j has [gstart[j], gstart[j+1])
+    griddep_launch_dependents();
+    griddep_wait();  // the partials and work entries of the main kernel
+    const int tid = threadIdx.x;
+    const int G = p.group;
+    const int chunks = (p.slot_rows + kCombRows - 1) / kCombRows;
+    const int c = blockIdx.x / chunks, r = blockIdx.x - c * chunks;
+    const int4 wk = __ldcg(p.work + c);
+    if (wk.x < 0) return;  // CTA c holds no cut unit's first tile (uniform per CTA)
+    const int s = wk.x, mt = wk.y, U0 = wk.z, T = wk.w;
+    const int h = c % p.num_kv_heads;
+    const int q0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_q + s);
+    const int B = p.num_seqs == 1 ? p.total_q : __ldg(p.cu_q + s + 1) - q0;
+    const int n = p.num_seqs == 1 ? p.total_kv : __ldg(p.cu_kv + s + 1) - __ldg(p.cu_kv + s);
+    const int rows = min(min(kM, B * G - mt * kM), p.slot_rows);
+    if (r * kCombRows >= rows) return;  // uniform per CTA
+    const int U1 = U0 + cdiv(n, kTileN);
+    const int ngroups = grid_main / p.num_kv_heads;
+    for (int j = tid; j <= ngroups; j += kCombThreads) gstart[j] = (int)((long long)j * T / ngroups);
+    __syncthreads();
+    // the group whose range holds the unit's last tile: the last j with gstart[j] <= U1 - 1
+    int lo = c / p.num_kv_heads, hi = ngroups;
+    while (hi - lo > 1) {
+        const int mid = (lo + hi) >> 1;
+        if (gstart[mid] <= U1 - 1) lo = mid; else hi = mid;
+    }
+    const int j0 = c / p.num_kv_heads, j1 = lo;
+    const int rl = r * kCombRows + tid / (kD / 4);  // the row within the unit
+    const int c4 = tid % (kD / 4);                  // its 16-byte chunk
+    if (rl >= rows) return;
+    const size_t slot_floats = (size_t)p.slot_rows * (kD + 2);
+    const size_t ml_off = (size_t)p.slot_rows * kD + 2 * rl;
+    float M = -INFINITY, Lsum = 0.f;
+    float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+    for (int jb = j0; jb <= j1; jb += kCombBatch) {
+        float2 ml[kCombBatch];
+        float4 v[kCombBatch];
+#pragma unroll
+        for (int k = 0; k < kCombBatch; ++k) {
+            const int j = jb + k;
+            ml[k] = make_float2(-INFINITY, 0.f);
+            v[k] = make_float4(0.f, 0.f, 0.f, 0.f);
+            if (j <= j1 && gstart[j] < gstart[j + 1]) {
+                // CTA (group j, head h): its first stretch (slot 0) unless its range began before the unit
+                const float* sp =
+                    p.part + (size_t)(2 * (j * p.num_kv_heads + h) + (gstart[j] >= U0 ? 0 : 1)) * slot_floats;
+                ml[k] = __ldcg(reinterpret_cast<const float2*>(sp + ml_off));
+                v[k] = __ldcg(reinterpret_cast<const float4*>(sp + (size_t)rl * kD + c4 * 4));
+            }
+        }
+#pragma unroll
+        for (int k = 0; k < kCombBatch; ++k) {
+            if (ml[k].x == -INFINITY) continue;  // nothing (or no visible key) in this partial
+            if (ml[k].x > M) {
+                const float sc = M == -INFINITY ? 0.f : fast_exp2(M - ml[k].x);
+                Lsum *= sc;
+                acc.x *= sc;
+                acc.y *= sc;
+                acc.z *= sc;
+                acc.w *= sc;
+                M = ml[k].x;
+            }
+            const float w = fast_exp2(ml[k].x - M);
+            Lsum += w * ml[k].y;
+            acc.x += w * v[k].x;
+            acc.y += w * v[k].y;
+            acc.z += w * v[k].z;
+            acc.w += w * v[k].w;
+        }
+    }
+    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+    const int lr = mt * kM + rl;
+    const size_t orow = (size_t)(q0 + lr / G) * p.num_q_heads + h * G + lr % G;
+    uint2 w2;
+    w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+    w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+    *reinterpret_cast<uint2*>(p.o + orow * kD + c4 * 4) = w2;
+    if (p.lse && c4 == 0) p.lse[orow] = (M + __log2f(Lsum)) * 0.6931471805599453f;
 }
 
 // --------------------------------------------------------------------------- fp32 SIMT path
@@ -663,6 +946,21 @@ __global__ void __launch_bounds__(128) attn_f32_simt_kernel(const float* __restr
 
 }  // namespace
 
+namespace {
+// Rows of one partial slot of the flat split: a unit's query rows (at most one 128-row tile), rounded
+// up to 16 so that every slot starts on a 16-byte boundary.
+int flat_slot_rows(int max_q_len, int group) {
+    const long long rows = (long long)max_q_len * group;
+    return (int)((std::min<long long>(kM, rows) + 15) / 16 * 16);
+}
+}  // namespace
+
+size_t attention_flat_scratch_bytes(int max_q_len, int group) {
+    if (max_q_len < 1 || group < 1) return 0;
+    return (size_t)2 * kAttnFlatMaxGrid * flat_slot_rows(max_q_len, group) * (kD + 2) * sizeof(float) +
+           (size_t)kAttnFlatMaxGrid * sizeof(int4);
+}
+
 int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
     if (a.head_dim != kD) return BP_ERR_UNSUPPORTED;
     const int G = a.num_q_heads / a.num_kv_heads;
@@ -716,6 +1014,9 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     p.pages_per_seq = paged ? a.pages_per_seq : 0;
     p.page_shift = 0;
     while (paged && (1 << p.page_shift) < a.page_size) ++p.page_shift;
+    p.part = nullptr;
+    p.work = nullptr;
+    p.slot_rows = flat_slot_rows(a.max_q_len, G);
     p.err = a.err_word;
     if (!q_tma) qmap = kmap;  // unused by the kernel
 
@@ -730,8 +1031,10 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     int max_active[kMaxCluster + 1];
     std::unique_lock<std::mutex> cfg_lock(cfg_mu);
     if (!configured[dev.device]) {
-        for (auto kern : {attn_bf16_tc_kernel<false, false>, attn_bf16_tc_kernel<true, false>,
-                          attn_bf16_tc_kernel<false, true>, attn_bf16_tc_kernel<true, true>})
+        for (auto kern : {attn_bf16_tc_kernel<false, false, false>, attn_bf16_tc_kernel<true, false, false>,
+                          attn_bf16_tc_kernel<false, true, false>, attn_bf16_tc_kernel<true, true, false>,
+                          attn_bf16_tc_kernel<false, false, true>, attn_bf16_tc_kernel<true, false, true>,
+                          attn_bf16_tc_kernel<false, true, true>, attn_bf16_tc_kernel<true, true, true>})
             if (cudaFuncSetAttribute(kern, cudaFuncAttributeMaxDynamicSharedMemorySize, kDynSmem) != cudaSuccess ||
                 cudaFuncSetAttribute(kern, cudaFuncAttributeNonPortableClusterSizeAllowed, 1) != cudaSuccess ||
                 cudaFuncSetAttribute(kern, cudaFuncAttributePreferredSharedMemoryCarveout,
@@ -750,7 +1053,7 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
             probe.attrs = pa;
             probe.numAttrs = 1;
             int n_clusters = 0;
-            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel<false, false>, &probe) !=
+            if (cudaOccupancyMaxActiveClusters(&n_clusters, attn_bf16_tc_kernel<false, false, false>, &probe) !=
                 cudaSuccess) {
                 cudaGetLastError();
                 n_clusters = 0;
@@ -761,11 +1064,19 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     }
     for (int c = 0; c <= kMaxCluster; ++c) max_active[c] = max_active_dev[dev.device][c];
     cfg_lock.unlock();
-    // cluster size: the largest split of each unit's keys for which every unit's cluster is resident
-    // in the same wave (a unit left for a second wave would double the time)
-    // (the tiles of the longest unit per CTA set the time: minimise them, then prefer the smallest
-    // cluster, whose merge is cheapest)
+
     const int max_tiles = (a.max_kv_len + kTileN - 1) / kTileN;
+    cudaLaunchConfig_t cfg = {};
+    cudaLaunchAttribute attr[2];
+    cfg.blockDim = dim3(kThreads, 1, 1);
+    cfg.dynamicSmemBytes = kDynSmem;
+    cfg.stream = stream;
+    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[1].val.programmaticStreamSerializationAllowed = 1;
+
+    // cluster split: the largest split of each unit's keys for which every unit's cluster is resident in
+    // the same wave (a unit left for a second wave would double the time); the tiles of the longest unit
+    // per CTA set the time: minimise them, then prefer the smallest cluster, whose merge is cheapest
     int cs = 1, best = max_tiles;
     for (int c = 2; c <= kMaxCluster; ++c) {
         if (c > max_tiles || units > max_active[c] || units * c > dev.sm_count) continue;
@@ -776,25 +1087,58 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
         }
     }
 
-    cudaLaunchConfig_t cfg = {};
-    cudaLaunchAttribute attr[2];
+    // flat split: the tiles of every sequence's query tiles cut evenly over groups of CTAs, one CTA per KV
+    // head and per SM (at most kAttnFlatMaxGrid in all, and no more groups than one head has tiles); units
+    // cut between groups are merged by a second kernel.  It needs the Q tile by TMA, the sequences'
+    // offsets in shared memory and the workspace's partial slots and work entries.  Measured on this GPU,
+    // it gains only where the cluster split leaves SMs idle and every CTA of the flat split streams a
+    // long run (8 x 32K keys: 171 vs 175 us); with short runs the second kernel and the stretch
+    // boundaries cost more than the idle SMs (1 x 2K keys: 13.4 vs 9.3 us).  BP_ATTENTION_SPLIT=flat or
+    // =cluster overrides the choice (for tests and measurements).
+    const long long tiles_bound = (long long)a.num_seqs * m_tiles * max_tiles;
+    const int ngroups = (int)std::min<long long>(std::min(dev.sm_count, kAttnFlatMaxGrid) / a.num_kv_heads,
+                                                 tiles_bound);
+    const int flat_grid = ngroups * a.num_kv_heads;
+    const bool flat_ok = q_tma && a.num_seqs <= kMaxOrderedSeqs && a.scratch != nullptr &&
+                         a.scratch_bytes >= attention_flat_scratch_bytes(a.max_q_len, G) && ngroups >= 1;
+    bool flat = flat_ok && units * cs * 10 <= (long long)dev.sm_count * 9 && tiles_bound >= 32LL * ngroups;
+    if (const char* force = getenv("BP_ATTENTION_SPLIT")) {
+        if (strcmp(force, "flat") == 0) flat = flat_ok;
+        else if (strcmp(force, "cluster") == 0) flat = false;
+    }
+    cudaError_t e;
+    if (flat) {
+        p.part = static_cast<float*>(a.scratch);
+        p.work = reinterpret_cast<int4*>(p.part + (size_t)2 * kAttnFlatMaxGrid * p.slot_rows * (kD + 2));
+        cfg.gridDim = dim3((unsigned)flat_grid, 1, 1);
+        cfg.attrs = &attr[1];
+        cfg.numAttrs = 1;
+        if (paged) e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, true, true>, qmap, kmap, vmap, p)
+                              : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, false, true>, qmap, kmap, vmap, p);
+        else e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, true, true>, qmap, kmap, vmap, p)
+                        : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, false, true>, qmap, kmap, vmap, p);
+        if (e != cudaSuccess) return BP_ERR_CUDA;
+        if (max_tiles <= 1) return BP_OK;  // every unit is one tile: none is cut between CTAs
+        cudaLaunchConfig_t cc = {};
+        cc.gridDim = dim3((unsigned)(flat_grid * ((p.slot_rows + kCombRows - 1) / kCombRows)), 1, 1);
+        cc.blockDim = dim3(kCombThreads, 1, 1);
+        cc.stream = stream;
+        cc.attrs = &attr[1];
+        cc.numAttrs = 1;
+        return cudaLaunchKernelEx(&cc, attn_combine_kernel, p, flat_grid) == cudaSuccess ? BP_OK : BP_ERR_CUDA;
+    }
+
     cfg.gridDim = dim3((unsigned)(units * cs), 1, 1);
-    cfg.blockDim = dim3(kThreads, 1, 1);
-    cfg.dynamicSmemBytes = kDynSmem;
-    cfg.stream = stream;
     attr[0].id = cudaLaunchAttributeClusterDimension;
     attr[0].val.clusterDim.x = cs;
     attr[0].val.clusterDim.y = 1;
     attr[0].val.clusterDim.z = 1;
-    attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
-    attr[1].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
     cfg.numAttrs = 2;
-    cudaError_t e;
-    if (paged) e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, true>, qmap, kmap, vmap, p)
-                          : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, false>, qmap, kmap, vmap, p);
-    else e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, true>, qmap, kmap, vmap, p)
-                    : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, false>, qmap, kmap, vmap, p);
+    if (paged) e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, true, false>, qmap, kmap, vmap, p)
+                          : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<true, false, false>, qmap, kmap, vmap, p);
+    else e = spread ? cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, true, false>, qmap, kmap, vmap, p)
+                    : cudaLaunchKernelEx(&cfg, attn_bf16_tc_kernel<false, false, false>, qmap, kmap, vmap, p);
     if (e != cudaSuccess) return BP_ERR_CUDA;
     return BP_OK;
 }

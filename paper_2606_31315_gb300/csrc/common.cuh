@@ -59,8 +59,15 @@ struct AttentionArgs {
     // paged KV cache (NULL block_table: contiguous rows from cu_kv); pool of num_pages pages
     const int32_t* block_table;
     int pages_per_seq, page_size, num_pages;
+    void* scratch;  // workspace past the header (the flat split's partial slots)
+    size_t scratch_bytes;
 };
 int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+// The flat split of the bf16 attention runs on at most this many CTAs (one per SM) and keeps two
+// partial (O, m, l) slots per CTA in the workspace; a workspace without room for them keeps the
+// cluster split.
+constexpr int kAttnFlatMaxGrid = 192;
+size_t attention_flat_scratch_bytes(int max_q_len, int group);
 
 struct KvAppendArgs {
     void* k_cache;

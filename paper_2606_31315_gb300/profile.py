@@ -1,7 +1,7 @@
 """One kernel of the hot path on its own, for profilers: seeded synthetic inputs of the benchmark's
 shapes on the device (nothing else allocated), a few warm-up calls, then N calls.
 
-    python -m paper_2606_31315_gb300.profile CASE [--calls N] [--warmup W]
+    python -m paper_2606_31315_gb300.profile CASE [--calls N] [--warmup W] [--split flat|cluster]
 
 CASE is one of:
   verify_epilogue_t1  Qwen3-4B LM head (151936 x 2560 bf16) fused with the acceptance, 16 target and
@@ -12,6 +12,13 @@ CASE is one of:
                       and 480 x 151936 draft fp32 logits), T = 1: the three throughput kernels
   accept_batch_t0     the same batch at T = 0 (target logits only)
   attention           causal verify attention, 1 sequence, 2048 + 16 keys, 32 / 8 heads, D = 128
+  attention_c3        causal verify attention over the ragged batch: 32 sequences, blocks 8..24,
+                      contexts 562..8118 (576 MB of K/V)
+  attention_c5        causal verify attention over the long-context batch: 8 sequences of 32768 + 16
+                      keys (1.07 GB of K/V)
+  accept_c5_t1        acceptance of the long-context batch at T = 1: 8 x 16 target and 8 x 15 draft
+                      rows over 151936 (150.7 MB): the three throughput kernels
+  step_c5             one long-context verify step: attention_c5, then accept_c5_t1
   policy              policy head, 32 requests, 2560 -> 2048 -> 9 bf16 (W1 loaded at once per CTA)
   policy_d151936      policy head at the paper's input width, 32 requests, 151936 -> 2048 -> 9 bf16
                       (W1 622 MB streamed through the ring)
@@ -21,12 +28,20 @@ CASE is one of:
 from __future__ import annotations
 
 import argparse
+import itertools
 
 import torch
 
 from . import _binding as bp
 
 V, H, CTX, B, HQ, HKV, D = 151936, 2560, 2048, 16, 32, 8, 128
+SPLIT = {"split": "flat"}  # attention cases: a full-size workspace (flat split) or the 256-byte header (cluster split)
+
+
+def _attn_ws(dev, num_seqs, max_q):
+    if SPLIT["split"] == "cluster":
+        return bp.workspace(256, dev)
+    return bp.workspace(bp.block_attention_workspace_size(num_seqs, max_q, HQ, HKV, D), dev)
 
 
 def _verify_epilogue(dev, gen, temperature):
@@ -71,8 +86,49 @@ def _attention(dev, gen):
     v = torch.randn(CTX + B, HKV, D, device=dev, generator=gen).to(torch.bfloat16)
     cu_q = torch.tensor([0, B], dtype=torch.int32, device=dev)
     cu_kv = torch.tensor([0, CTX + B], dtype=torch.int32, device=dev)
-    ws = bp.workspace(bp.block_attention_workspace_size(1, B, HQ, HKV, D), dev)
+    ws = _attn_ws(dev, 1, B)
     return lambda: bp.block_attention(q, k, v, cu_q, cu_kv, B, CTX + B, mask=bp.MASK_CAUSAL, ws=ws)
+
+
+def _batch_attention(dev, gen, ctx, block):
+    """Causal verify attention over sequences of the given contexts and blocks (Qwen3 heads)."""
+    kv = [c + b for c, b in zip(ctx, block)]
+    q = torch.randn(sum(block), HQ, D, device=dev, generator=gen).to(torch.bfloat16)
+    k = torch.randn(sum(kv), HKV, D, device=dev, generator=gen).to(torch.bfloat16)
+    v = torch.randn(sum(kv), HKV, D, device=dev, generator=gen).to(torch.bfloat16)
+    off = lambda xs: torch.tensor([0] + list(itertools.accumulate(xs)), dtype=torch.int32, device=dev)  # noqa
+    cu_q, cu_kv = off(block), off(kv)
+    ws = _attn_ws(dev, len(ctx), max(block))
+    return lambda: bp.block_attention(q, k, v, cu_q, cu_kv, max(block), max(kv), mask=bp.MASK_CAUSAL, ws=ws)
+
+
+def _accept_c5(dev, gen):
+    s, td = 8, 8 * (B - 1)
+    t = torch.randn(td + s, V, device=dev, generator=gen) * 3
+    trow = torch.tensor([i + i // (B - 1) for i in range(td)], device=dev)
+    d = t[trow] + torch.randn(td, V, device=dev, generator=gen)
+    tok = torch.randint(0, V, (td,), device=dev, generator=gen, dtype=torch.int32)
+    cu = torch.arange(0, td + 1, B - 1, dtype=torch.int32, device=dev)
+    ua, us = torch.rand(td, device=dev, generator=gen), torch.rand(s, device=dev, generator=gen)
+    ws = bp.workspace(bp.spec_accept_workspace_size(s, td, V), dev)
+    return lambda: bp.spec_accept(t, d, tok, cu, 1.0, ua, us, want_accept_prob=False, ws=ws)
+
+
+def _step_c5(dev, gen):
+    attn = _batch_attention(dev, gen, [32768] * 8, [B] * 8)
+    acc = _accept_c5(dev, gen)
+
+    def step():
+        attn()
+        acc()
+    return step
+
+
+def _ragged_shapes():
+    from . import workloads
+
+    w = workloads.get("ragged")
+    return list(w.ctx), list(w.block)
 
 
 def _policy(dev, gen, d_in):
@@ -104,6 +160,10 @@ CASES = {
     "accept_batch_t1": lambda dev, gen: _accept_batch(dev, gen, 1.0),
     "accept_batch_t0": lambda dev, gen: _accept_batch(dev, gen, 0.0),
     "attention": _attention,
+    "attention_c3": lambda dev, gen: _batch_attention(dev, gen, *_ragged_shapes()),
+    "attention_c5": lambda dev, gen: _batch_attention(dev, gen, [32768] * 8, [B] * 8),
+    "accept_c5_t1": _accept_c5,
+    "step_c5": _step_c5,
     "policy": lambda dev, gen: _policy(dev, gen, 2560),
     "policy_d151936": lambda dev, gen: _policy(dev, gen, V),
     "tau": _tau,
@@ -115,7 +175,9 @@ def main(argv=None) -> None:
     ap.add_argument("case", choices=sorted(CASES))
     ap.add_argument("--calls", type=int, default=3)
     ap.add_argument("--warmup", type=int, default=2)
+    ap.add_argument("--split", choices=["flat", "cluster"], default="flat")
     args = ap.parse_args(argv)
+    SPLIT["split"] = args.split
     dev = torch.device("cuda:0")
     gen = torch.Generator(device=dev)
     gen.manual_seed(7)

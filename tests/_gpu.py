@@ -2,6 +2,9 @@
 through the C ABI, run the oracle on the same inputs (whole or sampled) and compare."""
 from __future__ import annotations
 
+import contextlib
+import os
+
 import numpy as np
 import torch
 
@@ -25,14 +28,42 @@ def to_dev(x: np.ndarray, dtype: str | None = None) -> torch.Tensor:
     return torch.from_numpy(np.ascontiguousarray(x)).to(dev())
 
 
-def run_attention(a: dict, mask: int):
-    """CUDA path on the whole workload; returns (o fp32 numpy, lse numpy)."""
+def attention_ws(a: dict, split: str = "auto"):
+    """A workspace for the attention of workload a: the size the library asks for, or (split "cluster")
+    the 256-byte header alone, which keeps the cluster split of the bf16 path."""
+    if split == "cluster":
+        return bp.workspace(256, dev())
+    return bp.workspace(bp.block_attention_workspace_size(len(a["cu_q"]) - 1, a["max_q_len"], a["num_q_heads"],
+                                                          a["num_kv_heads"], a["head_dim"]), dev())
+
+
+@contextlib.contextmanager
+def forced_split(split: str):
+    """The library's choice between the flat and the cluster split of the keys ("auto"), or one of them
+    forced through BP_ATTENTION_SPLIT, which the library reads at every call."""
+    old = os.environ.get("BP_ATTENTION_SPLIT")
+    if split in ("flat", "cluster"):
+        os.environ["BP_ATTENTION_SPLIT"] = split
+    else:
+        os.environ.pop("BP_ATTENTION_SPLIT", None)
+    try:
+        yield
+    finally:
+        if old is None:
+            os.environ.pop("BP_ATTENTION_SPLIT", None)
+        else:
+            os.environ["BP_ATTENTION_SPLIT"] = old
+
+
+def run_attention(a: dict, mask: int, split: str = "auto"):
+    """CUDA path on the whole workload; returns (o fp32 numpy, lse numpy).  split: "auto" (the library
+    chooses), "flat" or "cluster" (forced)."""
     q, k, v = to_dev(a["q"], a["dtype"]), to_dev(a["k"], a["dtype"]), to_dev(a["v"], a["dtype"])
     cu_q, cu_kv = to_dev(a["cu_q"]), to_dev(a["cu_kv"])
     lse = torch.empty(q.shape[0], q.shape[1], dtype=torch.float32, device=dev())
-    ws = bp.workspace(bp.block_attention_workspace_size(len(a["cu_q"]) - 1, a["max_q_len"], q.shape[1], k.shape[1],
-                                                        q.shape[2]), dev())
-    o, _ = bp.block_attention(q, k, v, cu_q, cu_kv, a["max_q_len"], a["max_kv_len"], mask=mask, lse=lse, ws=ws)
+    ws = attention_ws(a, split)
+    with forced_split(split):
+        o, _ = bp.block_attention(q, k, v, cu_q, cu_kv, a["max_q_len"], a["max_kv_len"], mask=mask, lse=lse, ws=ws)
     assert bp.get_status(ws) == 0
     return o.float().cpu().numpy(), lse.cpu().numpy()
 

@@ -1,9 +1,10 @@
 """GPU parity of bp_block_attention against the fp64 oracle (bf16 tensor-core path and fp32 path).
 
 Tolerance: max |O - O_ref| / max |O_ref| <= 2e-2 per (sequence, query head) slice (bf16 inputs,
-fp32 accumulation); log-sum-exp within 2e-3.  Small ragged cases are compared in full; the
-full-size workloads run exactly as the benchmark launches them and are compared on sampled
-sequences (and KV heads for the 32K-context case).
+fp32 accumulation); log-sum-exp within 2e-3.  Small ragged cases are compared in full, on both
+splits of the keys (the flat split and the cluster split, each forced); the full-size workloads run
+exactly as the benchmark launches them (the library's own choice of split) and are compared on
+sampled sequences (and KV heads for the 32K-context case).
 """
 import numpy as np
 import pytest
@@ -27,8 +28,8 @@ def _lib():
     bp.load()
 
 
-def _check(a, mask, seqs=None, kv_head=None):
-    o, lse = run_attention(a, mask)
+def _check(a, mask, seqs=None, kv_head=None, split="auto"):
+    o, lse = run_attention(a, mask, split)
     seqs = range(len(a["cu_q"]) - 1) if seqs is None else seqs
     err, lerr = attention_errors(o, lse, a, mask, seqs, kv_head)
     assert err <= ATTN_TOL, err
@@ -43,16 +44,69 @@ def _check(a, mask, seqs=None, kv_head=None):
     ((2048,), (16,)),                                # Qwen3-4B verify shape, one sequence
     ((4000, 10, 255, 256, 257), (16, 16, 16, 16, 16)),
 ])
-def test_ragged_small(ctx, block, mask):
+@pytest.mark.parametrize("split", ["flat", "cluster"])
+def test_ragged_small(ctx, block, mask, split):
     w = wl.custom(seed=sum(ctx) + len(block), ctx=ctx, block=block, num_q_heads=32, num_kv_heads=8)
-    _check(wl.attention_inputs(w), mask)
+    _check(wl.attention_inputs(w), mask, split=split)
 
 
-@pytest.mark.parametrize("hq,hkv", [(8, 8), (64, 8), (16, 2), (4, 1)])
-def test_group_sizes(hq, hkv):
+@pytest.mark.parametrize("hq,hkv", [(8, 8), (64, 8), (16, 2), (4, 1), (24, 8)])
+@pytest.mark.parametrize("split", ["flat", "cluster"])
+def test_group_sizes(hq, hkv, split):
+    # (24, 8): a group of 3 does not divide the 128-row tile, so Q is gathered without TMA (cluster split)
     w = wl.custom(seed=hq * 10 + hkv, ctx=(300, 77), block=(12, 31), num_q_heads=hq, num_kv_heads=hkv)
     for mask in (CAUSAL, BIDIR):
-        _check(wl.attention_inputs(w), mask)
+        _check(wl.attention_inputs(w), mask, split=split)
+
+
+@pytest.mark.parametrize("ctx,block", [
+    ((3, 1, 0, 300), (1, 1, 2, 1)),                  # fewer key tiles than CTAs: CTAs without work
+    ((40000,), (16,)),                                # one unit per KV head cut over ~19 CTAs each
+    ((9000, 120, 130, 2500, 31), (16, 9, 64, 1, 24)),  # cuts mid-unit, B=64 (two query tiles), B=1
+])
+def test_flat_split_cuts(ctx, block):
+    """The flat split's ranges start and end anywhere inside a unit; partial stretches are merged by
+    the second kernel in CTA order."""
+    w = wl.custom(seed=len(ctx) * 7 + block[0], ctx=ctx, block=block, num_q_heads=32, num_kv_heads=8)
+    a = wl.attention_inputs(w)
+    for mask in (CAUSAL, BIDIR):
+        _check(a, mask, split="flat")
+
+
+@pytest.mark.parametrize("n", [256, 257])
+def test_many_sequences(n):
+    """Up to 256 sequences take the flat split (their offsets fit the CTA's table); 257 the cluster split."""
+    rng = np.random.default_rng(n)
+    w = wl.custom(seed=n, ctx=tuple(int(x) for x in rng.integers(0, 300, n)),
+                  block=tuple(int(x) for x in rng.integers(1, 17, n)), num_q_heads=32, num_kv_heads=8)
+    a = wl.attention_inputs(w)
+    _check(a, CAUSAL, seqs=[0, 1, n // 2, n - 1], split="flat")
+
+
+def _attn_kernels(a, split):
+    from torch.profiler import ProfilerActivity, profile
+
+    with profile(activities=[ProfilerActivity.CUDA]) as prof:
+        run_attention(a, CAUSAL, split)
+        torch.cuda.synchronize()
+    return {e.name for e in prof.events() if "attn_" in e.name}
+
+
+def test_split_choice():
+    """Left to the library, a batch-1 verify (2K keys) takes the cluster split and 8 sequences of 16K keys
+    the flat split (two kernels); a 256-byte workspace always keeps the cluster split."""
+    _attn_kernels(wl.attention_inputs(wl.custom(seed=1, ctx=(100,), block=(4,), num_q_heads=32, num_kv_heads=8)),
+                  "auto")  # the profiler's first session may miss kernels while it starts
+    small = wl.attention_inputs(wl.get("qwen3_4b"))
+    names = _attn_kernels(small, "auto")
+    assert not any("attn_combine_kernel" in x for x in names) and any("attn_bf16_tc_kernel" in x for x in names)
+    assert any("attn_combine_kernel" in x for x in _attn_kernels(small, "flat"))
+    long8 = wl.attention_inputs(wl.custom(seed=9, ctx=(16384,) * 8, block=(16,) * 8, num_q_heads=32,
+                                          num_kv_heads=8))
+    assert any("attn_combine_kernel" in x for x in _attn_kernels(long8, "auto"))
+    assert not any("attn_combine_kernel" in x for x in _attn_kernels(long8, "cluster"))
+    err, lerr = attention_errors(*run_attention(long8, CAUSAL), long8, CAUSAL, [0, 7], kv_head=3)
+    assert err <= ATTN_TOL and lerr <= LSE_TOL
 
 
 def test_qwen3_4b_full():

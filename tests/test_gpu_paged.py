@@ -10,7 +10,7 @@ import torch
 import paper_2606_31315_gb300 as bp
 from paper_2606_31315_gb300 import workloads as wl
 
-from _gpu import ATTN_TOL, LSE_TOL, attention_errors, dev, to_dev
+from _gpu import ATTN_TOL, LSE_TOL, attention_errors, attention_ws, dev, forced_split, to_dev
 
 pytestmark = pytest.mark.gpu
 
@@ -30,25 +30,26 @@ def _ragged():
     return wl.attention_inputs(w)
 
 
-def _run_paged(a, pk, mask):
+def _run_paged(a, pk, mask, split="auto"):
     q = to_dev(a["q"], "bf16")
     kc, vc = to_dev(pk["k_cache"], "bf16"), to_dev(pk["v_cache"], "bf16")
     cu_q, cu_kv, bt = to_dev(a["cu_q"]), to_dev(a["cu_kv"]), to_dev(pk["block_table"])
     lse = torch.empty(q.shape[0], q.shape[1], dtype=torch.float32, device=dev())
-    ws = bp.workspace(bp.block_attention_workspace_size(len(a["cu_q"]) - 1, a["max_q_len"], q.shape[1], kc.shape[1],
-                                                        q.shape[2]), dev())
-    o, _ = bp.block_attention_paged(q, kc, vc, cu_q, cu_kv, bt, pk["page_size"], int(a["cu_kv"][-1]),
-                                    a["max_q_len"], a["max_kv_len"], mask=mask, lse=lse, ws=ws)
+    ws = attention_ws(a, split)
+    with forced_split(split):
+        o, _ = bp.block_attention_paged(q, kc, vc, cu_q, cu_kv, bt, pk["page_size"], int(a["cu_kv"][-1]),
+                                        a["max_q_len"], a["max_kv_len"], mask=mask, lse=lse, ws=ws)
     assert bp.get_status(ws) == 0
     return o.float().cpu().numpy(), lse.cpu().numpy()
 
 
 @pytest.mark.parametrize("page_size", [16, 64, 128, 256])
 @pytest.mark.parametrize("mask", [bp.MASK_CAUSAL, bp.MASK_BIDIR])
-def test_paged_ragged_batch(page_size, mask):
+@pytest.mark.parametrize("split", ["flat", "cluster"])
+def test_paged_ragged_batch(page_size, mask, split):
     a = _ragged()
     pk = wl.paged_kv(a["k"], a["v"], a["cu_kv"], page_size, seed=page_size)
-    o, lse = _run_paged(a, pk, mask)
+    o, lse = _run_paged(a, pk, mask, split)
     err, lerr = attention_errors(o, lse, a, mask, range(len(a["cu_q"]) - 1))
     assert err <= ATTN_TOL and lerr <= LSE_TOL, (err, lerr)
 

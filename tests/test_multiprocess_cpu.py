@@ -86,7 +86,7 @@ def test_reference_arm_prints_the_contract_line():
 
     assert d["impl"] == "reference" and d["metric"] == bench.METRIC and d["unit"] == "tokens/s"
     assert d["higher_is_better"] is True and d["n_gpus"] == 1 and d["steps"] == 1 and d["value"] > 0
-    assert d["config"]["workload"].startswith("qwen3_4b")
+    assert d["config"] == bench.headline_config(1) and d["config"]["workload"].startswith("long_context")
     cb = d["cpu_baseline"]
     assert cb["kind"] == "oracle" and cb["cores"] >= 1 and cb["value"] == d["value"] and cb["sample"]
     assert d["e2e"] == {"value": d["value"], "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}
