@@ -596,14 +596,17 @@ def run_ours(args):
                    roofline_tokens_per_s=round(tokens / (nbytes / (peak * 1e9)), 1), workload=what)
         return out
 
-    batch_kernels1 = ["batch_stats_kernel<false,true>", "batch_decide_kernel<false>", "batch_draw_kernel"]
-    batch_kernels0 = ["batch_stats_kernel<true,true>", "batch_decide_kernel<true>"]
+    batch_kernels1 = ["batch_stats_kernel<false,true>", "batch_draw_kernel (decisions inside)"]
+    batch_kernels0 = ["batch_stats_kernel<true,true>", "batch_decide_kernel"]
     rows = {
-        "c5_attention_causal_8x32784": dict(row(t_h_attn, attn_h_bytes, ["attn_bf16_tc_kernel"]),
+        "c5_attention_causal_8x32784": dict(row(t_h_attn, attn_h_bytes, ["attn_bf16_tc_kernel (flat split)",
+                                                                         "attn_combine_kernel"]),
                                             traffic=committed_traffic("attn_c5")),
         "c5_accept_t1_8x16": row(t_h_acc1, accept_bytes(hw, 1.0), batch_kernels1),
         "c5_accept_greedy_t0_8x16": row(t_h_acc0, accept_bytes(hw, 0.0), batch_kernels0),
-        "c5_step_t0_attention_accept_greedy": step_row(t_h_step0, hw, 0.0, ["attn_bf16_tc_kernel"] + batch_kernels0,
+        "c5_step_t0_attention_accept_greedy": step_row(t_h_step0, hw, 0.0,
+                                                       ["attn_bf16_tc_kernel (flat split)", "attn_combine_kernel"]
+                                                       + batch_kernels0,
                                                        "8 sequences x (32768 + 16) keys, greedy acceptance"),
         "c3_step_ragged_32req_attention_accept_t1": step_row(
             t_rstep, rw, 1.0, ["attn_bf16_tc_kernel"] + batch_kernels1,
@@ -669,9 +672,11 @@ def run_ours(args):
         dist.destroy_process_group()
 
 
-# The kernels one headline step launches: the verify attention, then the acceptance's three throughput
-# kernels (the T = 1 acceptance of 8 x 31 rows reads 37.7M logits, past the 6.5M crossover).
-STEP_KERNELS = ["attn_bf16_tc_kernel", "batch_stats_kernel", "batch_decide_kernel", "batch_draw_kernel"]
+# The kernels one headline step launches: the verify attention (its flat split and the merge of the cut
+# units: 8 x 32784 keys leave the cluster split's SMs idle), then the acceptance's two throughput kernels
+# (the T = 1 acceptance of 8 x 31 rows reads 37.7M logits, past the 6.5M crossover; the draw kernel takes
+# the decisions).
+STEP_KERNELS = ["attn_bf16_tc_kernel", "attn_combine_kernel", "batch_stats_kernel", "batch_draw_kernel"]
 STEP_LAUNCHES = len(STEP_KERNELS)
 
 

@@ -9,15 +9,18 @@
 //   1. stats: one CTA per 16384-entry chunk of every target and drafter row streams the chunk once
 //      (coalesced 16-byte loads) and writes the chunk's (scaled max, sum of 2^(l*log2e/T - max)) --
 //      at T = 0 its (max, lowest index) -- so the whole batch is one HBM-bound pass;
-//   2. decide: one warp per sequence merges its rows' chunk statistics in a fixed order, forms the
-//      ratios a_i, the first rejection k and the outputs (at T = 0 the emitted argmax too).  (Taking
-//      the decisions in the statistics kernel, in the CTA that completes a sequence, costs every CTA a
-//      gpu-scope ticket behind its store: measured slower for large batches);
-//   3. draw (T > 0): one CTA per chunk of each sequence's draw row pair (the rejected row, or the bonus
-//      row) forms the chunk's segment masses of max(0, p_k - q_k) and of p_k in exact 2^-52 fixed
-//      point; the last CTA of the sequence (ticket) finds the chunk and the 128-entry segment where the
-//      inverse CDF crosses u_s * total from the stored masses, then the entry from that segment's 128
-//      logits, and writes the emitted token.
+//   2. T = 0: decide: one warp per sequence, one lane per block position, merges its row's chunk
+//      statistics in a fixed order and compares the drafted token with the argmax; the first mismatch k
+//      and the outputs (the emitted argmax too).  (Taking the decisions in the statistics kernel, in the
+//      CTA that completes a sequence, costs every CTA a gpu-scope ticket behind its store: measured
+//      slower for large batches);
+//   2. T > 0: draw: one CTA per chunk of each sequence's draw row pair (or per part of a chunk, when the
+//      chunks alone would leave SMs idle).  Its first warp derives the sequence's decisions the same
+//      way (ratios a_i, the first rejection k -- the rejected row k and its drafter row, or the bonus
+//      row -- one CTA writing the outputs); then every thread forms the part's segment masses of
+//      max(0, p_k - q_k) and of p_k in exact 2^-52 fixed point; the last CTA of the sequence (ticket)
+//      finds the part and the 128-entry segment where the inverse CDF crosses u_s * total from the
+//      stored masses, then the entry from that segment's 128 logits, and writes the emitted token.
 // Only the one draw row pair per sequence is read twice.  The kernels chain with programmatic dependent
 // launch.
 #include <cuda_runtime.h>
@@ -34,6 +37,7 @@ constexpr int kBThreads = 256;
 constexpr int kBChunk = 16384;                 // vocabulary entries per chunk
 constexpr int kBVec = kBChunk / 4 / kBThreads;  // 16-byte groups per thread: 16 (64 entries)
 constexpr int kBSegs = kBVec;                  // 128-entry segments per warp of a chunk
+constexpr int kMaxDrawSplit = 4;               // parts a draw chunk may be cut into
 
 struct BatchParams {
     const float* target;  // [rows_t][vocab]
@@ -48,10 +52,8 @@ struct BatchParams {
     int32_t* out_tokens;
     float* accept_prob;
     float2* part;      // [rows][chunks] chunk statistics (T = 0: value, index bits)
-    float2* rowstat;   // [rows] row statistics
-    float4* drawrec;   // [num_seqs][2] the draw's rows, weight constants and output slot (T > 0)
-    ulonglong2* ctot;  // [num_seqs][chunks] draw masses of r and p (fixed point)
-    unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses (chunks > 1)
+    ulonglong2* ctot;  // [num_seqs][chunks * parts] draw masses of r and p of the chunks' parts (fixed point)
+    unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses
     int* tickets;      // [num_seqs], zero between calls
     unsigned int* err;
 };
@@ -85,140 +87,12 @@ __device__ __forceinline__ void load_chunk(const float* __restrict__ src, int n,
     for (int j = 0; j < kBVec; ++j) v[j] = load4<VEC>(src, 4 * (tid + j * kBThreads), n);
 }
 
-// The draw of a sequence: its row pair, the constants of its weights and the output slot, written by
-// the decisions as two 16-byte words and read back by every draw CTA in one round trip.
+// The draw of a sequence: its row pair, the constants of its weights and the output slot.
 struct DrawPair {
     int trow, drow;  // drow < 0: a bonus draw from p alone
     float Mt, izt, Md, izd;
     int out;         // the emitted token's slot in out_tokens
 };
-__device__ __forceinline__ void store_draw(float4* rec, int trow, int drow, float2 st, float2 sd, int out) {
-    // a row whose entries are all -inf weighs every entry 0 (M = 0, 1/Z = 0 keep it free of NaN)
-    const bool tz = st.x == -INFINITY, dz = drow < 0 || sd.x == -INFINITY;
-    rec[0] = make_float4(__int_as_float(trow), __int_as_float(drow), tz ? 0.f : st.x, tz ? 0.f : __fdiv_rn(1.f, st.y));
-    rec[1] = make_float4(dz ? 0.f : sd.x, dz ? 0.f : __fdiv_rn(1.f, sd.y), __int_as_float(out), 0.f);
-}
-__device__ __forceinline__ DrawPair load_draw(const float4* rec) {
-    const float4 a = __ldcg(rec), b = __ldcg(rec + 1);
-    DrawPair d;
-    d.trow = __float_as_int(a.x);
-    d.drow = __float_as_int(a.y);
-    d.Mt = a.z;
-    d.izt = a.w;
-    d.Md = b.x;
-    d.izd = b.y;
-    d.out = __float_as_int(b.z);
-    return d;
-}
-
-// Decisions of sequence s, by one warp: its rows' statistics from their chunks', the ratios a_i, the
-// first rejection k and the outputs (at T = 0 the emitted argmax too).
-template <bool GREEDY>
-__device__ __forceinline__ void decide_seq(const BatchParams& p, int s, int lane) {
-    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
-    const int nrows = GREEDY ? g + 1 : 2 * g + 1;  // the target rows, then (T > 0) the drafter's
-    // the drafted tokens, their two logits and uniforms do not depend on the statistics: the first 32
-    // positions' loads are issued before the merges
-    struct Pick {
-        int x;
-        bool valid;
-        float tx, dx, u;
-    };
-    const auto pick = [&](int i) {
-        Pick q{-1, false, -INFINITY, -INFINITY, 1.f};
-        if (i < g) {
-            q.x = p.tokens[d0 + i];
-            q.valid = q.x >= 0 && q.x < p.vocab;
-            if (!GREEDY && q.valid) {
-                q.tx = p.target[(size_t)(t0 + i) * p.vocab + q.x];
-                q.dx = p.draft[(size_t)(d0 + i) * p.vocab + q.x];
-            }
-            if (!GREEDY) q.u = p.u_accept[d0 + i];
-        }
-        return q;
-    };
-    const Pick first = pick(lane);
-    // each lane merges whole rows (two at a time), chunks in order, eight chunks' loads in flight
-    constexpr int RH = 2, CQ = 8;
-    const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
-    for (int rr0 = lane; rr0 < nrows; rr0 += 32 * RH) {
-        int r[RH];
-        float2 acc[RH];
-#pragma unroll
-        for (int h = 0; h < RH; ++h) {
-            const int rr = rr0 + 32 * h;
-            r[h] = rr >= nrows ? -1 : rr <= g ? t0 + rr : p.rows_t + d0 + (rr - g - 1);
-            acc[h] = ident;
-        }
-        for (int c0 = 0; c0 < p.chunks; c0 += CQ) {
-            float2 x[RH][CQ];
-#pragma unroll
-            for (int h = 0; h < RH; ++h)
-#pragma unroll
-                for (int q = 0; q < CQ; ++q)
-                    x[h][q] = r[h] >= 0 && c0 + q < p.chunks ? __ldcg(&p.part[(size_t)r[h] * p.chunks + c0 + q])
-                                                             : ident;
-#pragma unroll
-            for (int h = 0; h < RH; ++h)
-#pragma unroll
-                for (int q = 0; q < CQ; ++q) {
-                    if (GREEDY) {
-                        int ai = __float_as_int(acc[h].y);
-                        amax_merge(acc[h].x, ai, x[h][q].x, __float_as_int(x[h][q].y));
-                        acc[h].y = __int_as_float(ai);
-                    } else {
-                        lse_merge(acc[h].x, acc[h].y, x[h][q].x, x[h][q].y);
-                    }
-                }
-        }
-#pragma unroll
-        for (int h = 0; h < RH; ++h) {
-            if (r[h] < 0) continue;
-            float2 a = acc[h];
-            if (GREEDY && __float_as_int(a.y) >= p.vocab) a.y = __int_as_float(0);  // every entry -inf: index 0
-            p.rowstat[r[h]] = a;
-        }
-    }
-    __syncwarp();  // the warp's row statistics are written (and visible to its lanes)
-    int k = g;
-    for (int i0 = 0; i0 < g; i0 += 32) {
-        const int i = i0 + lane;
-        const Pick q = i0 == 0 ? first : pick(i);
-        bool rej = false;
-        if (i < g) {
-            if (!q.valid) raise_error(p.err, kErrDeviceArg);
-            const float2 st = p.rowstat[t0 + i];
-            float a;
-            if (GREEDY) {
-                a = q.valid && q.x == __float_as_int(st.y) ? 1.f : 0.f;
-                rej = a == 0.f;
-            } else {
-                const float2 sd = p.rowstat[p.rows_t + d0 + i];
-                // a = min(1, p(x)/q(x)) in the log domain (q(x) = 0 < p(x) gives 1, p(x) = 0 gives 0)
-                if (!q.valid || q.tx == -INFINITY) a = 0.f;
-                else if (q.dx == -INFINITY) a = 1.f;
-                else a = fminf(1.f, ex2(__fmaf_rn(q.tx, p.c2, -st.x) - __fmaf_rn(q.dx, p.c2, -sd.x)) * (sd.y / st.y));
-                rej = !(q.u < a);
-            }
-            if (p.accept_prob) p.accept_prob[d0 + i] = a;
-        }
-        const unsigned b = __ballot_sync(0xffffffffu, rej);
-        if (b && k == g) k = i0 + __ffs(b) - 1;
-    }
-    for (int j = lane; j <= g; j += 32) {
-        if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
-        else if (j > k) p.out_tokens[t0 + j] = -1;
-        else if (GREEDY) p.out_tokens[t0 + j] = __float_as_int(p.rowstat[t0 + k].y);
-    }
-    if (lane == 0) {
-        p.n_accepted[s] = k;
-        if (!GREEDY) {
-            const int drow = k < g ? p.rows_t + d0 + k : -1;
-            store_draw(p.drawrec + 2 * s, t0 + k, drow, p.rowstat[t0 + k],
-                       drow >= 0 ? p.rowstat[drow] : make_float2(-INFINITY, 0.f), t0 + k);
-        }
-    }
-}
 
 // ---- 1. chunk statistics of every row
 template <bool GREEDY, bool VEC>
@@ -285,13 +159,162 @@ __global__ void __launch_bounds__(kBThreads) batch_stats_kernel(const BatchParam
     }
 }
 
-// ---- 2. decisions: one warp per sequence
+
+// Statistics of row r from its chunks', merged in chunk order by one lane (the order every path uses),
+// all chunks' loads in flight at once (up to kMergeBatch chunks, i.e. vocabularies up to 262144, in
+// one round trip).  GREEDY: (max, lowest index); else (scaled max, sum of 2^(l*c2 - max)).
+constexpr int kMergeBatch = 16;
 template <bool GREEDY>
+__device__ __forceinline__ void load_row_parts(const BatchParams& p, int r, int c0, float2 (&x)[kMergeBatch]) {
+    const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
+#pragma unroll
+    for (int q = 0; q < kMergeBatch; ++q)
+        x[q] = r >= 0 && c0 + q < p.chunks ? __ldcg(&p.part[(size_t)r * p.chunks + c0 + q]) : ident;
+}
+template <bool GREEDY>
+__device__ __forceinline__ void merge_parts(float2& acc, const float2 (&x)[kMergeBatch]) {
+#pragma unroll
+    for (int q = 0; q < kMergeBatch; ++q) {
+        if (GREEDY) {
+            int ai = __float_as_int(acc.y);
+            amax_merge(acc.x, ai, x[q].x, __float_as_int(x[q].y));
+            acc.y = __int_as_float(ai);
+        } else {
+            lse_merge(acc.x, acc.y, x[q].x, x[q].y);
+        }
+    }
+}
+// Both rows r1, r2 (r2 < 0: none) at once: every load of the first batch is issued before any merge.
+template <bool GREEDY>
+__device__ __forceinline__ void merge_rows(const BatchParams& p, int r1, int r2, float2& a1, float2& a2) {
+    const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
+    a1 = ident;
+    a2 = ident;
+    for (int c0 = 0; c0 < p.chunks; c0 += kMergeBatch) {
+        float2 x1[kMergeBatch], x2[kMergeBatch];
+        load_row_parts<GREEDY>(p, r1, c0, x1);
+        load_row_parts<GREEDY>(p, r2, c0, x2);
+        merge_parts<GREEDY>(a1, x1);
+        merge_parts<GREEDY>(a2, x2);
+    }
+}
+
+// Greedy decisions (T = 0) of sequence s by one warp, one lane per block position (32 at a time): lane
+// i <= gamma merges target row i's (max, lowest index) from its chunks' and compares drafted token i
+// with it; the first mismatch k by ballot; the emitted token is row k's argmax (the bonus row's when
+// every draft matches).
+__device__ __forceinline__ void decide_greedy(const BatchParams& p, int s, int lane) {
+    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
+    int k = g, emitted = 0, bonus = 0;
+    for (int i0 = 0; i0 <= g; i0 += 32) {
+        const int i = i0 + lane;
+        const int x = i < g ? p.tokens[d0 + i] : -1;
+        float2 st, none;
+        merge_rows<true>(p, i <= g ? t0 + i : -1, -1, st, none);
+        int am = __float_as_int(st.y);
+        if (am >= p.vocab) am = 0;  // every entry -inf: index 0
+        bool rej = false;
+        if (i < g) {
+            const bool valid = x >= 0 && x < p.vocab;
+            if (!valid) raise_error(p.err, kErrDeviceArg);
+            rej = !(valid && x == am);
+            if (p.accept_prob) p.accept_prob[d0 + i] = rej ? 0.f : 1.f;
+        }
+        if (g - i0 < 32) bonus = __shfl_sync(0xffffffffu, am, g - i0);
+        const unsigned b = __ballot_sync(0xffffffffu, rej);
+        if (b && k == g) {
+            const int l = __ffs(b) - 1;
+            k = i0 + l;
+            emitted = __shfl_sync(0xffffffffu, am, l);
+        }
+    }
+    if (k == g) emitted = bonus;
+    for (int j = lane; j <= g; j += 32) {
+        if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
+        else if (j > k) p.out_tokens[t0 + j] = -1;
+        else p.out_tokens[t0 + j] = emitted;
+    }
+    if (lane == 0) p.n_accepted[s] = k;
+}
+
+// The decisions of sequence s at T > 0 by one warp, one lane per block position (32 at a time): lane
+// i < gamma takes drafted position i -- its target and drafter row statistics, a_i -- and lane i =
+// gamma the bonus row's statistics; the first rejection k by ballot; then the draw's row pair and the
+// constants of its weights into *d (lane 0).  Every CTA of the sequence's draw derives the same k; the
+// writer CTA also writes n_accepted, accept_prob and the out_tokens slots other than the emitted
+// token's, and reports draft tokens outside the vocabulary; the others stop at the first block of 32
+// positions that holds a rejection.
+__device__ __forceinline__ void decide_draw(const BatchParams& p, int s, int lane, bool writer, DrawPair* d) {
+    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
+    int k = g;
+    float2 stk = make_float2(-INFINITY, 0.f), sdk = stk, bonus = stk;
+    for (int i0 = 0; i0 <= g; i0 += 32) {
+        const int i = i0 + lane;
+        const bool draft = i < g;
+        // every load at once: the tokens (their logits follow), the uniforms, both rows' chunk statistics
+        const int x = draft ? p.tokens[d0 + i] : -1;
+        const float u = draft ? p.u_accept[d0 + i] : 1.f;
+        float2 st, sd;
+        merge_rows<false>(p, i <= g ? t0 + i : -1, draft ? p.rows_t + d0 + i : -1, st, sd);
+        bool rej = false;
+        if (draft) {
+            const bool valid = x >= 0 && x < p.vocab;
+            float tx = -INFINITY, dx = -INFINITY;
+            if (valid) {
+                tx = p.target[(size_t)(t0 + i) * p.vocab + x];
+                dx = p.draft[(size_t)(d0 + i) * p.vocab + x];
+            }
+            // a = min(1, p(x)/q(x)) in the log domain (q(x) = 0 < p(x) gives 1, p(x) = 0 gives 0)
+            float a;
+            if (!valid || tx == -INFINITY) a = 0.f;
+            else if (dx == -INFINITY) a = 1.f;
+            else a = fminf(1.f, ex2(__fmaf_rn(tx, p.c2, -st.x) - __fmaf_rn(dx, p.c2, -sd.x)) * (sd.y / st.y));
+            rej = !(u < a);
+            if (writer) {
+                if (!valid) raise_error(p.err, kErrDeviceArg);
+                if (p.accept_prob) p.accept_prob[d0 + i] = a;
+            }
+        }
+        if (g - i0 < 32) {  // this block holds the bonus row (lane g - i0)
+            bonus.x = __shfl_sync(0xffffffffu, st.x, g - i0);
+            bonus.y = __shfl_sync(0xffffffffu, st.y, g - i0);
+        }
+        const unsigned b = __ballot_sync(0xffffffffu, rej);
+        if (b && k == g) {
+            const int l = __ffs(b) - 1;
+            k = i0 + l;
+            stk = make_float2(__shfl_sync(0xffffffffu, st.x, l), __shfl_sync(0xffffffffu, st.y, l));
+            sdk = make_float2(__shfl_sync(0xffffffffu, sd.x, l), __shfl_sync(0xffffffffu, sd.y, l));
+            if (!writer) break;
+        }
+    }
+    if (k == g) stk = bonus;  // every draft accepted: the bonus row
+    if (writer) {
+        for (int j = lane; j <= g; j += 32) {
+            if (j < k) p.out_tokens[t0 + j] = p.tokens[d0 + j];
+            else if (j > k) p.out_tokens[t0 + j] = -1;
+        }
+        if (lane == 0) p.n_accepted[s] = k;
+    }
+    if (lane == 0) {
+        // a row whose entries are all -inf weighs every entry 0 (M = 0, 1/Z = 0 keep it free of NaN)
+        const bool tz = stk.x == -INFINITY, dz = k == g || sdk.x == -INFINITY;
+        d->trow = t0 + k;
+        d->drow = k < g ? p.rows_t + d0 + k : -1;
+        d->Mt = tz ? 0.f : stk.x;
+        d->izt = tz ? 0.f : __fdiv_rn(1.f, stk.y);
+        d->Md = dz ? 0.f : sdk.x;
+        d->izd = dz ? 0.f : __fdiv_rn(1.f, sdk.y);
+        d->out = t0 + k;
+    }
+}
+
+// ---- 2. greedy decisions (T = 0): one warp per sequence.  (At T > 0 the draw kernel decides.)
 __global__ void __launch_bounds__(kBThreads) batch_decide_kernel(const BatchParams p) {
     griddep_launch_dependents();
     griddep_wait();
     const int s = blockIdx.x * (kBThreads / 32) + (threadIdx.x >> 5);
-    if (s < p.num_seqs) decide_seq<GREEDY>(p, s, threadIdx.x & 31);
+    if (s < p.num_seqs) decide_greedy(p, s, threadIdx.x & 31);
 }
 
 // Weights of four entries: (r = max(0, p - q), p) with p = 2^(l*c2 - Mt) / Zt (r = 0 without a draft row).
@@ -310,60 +333,83 @@ __device__ __forceinline__ float sum4f(float4 v) { return (v.x + v.y) + (v.z + v
 
 // Masses of the 128-entry segments (j, warp) of one chunk of the draw pair, 2^-52 fixed point, into
 // segR / segP; returns the calling thread's one: segment (lane, warp)'s r mass for lanes below 16,
-// segment (lane - 16, warp)'s p mass above.  The chunk's 16-byte groups are loaded in PH phases: one
-// keeps every load in flight (for grids of at most one CTA per SM), two fit 128 registers, i.e. two
-// CTAs per SM (for larger grids).
-template <bool VEC, int PH>
-__device__ __forceinline__ unsigned long long chunk_masses(const BatchParams& p, const DrawPair& d, int chunk, int tid,
-                                                           unsigned long long (*segR)[kBSegs],
+// segment (lane - 16, warp)'s p mass above.  With SPLIT > 1 the CTA takes part `sub` of the chunk only
+// (groups j in [sub * 16 / SPLIT, (sub + 1) * 16 / SPLIT): 16384 / SPLIT consecutive entries); the other
+// segments come out 0.  The part's 16-byte groups are loaded in PH phases: one keeps every load in
+// flight, two fit 128 registers, i.e. two CTAs per SM (for grids larger than the SM count).
+template <bool VEC, int PH, int SPLIT>
+__device__ __forceinline__ unsigned long long chunk_masses(const BatchParams& p, const DrawPair& d, int chunk, int sub,
+                                                           int tid, unsigned long long (*segR)[kBSegs],
                                                            unsigned long long (*segP)[kBSegs]) {
     const int lane = tid & 31, warp = tid >> 5;
     const int v0 = chunk * kBChunk, n = min(kBChunk, p.vocab - v0);
     const float* tp = row_ptr(p, d.trow) + v0;
     const float* dp = d.drow >= 0 ? row_ptr(p, d.drow) + v0 : tp;
-    constexpr int JP = kBVec / PH;
-    float v[32];  // the lane's r sums of segments j = 0..15, then its p sums
+    constexpr int JS = kBVec / SPLIT, JP = JS / PH;
+    float vr[JS], vp[JS];  // the lane's r and p sums of its part's segments
 #pragma unroll
     for (int h = 0; h < PH; ++h) {
         float4 lt[JP], ld[JP];
 #pragma unroll
         for (int jj = 0; jj < JP; ++jj) {
-            const int e = 4 * (tid + (h * JP + jj) * kBThreads);
+            const int e = 4 * (tid + (sub * JS + h * JP + jj) * kBThreads);
             lt[jj] = load4<VEC>(tp, e, n);
             if (d.drow >= 0) ld[jj] = load4<VEC>(dp, e, n);
         }
 #pragma unroll
         for (int jj = 0; jj < JP; ++jj) {
-            const int j = h * JP + jj;
             float4 r, pw;
             weights4(lt[jj], d.drow >= 0 ? ld[jj] : lt[jj], d, p.c2, r, pw);
-            v[j] = sum4f(r);
-            v[kBVec + j] = sum4f(pw);
+            vr[h * JP + jj] = sum4f(r);
+            vp[h * JP + jj] = sum4f(pw);
         }
     }
+    float v[32];  // segment j's r sum at v[j], its p sum at v[16 + j] (0 outside the part)
+#pragma unroll
+    for (int j = 0; j < kBVec; ++j) {
+        v[j] = 0.f;
+        v[kBVec + j] = 0.f;
+    }
+#pragma unroll
+    for (int q = 0; q < SPLIT; ++q)
+        if (q == sub)
+#pragma unroll
+            for (int jj = 0; jj < JS; ++jj) {
+                v[q * JS + jj] = vr[jj];
+                v[kBVec + q * JS + jj] = vp[jj];
+            }
     const unsigned long long f = to_fix(reduce_scatter32(v, lane));  // lane j: segment j's r; 16 + j: its p
     if (lane < kBSegs) segR[warp][lane] = f;
     else segP[warp][lane - kBSegs] = f;
     return f;
 }
 
-// ---- 3. the draw (T > 0): chunk masses, then the last chunk of the sequence finds the entry
-template <bool VEC, int PH>
-__global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchParams p) {
+// ---- 3. the draw (T > 0): the sequence's decisions, chunk-part masses, then the last part of the
+// sequence finds the entry.  One CTA per (sequence, chunk, part): SPLIT parts of 16384 / SPLIT entries
+// per chunk when the sequences' chunks alone would leave SMs idle.
+template <bool VEC, int PH, int SPLIT>
+__global__ void __launch_bounds__(kBThreads, SPLIT > 1 ? 2 : PH) batch_draw_kernel(const BatchParams p) {
     __shared__ unsigned long long segR[kBThreads / 32][kBSegs], segP[kBThreads / 32][kBSegs];
     __shared__ int last_sh, cstar_sh, jstar_sh, wstar_sh, use_r_sh;
     __shared__ unsigned long long off_sh, base_sh;
+    __shared__ DrawPair d_sh;
     griddep_launch_dependents();
     griddep_wait();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
-    const int s = blockIdx.x / p.chunks, chunk = blockIdx.x - s * p.chunks;
-    const DrawPair d = load_draw(p.drawrec + 2 * s);
+    const int units = p.chunks * SPLIT;  // parts of the sequence's draw, in entry order
+    const int s = blockIdx.x / units, unit = blockIdx.x - s * units;
+    const int chunk = unit / SPLIT, sub = unit - chunk * SPLIT;
+    if (warp == 0) decide_draw(p, s, lane, unit == 0, &d_sh);
+    __syncthreads();
+    const DrawPair d = d_sh;
     constexpr int kSeg = kBThreads / 32 * kBSegs;  // 128 segments per chunk
+    constexpr int kJS = kBVec / SPLIT;             // segment rows j of one part
     static_assert(kBSegs == 16 && 2 * kSeg == kBThreads, "one segment mass per thread");
-    const unsigned long long f = chunk_masses<VEC, PH>(p, d, chunk, tid, segR, segP);
-    if (p.chunks > 1) {  // the segment masses, for the last CTA should the crossing fall in this chunk
+    const unsigned long long f = chunk_masses<VEC, PH, SPLIT>(p, d, chunk, sub, tid, segR, segP);
+    if (p.chunks > 1 || SPLIT > 1) {  // this part's segment masses, for the last CTA should the crossing fall here
         unsigned long long* segm = p.segm + ((size_t)s * p.chunks + chunk) * 2 * kSeg;
-        segm[(lane < kBSegs ? 0 : kSeg) + warp * kBSegs + (lane & (kBSegs - 1))] = f;  // segR / segP layout
+        if ((lane & (kBSegs - 1)) / kJS == sub)
+            segm[(lane < kBSegs ? 0 : kSeg) + warp * kBSegs + (lane & (kBSegs - 1))] = f;  // segR / segP layout
     }
     __syncthreads();
     if (warp == 0) {
@@ -379,19 +425,19 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
             P += __shfl_xor_sync(0xffffffffu, P, o);
         }
         if (lane == 0) {
-            p.ctot[(size_t)s * p.chunks + chunk] = make_ulonglong2(R, P);
-            // release (cumulative through the barrier): this chunk's total and every thread's segment
-            // mass before the ticket; acquire: the last CTA sees every chunk's
-            last_sh = ticket_acq_rel(p.tickets + s) == p.chunks - 1;
+            p.ctot[(size_t)s * units + unit] = make_ulonglong2(R, P);
+            // release (cumulative through the barrier): this part's total and every thread's segment
+            // mass before the ticket; acquire: the last CTA sees every part's
+            last_sh = ticket_acq_rel(p.tickets + s) == units - 1;
         }
     }
     __syncthreads();
     if (!last_sh) return;
-    // ---- every chunk is in: the distribution, the threshold and the crossing chunk (exact sums)
+    // ---- every part is in: the distribution, the threshold and the crossing part (exact sums)
     if (warp == 0) {
         unsigned long long R = 0, P = 0;
-        for (int c = lane; c < p.chunks; c += 32) {
-            const ulonglong2 x = __ldcg(&p.ctot[(size_t)s * p.chunks + c]);
+        for (int c = lane; c < units; c += 32) {
+            const ulonglong2 x = __ldcg(&p.ctot[(size_t)s * units + c]);
             R += x.x;
             P += x.y;
         }
@@ -408,11 +454,11 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
         const unsigned long long thr = __umul64hi(__float2ull_rn(u * 18446744073709551616.f), total);
         int cstar = -1;
         unsigned long long below = 0;
-        for (int c0 = 0; c0 < p.chunks && cstar < 0; c0 += 32) {  // chunks in order, 32 at a time
+        for (int c0 = 0; c0 < units && cstar < 0; c0 += 32) {  // parts in entry order, 32 at a time
             const int c = c0 + lane;
             unsigned long long x = 0;
-            if (c < p.chunks) {
-                const ulonglong2 t = __ldcg(&p.ctot[(size_t)s * p.chunks + c]);
+            if (c < units) {
+                const ulonglong2 t = __ldcg(&p.ctot[(size_t)s * units + c]);
                 x = use_r ? t.x : t.y;
             }
             const unsigned long long incl = warp_incl_scan(x, lane) + below;
@@ -438,12 +484,15 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
         }
     }
     __syncthreads();
-    const int cstar = cstar_sh;
+    const int ustar = cstar_sh;                                  // the crossing part
+    const int cstar = ustar < 0 ? -1 : ustar / SPLIT;            // its chunk
     if (cstar >= 0) {
-        // ---- the crossing chunk's segment masses (stored by its CTA), then the segment
-        if (cstar != chunk) {
+        // ---- the crossing part's segment masses (stored by its CTA; this CTA's own are in shared memory,
+        // the rest of its chunk's at 0), then the segment
+        if (ustar != unit) {
             const unsigned long long* sm = p.segm + ((size_t)s * p.chunks + cstar) * 2 * kSeg;
-            const unsigned long long x = __ldcg(sm + tid);
+            const int j = (tid & (kSeg - 1) & (kBSegs - 1));  // layout [r / p][warp][j]
+            const unsigned long long x = j / kJS == ustar - cstar * SPLIT ? __ldcg(sm + tid) : 0ull;
             if (tid < kSeg) (&segR[0][0])[tid] = x;
             else (&segP[0][0])[tid - kSeg] = x;
             __syncthreads();
@@ -528,10 +577,9 @@ __global__ void __launch_bounds__(kBThreads, PH) batch_draw_kernel(const BatchPa
 size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
     const size_t chunks = ((size_t)vocab + kBChunk - 1) / kBChunk;
     const size_t rows = 2 * (size_t)total_draft + num_seqs;
-    const size_t segm = chunks > 1 ? (size_t)num_seqs * chunks * 2 * 128 * sizeof(unsigned long long) : 0;
-    return align_up(rows * chunks * sizeof(float2), 256) + align_up(rows * sizeof(float2), 256) +
-           align_up((size_t)num_seqs * 2 * sizeof(float4), 256) +
-           align_up((size_t)num_seqs * chunks * sizeof(ulonglong2), 256) + align_up(segm, 256);
+    const size_t segm = (size_t)num_seqs * chunks * 2 * 128 * sizeof(unsigned long long);
+    return align_up(rows * chunks * sizeof(float2), 256) +
+           align_up((size_t)num_seqs * chunks * kMaxDrawSplit * sizeof(ulonglong2), 256) + align_up(segm, 256);
 }
 
 namespace {
@@ -555,12 +603,16 @@ int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
     int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
     if (rc != BP_OK) return rc;
-    rc = launch_pdl(batch_decide_kernel<GREEDY>, (unsigned)((p.num_seqs + kBThreads / 32 - 1) / (kBThreads / 32)), p,
-                    stream);
-    if (rc != BP_OK || GREEDY) return rc;
-    const unsigned draw_ctas = (unsigned)(p.num_seqs * p.chunks);
-    return draw_ctas > (unsigned)sm_count ? launch_pdl(batch_draw_kernel<VEC, 2>, draw_ctas, p, stream)
-                                          : launch_pdl(batch_draw_kernel<VEC, 1>, draw_ctas, p, stream);
+    if (GREEDY)
+        return launch_pdl(batch_decide_kernel, (unsigned)((p.num_seqs + kBThreads / 32 - 1) / (kBThreads / 32)), p,
+                          stream);
+    // the draw (with the decisions): its chunks cut into 4 or 2 parts while every CTA stays in the first
+    // wave (two CTAs per SM: the sequences' chunks alone would leave SMs idle), else whole chunks
+    const long long draw = (long long)p.num_seqs * p.chunks;
+    if (draw * 4 <= 2LL * sm_count) return launch_pdl(batch_draw_kernel<VEC, 1, 4>, (unsigned)(draw * 4), p, stream);
+    if (draw * 2 <= 2LL * sm_count) return launch_pdl(batch_draw_kernel<VEC, 1, 2>, (unsigned)(draw * 2), p, stream);
+    return draw > sm_count ? launch_pdl(batch_draw_kernel<VEC, 2, 1>, (unsigned)draw, p, stream)
+                           : launch_pdl(batch_draw_kernel<VEC, 1, 1>, (unsigned)draw, p, stream);
 }
 }  // namespace
 
@@ -586,12 +638,8 @@ int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* s
     uint8_t* w = static_cast<uint8_t*>(scratch);
     p.part = reinterpret_cast<float2*>(w);
     w += align_up(rows * chunks * sizeof(float2), 256);
-    p.rowstat = reinterpret_cast<float2*>(w);
-    w += align_up(rows * sizeof(float2), 256);
-    p.drawrec = reinterpret_cast<float4*>(w);
-    w += align_up((size_t)a.num_seqs * 2 * sizeof(float4), 256);
     p.ctot = reinterpret_cast<ulonglong2*>(w);
-    w += align_up((size_t)a.num_seqs * chunks * sizeof(ulonglong2), 256);
+    w += align_up((size_t)a.num_seqs * chunks * kMaxDrawSplit * sizeof(ulonglong2), 256);
     p.segm = reinterpret_cast<unsigned long long*>(w);
     p.tickets = tickets;
     p.err = a.err_word;

@@ -70,8 +70,8 @@ struct AttnParams {
     const int32_t* block_table;
     int pages_per_seq, page_shift;
     // flat split: partial (O, m, l) slots in the workspace, two per CTA, slot_rows rows each; and one
-    // work entry per CTA for the merge: (sequence, query tile, first tile, all tiles) of the cut unit
-    // whose first tile the CTA holds, or sequence -1
+    // work entry (two int4) per CTA for the merge: (first tile, end tile, all tiles, rows) and (first
+    // query row, query tile) of the cut unit whose first tile the CTA holds, or first tile -1
     float* part;
     int4* work;
     int slot_rows;
@@ -524,10 +524,13 @@ __global__ void __launch_bounds__(kThreads, 1)
 
     if (is_softmax) {
         int J = 0, nq = 0;
-        int4 entry = make_int4(-1, 0, 0, 0);  // flat split: this CTA's work entry for the merge
+        int4 entry = make_int4(-1, 0, 0, 0), entry2 = make_int4(0, 0, 0, 0);  // flat split: the merge's work entry
         for (int t = t_begin; t < t_end && !failed;) {
             const Seg g = seg_at(t, t == t_begin);
-            if (FLAT && !g.whole && g.jt0 == 0) entry = make_int4(g.s, g.mt, t, T);  // a cut unit that starts here
+            if (FLAT && !g.whole && g.jt0 == 0) {  // a cut unit that starts here
+                entry = make_int4(t, t + cdiv(g.n, kTileN), T, min(min(kM, g.B * G - g.mt * kM), p.slot_rows));
+                entry2 = make_int4(g.q0, g.mt, 0, 0);
+            }
             t += seg_len(g);
             const int row0 = g.mt * kM;
             m_valid = min(kM, g.B * G - row0);
@@ -679,7 +682,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             }
         }
         if (failed) raise_error(p.err, kErrTimeout);
-        if (FLAT && tid == 64) p.work[blockIdx.x] = entry;
+        if (FLAT && tid == 64) {
+            p.work[2 * blockIdx.x] = entry;
+            p.work[2 * blockIdx.x + 1] = entry2;
+        }
     }
 
     if (!FLAT) {
@@ -784,8 +790,8 @@ __global__ void __launch_bounds__(kThreads, 1)
 // (O, m, l) of the unit's CTAs in order -- O = sum_j 2^(m_j - M) O_j / sum_j 2^(m_j - M) l_j, M the
 // largest m_j, as a running merge over batches of kCombBatch partials whose loads are all in flight --
 // and writes the bf16 output chunk (and the row's log-sum-exp).
-constexpr int kCombRows = 16;
-constexpr int kCombThreads = kCombRows * kD / 4;  // 512: one 16-byte chunk of a row each
+constexpr int kCombRows = 8;
+constexpr int kCombThreads = kCombRows * kD / 4;  // 256: one 16-byte chunk of a row each
 constexpr int kCombBatch = 8;
 __global__ void __launch_bounds__(kCombThreads) attn_combine_kernel(const AttnParams p, int grid_main) {
     __shared__ int32_t gstart[kAttnFlatMaxGrid + 1];  // the CTA groups' ranges: group j has [gstart[j], gstart[j+1])
@@ -795,16 +801,11 @@ __global__ void __launch_bounds__(kCombThreads) attn_combine_kernel(const AttnPa
     const int G = p.group;
     const int chunks = (p.slot_rows + kCombRows - 1) / kCombRows;
     const int c = blockIdx.x / chunks, r = blockIdx.x - c * chunks;
-    const int4 wk = __ldcg(p.work + c);
+    const int4 wk = __ldcg(p.work + 2 * c), wk2 = __ldcg(p.work + 2 * c + 1);
     if (wk.x < 0) return;  // CTA c holds no cut unit's first tile (uniform per CTA)
-    const int s = wk.x, mt = wk.y, U0 = wk.z, T = wk.w;
+    const int U0 = wk.x, U1 = wk.y, T = wk.z, rows = wk.w, q0 = wk2.x, mt = wk2.y;
     const int h = c % p.num_kv_heads;
-    const int q0 = p.num_seqs == 1 ? 0 : __ldg(p.cu_q + s);
-    const int B = p.num_seqs == 1 ? p.total_q : __ldg(p.cu_q + s + 1) - q0;
-    const int n = p.num_seqs == 1 ? p.total_kv : __ldg(p.cu_kv + s + 1) - __ldg(p.cu_kv + s);
-    const int rows = min(min(kM, B * G - mt * kM), p.slot_rows);
     if (r * kCombRows >= rows) return;  // uniform per CTA
-    const int U1 = U0 + cdiv(n, kTileN);
     const int ngroups = grid_main / p.num_kv_heads;
     for (int j = tid; j <= ngroups; j += kCombThreads) gstart[j] = (int)((long long)j * T / ngroups);
     __syncthreads();
@@ -958,7 +959,7 @@ int flat_slot_rows(int max_q_len, int group) {
 size_t attention_flat_scratch_bytes(int max_q_len, int group) {
     if (max_q_len < 1 || group < 1) return 0;
     return (size_t)2 * kAttnFlatMaxGrid * flat_slot_rows(max_q_len, group) * (kD + 2) * sizeof(float) +
-           (size_t)kAttnFlatMaxGrid * sizeof(int4);
+           (size_t)2 * kAttnFlatMaxGrid * sizeof(int4);
 }
 
 int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStream_t stream) {
@@ -1091,17 +1092,20 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     // head and per SM (at most kAttnFlatMaxGrid in all, and no more groups than one head has tiles); units
     // cut between groups are merged by a second kernel.  It needs the Q tile by TMA, the sequences'
     // offsets in shared memory and the workspace's partial slots and work entries.  Measured on this GPU,
-    // it gains only where the cluster split leaves SMs idle and every CTA of the flat split streams a
-    // long run (8 x 32K keys: 171 vs 175 us); with short runs the second kernel and the stretch
-    // boundaries cost more than the idle SMs (1 x 2K keys: 13.4 vs 9.3 us).  BP_ATTENTION_SPLIT=flat or
-    // =cluster overrides the choice (for tests and measurements).
+    // it gains where the cluster split leaves SMs idle while every CTA of the flat split streams a long
+    // run (8 x 32K keys: 170 vs 175 us), and where the cluster split needs three or more waves (64 x 528
+    // keys: 46 vs 50 us); elsewhere the second kernel and the stretch boundaries cost more than the idle
+    // SMs (1 x 2K keys: 13.8 vs 9.3 us; 16 x 4K: 60 vs 52 us; the ragged 32: 109 vs 100 us).
+    // BP_ATTENTION_SPLIT=flat or =cluster overrides the choice (for tests and measurements).
     const long long tiles_bound = (long long)a.num_seqs * m_tiles * max_tiles;
     const int ngroups = (int)std::min<long long>(std::min(dev.sm_count, kAttnFlatMaxGrid) / a.num_kv_heads,
                                                  tiles_bound);
     const int flat_grid = ngroups * a.num_kv_heads;
     const bool flat_ok = q_tma && a.num_seqs <= kMaxOrderedSeqs && a.scratch != nullptr &&
                          a.scratch_bytes >= attention_flat_scratch_bytes(a.max_q_len, G) && ngroups >= 1;
-    bool flat = flat_ok && units * cs * 10 <= (long long)dev.sm_count * 9 && tiles_bound >= 32LL * ngroups;
+    const long long cluster_ctas = units * cs;
+    bool flat = flat_ok && ((cluster_ctas * 10 <= 9LL * dev.sm_count && tiles_bound >= 64LL * ngroups) ||
+                            cluster_ctas >= 3LL * dev.sm_count);
     if (const char* force = getenv("BP_ATTENTION_SPLIT")) {
         if (strcmp(force, "flat") == 0) flat = flat_ok;
         else if (strcmp(force, "cluster") == 0) flat = false;

@@ -66,17 +66,17 @@ def _align(x, a=256):
                                         (2, 23, 151936), (3, 23, 151936), (1, 0, 5), (32, 470, 151936),
                                         (200000, 200000, 16), (9, 100, 16385)])
 def test_acceptance_workspace_follows_the_path_choice(lib, s, td, vocab):
-    """The workspace carries the throughput kernels' regions (chunk and row statistics, draw records,
-    chunk totals, segment masses) exactly when either temperature takes those kernels: this pins the
-    tests' mirror of the library's choice (accept_uses_batch) to the library, on the CPU."""
+    """The workspace carries the throughput kernels' regions (chunk statistics, the totals of the
+    draw's chunk parts (up to 4 per chunk), segment masses) exactly when either temperature takes
+    those kernels: this pins the tests' mirror of the library's choice (accept_uses_batch) to the
+    library, on the CPU."""
     from _gpu import accept_uses_batch
 
     blocks = (td + 1,) + (1,) * (s - 1)
     cluster = 256 + _align(4 * s) + _align(4 * td) + _align(4 * (td + s))
     chunks = -(-vocab // 16384)
     rows = 2 * td + s
-    batch = (_align(rows * chunks * 8) + _align(rows * 8) + _align(s * 32) + _align(s * chunks * 16)
-             + _align(s * chunks * 256 * 8 if chunks > 1 else 0))
+    batch = _align(rows * chunks * 8) + _align(s * chunks * 4 * 16) + _align(s * chunks * 256 * 8)
     may = accept_uses_batch(blocks, vocab, 0.0) or accept_uses_batch(blocks, vocab, 1.0)
     assert bp.spec_accept_workspace_size(s, td, vocab) == cluster + (batch if may else 0)
 

@@ -72,6 +72,20 @@ def test_planted_long_prefixes(temp):
     assert n_acc.max() >= 10
 
 
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_blocks_longer_than_a_warp_batch(temp):
+    """Blocks of up to 64 positions on the throughput kernels, drafts mostly copies of their target rows:
+    first rejections past the first 32 positions (the decisions take positions 32 at a time) and bonus
+    draws after 63 accepted drafts."""
+    blocks = (64, 40, 33, 1, 64, 2) * 3
+    assert accept_uses_batch(blocks, 32000, temp)
+    w = wl.custom(seed=47, ctx=(0,) * len(blocks), block=blocks, vocab=32000)
+    inp = wl.accept_inputs(w, temp, planted_match=0.97)
+    compare_accept(inp, temp)
+    n_acc, _, _, _ = run_accept(inp, temp)
+    assert n_acc.max() > 32
+
+
 @pytest.mark.parametrize("batch", [False, True])
 @pytest.mark.parametrize("vocab", [5, 1001, 4099, 16384, 32000, 50001])
 def test_vocab_sizes_and_scalar_path(vocab, batch):

@@ -93,19 +93,20 @@ def _attn_kernels(a, split):
 
 
 def test_split_choice():
-    """Left to the library, a batch-1 verify (2K keys) takes the cluster split and 8 sequences of 16K keys
-    the flat split (two kernels); a 256-byte workspace always keeps the cluster split."""
+    """Left to the library, a batch-1 verify (2K keys) takes the cluster split (one kernel) and 64 short
+    sequences, which would need four waves of the cluster split, the flat split (two kernels); each can
+    be forced."""
     _attn_kernels(wl.attention_inputs(wl.custom(seed=1, ctx=(100,), block=(4,), num_q_heads=32, num_kv_heads=8)),
                   "auto")  # the profiler's first session may miss kernels while it starts
     small = wl.attention_inputs(wl.get("qwen3_4b"))
     names = _attn_kernels(small, "auto")
     assert not any("attn_combine_kernel" in x for x in names) and any("attn_bf16_tc_kernel" in x for x in names)
     assert any("attn_combine_kernel" in x for x in _attn_kernels(small, "flat"))
-    long8 = wl.attention_inputs(wl.custom(seed=9, ctx=(16384,) * 8, block=(16,) * 8, num_q_heads=32,
-                                          num_kv_heads=8))
-    assert any("attn_combine_kernel" in x for x in _attn_kernels(long8, "auto"))
-    assert not any("attn_combine_kernel" in x for x in _attn_kernels(long8, "cluster"))
-    err, lerr = attention_errors(*run_attention(long8, CAUSAL), long8, CAUSAL, [0, 7], kv_head=3)
+    many = wl.attention_inputs(wl.custom(seed=9, ctx=(512,) * 64, block=(16,) * 64, num_q_heads=32,
+                                         num_kv_heads=8))
+    assert any("attn_combine_kernel" in x for x in _attn_kernels(many, "auto"))
+    assert not any("attn_combine_kernel" in x for x in _attn_kernels(many, "cluster"))
+    err, lerr = attention_errors(*run_attention(many, CAUSAL), many, CAUSAL, [0, 17, 63])
     assert err <= ATTN_TOL and lerr <= LSE_TOL
 
 
