@@ -1,4 +1,10 @@
-"""Builds libblockpilot.so in-tree with nvcc for sm_103a (translation units compiled in parallel)."""
+"""Builds libblockpilot.so in-tree with nvcc for sm_103a (translation units compiled in parallel).
+
+Beside it, libblockpilot_shortwait.so: the same sources built with BP_TEST_SHORT_WAITS, where every
+bounded wait for work to arrive is a single non-blocking test.  It exists only for the test of the
+kernels' wind-down path (an expired wait reports BP_ERR_TIMEOUT, drains the kernel's own copies and
+tensor-core operations, releases tensor memory and returns); nothing else loads it.
+"""
 from __future__ import annotations
 
 import concurrent.futures as cf
@@ -10,6 +16,7 @@ PKG = os.path.dirname(os.path.abspath(__file__))
 CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libblockpilot.so")
+TEST_LIB = os.path.join(PKG, "libblockpilot_shortwait.so")  # test-only build (see above)
 SOURCES = ("api.cu", "attention.cu", "accept.cu", "accept_batch.cu", "policy.cu", "verify_epilogue.cu", "tau.cu", "commit.cu")
 HEADERS = ("common.cuh", "ptx_sm103.cuh", "softmax_math.cuh")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
@@ -31,29 +38,34 @@ def _inputs_mtime() -> float:
 
 
 def build(force: bool = False, verbose: bool = False) -> str:
-    """Compile and link; returns the path of the shared library."""
-    if not force and os.path.exists(LIB) and os.path.getmtime(LIB) >= _inputs_mtime():
+    """Compile and link both libraries; returns the path of the product library."""
+    stale = force or not all(os.path.exists(x) and os.path.getmtime(x) >= _inputs_mtime() for x in (LIB, TEST_LIB))
+    if not stale:
         return LIB
-    os.makedirs(BUILD, exist_ok=True)
+    os.makedirs(os.path.join(BUILD, "shortwait"), exist_ok=True)
     nvcc = _nvcc()
 
-    def compile_one(src: str) -> str:
-        obj = os.path.join(BUILD, src.replace(".cu", ".o"))
-        cmd = [nvcc, *ARCH, *FLAGS, "-c", os.path.join(CSRC, src), "-o", obj]
+    def compile_one(job) -> str:
+        src, test = job
+        obj = os.path.join(BUILD, "shortwait" if test else "", src.replace(".cu", ".o"))
+        cmd = [nvcc, *ARCH, *FLAGS, *(["-DBP_TEST_SHORT_WAITS"] if test else []), "-c", os.path.join(CSRC, src), "-o",
+               obj]
         res = subprocess.run(cmd, capture_output=True, text=True)
         if res.returncode != 0:
-            raise RuntimeError(f"nvcc failed on {src}:\n{res.stdout}\n{res.stderr}")
+            raise RuntimeError(f"nvcc failed on {src}{' (short waits)' if test else ''}:\n{res.stdout}\n{res.stderr}")
         if verbose:
             print(res.stdout + res.stderr)
         return obj
 
-    with cf.ThreadPoolExecutor(max_workers=len(SOURCES)) as ex:
-        objs = list(ex.map(compile_one, SOURCES))
-    tmp = LIB + f".tmp{os.getpid()}"
-    res = subprocess.run([nvcc, *ARCH, "-shared", *objs, "-o", tmp], capture_output=True, text=True)
-    if res.returncode != 0:
-        raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
-    os.replace(tmp, LIB)
+    jobs = [(src, test) for test in (False, True) for src in SOURCES]
+    with cf.ThreadPoolExecutor(max_workers=len(jobs)) as ex:
+        objs = list(ex.map(compile_one, jobs))
+    for lib, part in ((LIB, objs[:len(SOURCES)]), (TEST_LIB, objs[len(SOURCES):])):
+        tmp = lib + f".tmp{os.getpid()}"
+        res = subprocess.run([nvcc, *ARCH, "-shared", *part, "-o", tmp], capture_output=True, text=True)
+        if res.returncode != 0:
+            raise RuntimeError(f"link failed:\n{res.stdout}\n{res.stderr}")
+        os.replace(tmp, lib)
     return LIB
 
 

@@ -111,9 +111,14 @@ __device__ __forceinline__ void fetch_range(float4* dst, const float* row, int f
         __syncwarp();
     }
 }
+// Waits for the warp's copy; if the wait expires, the error is recorded and the copy is still waited
+// out (drain budget): no copy may land in shared memory after the CTA has moved on or left.
 template <bool VEC>
 __device__ __forceinline__ void wait_range(uint64_t* bar, int nw, unsigned int* err) {
-    if (VEC && nw > 0 && !mbar_wait(bar, 0, kWaitBudget)) raise_error(err, kErrTimeout);
+    if (VEC && nw > 0 && !mbar_wait(bar, 0, kWaitBudget)) {
+        raise_error(err, kErrTimeout);
+        mbar_wait(bar, 0, kDrainBudget);
+    }
 }
 
 // Scaled maximum l*c2 of a lane's entries of a range (-inf if none is finite), then the weights

@@ -425,8 +425,8 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (!ok) raise_error(p.err, kErrTimeout);
             // no copy may still be in flight when the CTA leaves
             for (int j = max(0, J - kStages); j < J; ++j)
-                if (!mbar_wait(&bar_kv_full[j % kStages], (j / kStages) & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
-            if (nq > 0 && !mbar_wait(&bar_q_full, (nq - 1) & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
+                if (!mbar_wait(&bar_kv_full[j % kStages], (j / kStages) & 1, kDrainBudget)) raise_error(p.err, kErrTimeout);
+            if (nq > 0 && !mbar_wait(&bar_q_full, (nq - 1) & 1, kDrainBudget)) raise_error(p.err, kErrTimeout);
         }
     } else if (warp == 1) {
         // ================= MMA issuer
@@ -482,7 +482,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             if (J > 0) {
                 // no MMA may still be writing tensor memory when it is released
                 umma_commit(&bar_o_done);
-                if (!mbar_wait(&bar_o_done, nq & 1, kWaitBudget)) raise_error(p.err, kErrTimeout);
+                if (!mbar_wait(&bar_o_done, nq & 1, kDrainBudget)) raise_error(p.err, kErrTimeout);
             }
         }
     }
@@ -703,6 +703,7 @@ __global__ void __launch_bounds__(kThreads, 1)
             cg::cluster_group cluster = cg::this_cluster();
             float* opart = reinterpret_cast<float*>(sKV);
             float2* row_ml = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float));
+            __syncthreads();  // the producer has drained the ring (after an expired wait copies may still land)
             if (is_softmax) {
                 if (row_active) {
 #pragma unroll

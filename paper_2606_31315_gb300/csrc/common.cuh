@@ -20,8 +20,18 @@ static_assert(sizeof(WorkspaceHeader) == 256, "workspace header is 256 bytes");
 
 enum : unsigned int { kErrTimeout = 1u, kErrDeviceArg = 2u };
 
-// Cycle budget of every bounded device-side wait (about one second at 2 GHz).
+// Cycle budget of every bounded device-side wait for work to arrive (about one second at 2 GHz).  A
+// wait that expires records kErrTimeout and the kernel winds down; before a CTA leaves it waits out its
+// own copies and tensor-core operations still in flight with kDrainBudget, so nothing writes into its
+// shared or tensor memory after it.  BP_TEST_SHORT_WAITS (a test-only build of the library) makes every
+// such wait a single non-blocking test, so that the tests can take the wind-down path on purpose; the
+// drains keep their budget.
+#ifdef BP_TEST_SHORT_WAITS
+constexpr long long kWaitBudget = 0;
+#else
 constexpr long long kWaitBudget = 2000000000LL;
+#endif
+constexpr long long kDrainBudget = 2000000000LL;
 
 __device__ __forceinline__ void raise_error(unsigned int* err_word, unsigned int bits) {
     if (err_word) atomicOr(err_word, bits);

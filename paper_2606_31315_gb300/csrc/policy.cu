@@ -274,7 +274,8 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
         static_assert(!RING || (S >= 2 && S <= kTcStages && S <= kTcMaxAtoms), "ring depth");
         const uint32_t stage_bytes = (uint32_t)(kTcAtomBytes + npad * 128);
         if (tid == 0) {  // producer: W1 and x atoms through the ring
-            for (int j = 0; j < na; ++j) {
+            int j = 0;
+            for (; j < na; ++j) {
                 const int st = j % S;
                 if (j >= S && !mbar_wait(&bar_empty[st], ((j / S) - 1) & 1, kWaitBudget)) {
                     raise_error(p.err, kErrTimeout);
@@ -284,6 +285,8 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
                 tma_load_2d(sW + st * kTcAtomBytes, &w1map, &bar_w[st], (a0 + j) * kTcAtom, m0);
                 tma_load_2d(sX + st * npad * 128, &xmap, &bar_w[st], (a0 + j) * kTcAtom, n0);
             }
+            if (j < na)  // wound down early: the copies still in flight land before the CTA moves on
+                for (int jj = max(0, j - S); jj < j; ++jj) mbar_wait(&bar_w[jj % S], (jj / S) & 1, kDrainBudget);
         } else if (tid == 32) {  // MMA issuer
             if (na > 0) {
                 const uint32_t idesc = idesc_bf16_f32(kTcM, npad, false, false);
@@ -370,7 +373,10 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
                     umma_ss(tmem, smem_desc(wa + kk * 32, 16, 1024, kSwizzle128B),
                             smem_desc(xa + kk * 32, 16, 1024, kSwizzle128B), idesc, (a | kk) ? 1u : 0u);
             }
-            if (!ok) raise_error(p.err, kErrTimeout);
+            if (!ok) {  // every W1 atom's copy lands before the CTA moves on
+                raise_error(p.err, kErrTimeout);
+                for (int a = 0; a < na; ++a) mbar_wait(&bar_w[a], 0, kDrainBudget);
+            }
             umma_commit(&bar_mma);
         }
     }
@@ -379,7 +385,7 @@ __global__ void __launch_bounds__(kTcThreads) policy_tc_kernel(const __grid_cons
 #pragma unroll
     for (int e = 0; e < kTcMaxN; ++e) d[e] = 0.f;
     if (na > 0) {
-        if (!mbar_wait(&bar_mma, 0, kWaitBudget)) raise_error(p.err, kErrTimeout);
+        if (!mbar_wait(&bar_mma, 0, kDrainBudget)) raise_error(p.err, kErrTimeout);
         tc_fence_after();
 #pragma unroll
         for (int c0 = 0; c0 < kTcMaxN; c0 += 16) {

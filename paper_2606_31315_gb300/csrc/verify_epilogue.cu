@@ -268,7 +268,7 @@ __global__ void __launch_bounds__(kVeThreads, 1)
             }
             if (issued < J)  // wound down early: let the copies still in flight land before exiting
                 for (int j = max(0, issued - STG); j < issued; ++j)
-                    mbar_wait(&wfull[j % STG], (j / STG) & 1, kWaitBudget);
+                    mbar_wait(&wfull[j % STG], (j / STG) & 1, kDrainBudget);
         }
     } else if (warp == 2) {
         // ---- state producer: row n's 16-byte chunk ch of atom a goes to chunk ch ^ (n & 7) of row n
@@ -332,7 +332,7 @@ __global__ void __launch_bounds__(kVeThreads, 1)
                 if (a0 + APS == p.atoms) umma_commit(&acc_full[t]);
             }
             umma_commit(&mma_done);  // every MMA issued is complete before tensor memory is released
-            mbar_wait(&mma_done, 0, kWaitBudget);
+            mbar_wait(&mma_done, 0, kDrainBudget);
         }
     } else if (warp == 3) {
         // ---- sequence offsets (read by every warp after grid barrier 1), then the draft tokens held
