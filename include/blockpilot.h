@@ -191,13 +191,16 @@ BP_API int bp_spec_accept(const float* target_logits, const float* draft_logits,
  *     library, held on every GPU that loads the library until the process exits;
  *   - the three throughput kernels run only when their scratch fits in the array too; other
  *     problems large enough for them run on the single kernel;
- *   - problems whose single-kernel scratch would exceed it return BP_ERR_WORKSPACE (about 8
- *     bytes per target row plus 4 per sequence, so roughly a million target rows fit);
+ *   - problems whose single-kernel scratch would exceed it return BP_ERR_WORKSPACE (8 bytes per
+ *     target row, i.e. per total_draft + num_seqs, so about a million target rows fit);
  *   - device-detected errors are OR-ed into *device_error (a caller-owned device word, may be
  *     NULL to drop them) instead of a workspace: 1 = a wait timed out, 2 = a draft token id
  *     outside [0, vocab);
- *   - the first call on each device looks up the array's device address (cached afterwards);
- *   - every call clears the array's per-sequence counters on `stream` before its kernel runs;
+ *   - the first call on each device may load the library's acceptance module (placing the
+ *     array in device memory) and looks up the array's device address (cached afterwards): make
+ *     that first call during set-up, before any stream capture;
+ *   - every call clears the array's per-sequence counters on `stream` before its kernel runs (the
+ *     kernels leave them at zero, so this only matters after a call that did not finish normally);
  *     calls that run concurrently on the GPU (unordered streams) share the array and race.
  * ------------------------------------------------------------------------------- */
 #define BP_NOALLOC_SCRATCH_BYTES (8u << 20)

@@ -227,3 +227,25 @@ def test_build_compiles_every_source():
     headers = sorted(f for f in os.listdir(csrc) if f.endswith(".cuh"))
     assert sorted(_build.SOURCES) == on_disk
     assert sorted(_build.HEADERS) == headers
+
+
+def test_noalloc_host_validation_needs_no_gpu(lib):
+    """bp_spec_accept_noalloc checks its arguments as bp_spec_accept does, before touching CUDA."""
+    vp, i32, f32 = ctypes.c_void_p, ctypes.c_int, ctypes.c_float
+    lib.bp_spec_accept_noalloc.argtypes = [vp, vp, vp, vp, i32, i32, i32, f32, vp, vp, vp, vp, vp, vp, vp]
+    lib.bp_spec_accept_noalloc.restype = i32
+    fake = vp(0x10000)
+
+    def call(target=fake, draft=fake, tokens=fake, cu=fake, s=1, td=15, vocab=1000, temp=1.0, ua=fake, us=fake,
+             n_acc=fake, out=fake):
+        return lib.bp_spec_accept_noalloc(target, draft, tokens, cu, s, td, vocab, f32(temp), ua, us, n_acc, out,
+                                          None, None, None)
+    assert call(s=0) == 0                            # nothing to compute
+    assert call(s=-1) == 1 and call(td=-1) == 1 and call(vocab=0) == 1
+    assert call(target=None) == 1 and call(cu=None) == 1 and call(n_acc=None) == 1 and call(out=None) == 1
+    assert call(tokens=None) == 1                    # drafts without their tokens
+    assert call(temp=-1.0) == 1 and call(temp=float("inf")) == 1
+    assert call(us=None) == 1 and call(draft=None) == 1 and call(ua=None) == 1  # T > 0 needs them
+    assert call(temp=0.0, draft=None, ua=None, us=None) == 3  # greedy needs none of them; then no device
+    assert call(s=1 << 20, td=1 << 20, vocab=1 << 20) == 2   # more than 2^40 logits
+    assert call() == 3                               # valid arguments, no sm_103 device: BP_ERR_CUDA

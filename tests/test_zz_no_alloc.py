@@ -7,7 +7,8 @@ point keeps its scratch in a fixed array inside the library instead.  The test c
 the C ABI twice in a row, on two different problems (so the second call runs on whatever the
 first left in the shared array), and checks each result against bp_spec_accept with a
 caller-provided workspace: emitted tokens and accepted lengths identical, acceptance
-probabilities within 1e-5.  It also checks that a problem too large for the array is refused.
+probabilities within 1e-5.  It also checks that a problem too large for the array is refused, and
+which kernels run: the throughput kernels when their regions fit in the array, else the single one.
 """
 import ctypes
 
@@ -69,6 +70,17 @@ def _noalloc(lib, g, temp):
     return n_acc.cpu().numpy(), out.cpu().numpy(), ap.cpu().numpy()
 
 
+def _kernels(fn):
+    """Names of the GPU kernels fn() launches (a warm-up session first: the first may miss some)."""
+    from torch.profiler import ProfilerActivity, profile
+
+    for _ in range(2):
+        with profile(activities=[ProfilerActivity.CUDA]) as prof:
+            fn()
+            torch.cuda.synchronize()
+    return {e.name for e in prof.events() if "bp::" in e.name}
+
+
 def _with_workspace(g, temp):
     n_acc, out, ap = bp.spec_accept(g["target_logits"], g["draft_logits"], g["draft_tokens"], g["cu_draft"], temp,
                                     g["u_accept"], g["u_sample"])
@@ -83,10 +95,18 @@ def _same(a, b):
 
 @pytest.mark.parametrize("temp", [1.0, 0.0])
 def test_two_calls_in_a_row_match_the_workspace_entry_point(lib, temp):
-    first = _inputs("ragged", 1.0)        # 32 sequences, 530 target rows
+    first = _inputs("ragged", 1.0)        # 32 sequences, 502 target rows
     second = _inputs("qwen3_4b", temp)    # 1 sequence, 16 target rows
     _same(_noalloc(lib, first, 1.0), _with_workspace(first, 1.0))
     _same(_noalloc(lib, second, temp), _with_workspace(second, temp))
+
+
+def test_the_array_holds_the_throughput_kernels_when_they_fit(lib):
+    """The ragged batch's throughput-kernel regions (under 1 MB) fit the fixed array: those kernels run."""
+    g = _inputs("ragged", 1.0)
+    names = _kernels(lambda: _noalloc(lib, g, 1.0))
+    assert any("batch_stats_kernel" in n for n in names) and any("batch_draw_kernel" in n for n in names), names
+    assert not any("accept_kernel" in n for n in names), names
 
 
 def test_too_large_problem_is_refused(lib):
@@ -109,9 +129,9 @@ def test_too_large_problem_is_refused(lib):
 def test_large_batch_falls_back_to_the_single_kernel(lib):
     # 200000 sequences of one draft each over a 16-token vocabulary: 400000 target rows.  The
     # single kernel's scratch (tickets, ratios, row tokens: about 3.2 MB) fits in the fixed array;
-    # the throughput kernels' regions on top of it (chunk and row statistics of 600000 rows,
-    # per-sequence draw masses: about 14 MB more) do not, so the call runs the single kernel.
-    # Checked against the oracle on the first 20000 sequences.
+    # the throughput kernels' regions on top of it (chunk statistics of 600000 rows, per-sequence
+    # draw masses: about 15 MB more) do not, so the call runs the single kernel (checked by the
+    # kernels it launches).  Checked against the oracle on the first 20000 sequences.
     s, v = 200_000, 16
     rng = np.random.default_rng(81)
     tl = rng.normal(0.0, 2.0, size=(2 * s, v)).astype(np.float32)
@@ -121,6 +141,8 @@ def test_large_batch_falls_back_to_the_single_kernel(lib):
                u_sample=rng.random(s, dtype=np.float32))
     assert bp.spec_accept_workspace_size(s, s, v) > (8 << 20)  # the throughput kernels' layout is larger
     g = {k: torch.from_numpy(np.ascontiguousarray(x)).cuda() for k, x in inp.items()}
+    names = _kernels(lambda: _noalloc(lib, g, 1.0))
+    assert any("accept_kernel" in n for n in names) and not any("batch_" in n for n in names), names
     n_acc, out, ap = _noalloc(lib, g, 1.0)
     m = 20_000
     small = {k: x[: 2 * m] if k == "target_logits" else x[: m + 1] if k == "cu_draft" else x[:m]
