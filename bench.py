@@ -60,6 +60,17 @@ def peaks():
     return 6800.0, "fallback"
 
 
+def tensor_peak():
+    """Sustained dense bf16 TFLOP/s (a kernel timed inside a long run), measured or the fallback."""
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    if os.path.exists(path):
+        with open(path) as f:
+            d = json.load(f)
+        if "bf16_tflops_sustained" in d:
+            return float(d["bf16_tflops_sustained"]), "measured"
+    return 1700.0, "fallback"
+
+
 def dist_env():
     return int(os.environ.get("RANK", 0)), int(os.environ.get("WORLD_SIZE", 1)), int(os.environ.get("LOCAL_RANK", 0))
 
@@ -471,7 +482,7 @@ def run_ours(args):
     ve_cu = torch.tensor([0, td_q], dtype=torch.int32, device=dev)
     ve_ua, ve_us = torch.rand(td_q, device=dev, generator=gen), torch.rand(1, device=dev, generator=gen)
     ve_n, ve_o = torch.empty(1, dtype=torch.int32, device=dev), torch.empty(td_q + 1, dtype=torch.int32, device=dev)
-    ws_ve = bp.workspace(bp.verify_epilogue_workspace_size(1, td_q), dev)
+    ws_ve = bp.workspace(bp.verify_epilogue_workspace_size(1, td_q, w.vocab), dev)
 
     def fused(_c):
         bp.verify_epilogue(w_lm, h_t, h_d, ve_tok, ve_cu, 1.0, ve_ua, ve_us, n_accepted=ve_n, out_tokens=ve_o,
@@ -490,7 +501,44 @@ def run_ours(args):
     t_ve = time_calls(fused)
     t_unfused = time_calls(unfused)
     ve_bytes = float(w_lm.numel() * 2 + h_all.numel() * 2)
-    del w_lm, lg
+    del lg
+
+    # next row: the same LM head over the long-context batch at T=1 -- 8 sequences x 16 positions, 128
+    # target and 120 drafter states (248 rows: more logits than tensor memory holds, so the projection
+    # streams and writes the logits once; the draw reads back only its row pairs) -- beside the unfused path
+    lc = wl.get("long_context")
+    S5, g5 = lc.num_seqs, int(lc.block[0]) - 1
+    td5 = S5 * g5
+    h5_t = torch.randn(td5 + S5, lm_h, device=dev, generator=gen).to(torch.bfloat16)
+    trow5 = torch.arange(td5, device=dev) + torch.arange(td5, device=dev) // g5  # target row of draft i
+    h5_d = (h5_t[trow5].float() + torch.randn(td5, lm_h, device=dev, generator=gen) / lc.logit_std).to(torch.bfloat16)
+    tok5 = torch.randint(0, lc.vocab, (td5,), device=dev, generator=gen, dtype=torch.int32)
+    cu5 = torch.arange(0, td5 + 1, g5, dtype=torch.int32, device=dev)
+    ua5, us5 = torch.rand(td5, device=dev, generator=gen), torch.rand(S5, device=dev, generator=gen)
+    n5, o5 = torch.empty(S5, dtype=torch.int32, device=dev), torch.empty(td5 + S5, dtype=torch.int32, device=dev)
+    ws_ve5 = bp.workspace(bp.verify_epilogue_workspace_size(S5, td5, lc.vocab), dev)
+
+    def fused5(_c):
+        bp.verify_epilogue(w_lm, h5_t, h5_d, tok5, cu5, 1.0, ua5, us5, n_accepted=n5, out_tokens=o5,
+                           want_accept_prob=False, ws=ws_ve5, stream=stream)
+
+    h5_all = torch.cat([h5_t, h5_d])
+    lg5 = torch.empty(h5_all.shape[0], lc.vocab, dtype=torch.float32, device=dev)
+    ws_u5 = bp.workspace(bp.spec_accept_workspace_size(S5, td5, lc.vocab), dev)
+
+    def unfused5(_c):
+        with torch.cuda.stream(stream):
+            lg5.copy_(torch.matmul(h5_all, w_lm.t()))
+        bp.spec_accept(lg5[:td5 + S5], lg5[td5 + S5:], tok5, cu5, 1.0, ua5, us5, n_accepted=n5, out_tokens=o5,
+                       want_accept_prob=False, ws=ws_u5, stream=stream)
+
+    t_ve5 = time_calls(fused5)
+    t_unfused5 = time_calls(unfused5)
+    rows5 = h5_all.shape[0]
+    ve5_bytes = float(w_lm.numel() * 2 + h5_all.numel() * 2)  # the operation's own operands
+    ve5_hbm = ve5_bytes + rows5 * lc.vocab * 4.0 + 2 * S5 * lc.vocab * 4.0  # + logits written, draw pairs read
+    ve5_flops = 2.0 * rows5 * lc.vocab * lm_h
+    del w_lm, lg5, ws_ve5, ws_u5
 
     # next row: the decoding loop on the device -- each step runs 36 layers (Qwen3-4B) of append-the-block
     # + paged verify attention, the T=1 acceptance and the commit (lengths back to the accepted prefix,
@@ -637,6 +685,16 @@ def run_ours(args):
             traffic=committed_traffic("verify_epilogue_kernel"),
             unfused_us=round(t_unfused * 1e6, 3),
             unfused="cuBLAS bf16 GEMM to logits + fp32 cast + accept_kernel"),
+        "next1_fused_verify_epilogue_long_context_t1": dict(
+            row(t_ve5, ve5_bytes, ["lm_head_stream_kernel<false,2,true>", "lm_head_row_merge_kernel",
+                                   "batch_draw_kernel"]),
+            traffic=committed_traffic("lm_head_stream_kernel"),
+            rows=int(rows5), design_hbm_bytes=ve5_hbm,
+            design_frac=round(ve5_hbm / t_ve5 / 1e9 / peak, 4),
+            tflops=round(ve5_flops / t_ve5 / 1e12, 1),
+            tensor_frac=round(ve5_flops / t_ve5 / 1e12 / tensor_peak()[0], 4),
+            unfused_us=round(t_unfused5 * 1e6, 3),
+            unfused="cuBLAS bf16 GEMM to logits + fp32 cast + the throughput acceptance (statistics, draw)"),
         "next3_verify_loop_step_qwen3_4b_36_layers": dict(
             row(t_loop, loop_bytes, ["kv_append_kernel", "attn_bf16_tc_kernel (paged)", "accept_kernel<false,true>",
                                      "verify_commit_kernel"]),

@@ -238,7 +238,7 @@ BP_API int bp_policy_select(const void* feats, int64_t feat_row_stride, const in
 
 /* ---------------------------------------------------------------------------------
  * Verify epilogue: the LM-head projection of the final hidden states fused with the lossless
- * acceptance of bp_spec_accept, without writing the logits to memory.  Section 2.1 and the
+ * acceptance of bp_spec_accept; up to 64 rows without writing the logits to memory.  Section 2.1 and the
  * Figure 1 caption: the target scores every position of the drafted block in one pass and
  * keeps the longest accepted prefix; the distributions it compares are
  *
@@ -256,15 +256,25 @@ BP_API int bp_policy_select(const void* feats, int64_t feat_row_stride, const in
  *   draft_tokens, cu_draft, u_accept, u_sample, n_accepted, out_tokens, accept_prob: as in
  *                bp_spec_accept
  *   logits_out   [rows][vocab] fp32, may be NULL: if given, the logits are also written (rows:
- *                the target rows, then at T > 0 the drafter rows) -- for testing; it adds the
- *                write traffic the fusion exists to avoid
- * Limits (else BP_ERR_UNSUPPORTED): hidden % 64 == 0; rows = total_draft + num_seqs (+
- * total_draft at T > 0) <= 64; the vocabulary split over the SMs must leave each CTA at most
- * 16 tiles of 128 entries and tiles x (32 if rows <= 32 else 64) <= 512 tensor-memory columns
- * (152 SMs: vocab <= 155,648 at rows <= 64, 311,296 at rows <= 32).  The kernel is a
- * cooperative launch of one CTA per SM.
+ *                the target rows, then at T > 0 the drafter rows)
+ * Two paths, chosen by rows = total_draft + num_seqs (+ total_draft at T > 0):
+ *   rows <= 64: one cooperative launch of one CTA per SM keeps every logit in tensor memory; the
+ *     logits never reach memory unless logits_out asks for them (then for testing: it adds the write
+ *     traffic the fusion exists to avoid).  Limits: the vocabulary split over the SMs must leave each
+ *     CTA at most 16 tiles of 128 entries and tiles x (32 if rows <= 32 else 64) <= 512 tensor-memory
+ *     columns (152 SMs: vocab <= 155,648 at rows <= 64, 311,296 at rows <= 32).
+ *   rows > 64: the logits of that many rows do not fit on chip (the GPU's tensor memory holds about
+ *     39 MB; 248 rows of a 151,936-entry vocabulary take 151 MB), so the LM head is streamed in
+ *     256-entry passes, groups of at most 256 rows per pass over W, and every row's statistics are
+ *     formed in the projection's epilogue.  At T = 0 only the statistics leave the chip.  At T > 0
+ *     the logits are written once (into logits_out if given, else into the workspace) and only the
+ *     draw's row pair of each sequence and the logits at the drafted tokens are read back.  Any
+ *     vocabulary; W is read once per group of 256 rows.
+ * Limits (else BP_ERR_UNSUPPORTED): hidden % 64 == 0; the rows <= 64 limits above.
+ * Workspace: bp_verify_epilogue_workspace_size(num_seqs, total_draft, vocab), sized for T > 0 (at
+ * more than 64 rows it holds the [rows][vocab] fp32 logits; logits_out given, that part is unused).
  * ------------------------------------------------------------------------------- */
-BP_API size_t bp_verify_epilogue_workspace_size(int num_seqs, int total_draft);
+BP_API size_t bp_verify_epilogue_workspace_size(int num_seqs, int total_draft, int vocab);
 BP_API int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_draft, int hidden, int vocab,
                               const int32_t* draft_tokens, const int32_t* cu_draft, int num_seqs, int total_draft,
                               float temperature, const float* u_accept, const float* u_sample,

@@ -73,7 +73,7 @@ def load():
     lib.bp_policy_select_workspace_size.restype = sz
     lib.bp_policy_select.argtypes = [vp, i64, vp, i32, i32, vp, vp, i32, vp, vp, i32, vp, i32, vp, vp, vp, sz, vp]
     lib.bp_policy_select.restype = i32
-    lib.bp_verify_epilogue_workspace_size.argtypes = [i32, i32]
+    lib.bp_verify_epilogue_workspace_size.argtypes = [i32, i32, i32]
     lib.bp_verify_epilogue_workspace_size.restype = sz
     lib.bp_verify_epilogue.argtypes = [vp, vp, vp, i32, i32, vp, vp, i32, i32, f32, vp, vp, vp, vp, vp, vp, vp, sz,
                                        vp]
@@ -225,8 +225,8 @@ def spec_accept(target_logits, draft_logits, draft_tokens, cu_draft, temperature
 
 
 # --------------------------------------------------------------------------- verify epilogue
-def verify_epilogue_workspace_size(num_seqs, total_draft) -> int:
-    return int(load().bp_verify_epilogue_workspace_size(num_seqs, total_draft))
+def verify_epilogue_workspace_size(num_seqs, total_draft, vocab) -> int:
+    return int(load().bp_verify_epilogue_workspace_size(num_seqs, total_draft, vocab))
 
 
 def verify_epilogue(lm_head, h_target, h_draft, draft_tokens, cu_draft, temperature: float, u_accept=None,
@@ -251,7 +251,7 @@ def verify_epilogue(lm_head, h_target, h_draft, draft_tokens, cu_draft, temperat
     if accept_prob is None and want_accept_prob:
         accept_prob = torch.empty(total_draft, dtype=torch.float32, device=dev)
     if ws is None:
-        ws = workspace(lib.bp_verify_epilogue_workspace_size(s, total_draft), dev)
+        ws = workspace(lib.bp_verify_epilogue_workspace_size(s, total_draft, vocab), dev)
     rc = lib.bp_verify_epilogue(_ptr(lm_head), _ptr(h_target), _ptr(h_draft), hidden, vocab, _ptr(draft_tokens),
                                 _ptr(cu_draft), s, total_draft, float(temperature), _ptr(u_accept), _ptr(u_sample),
                                 _ptr(n_accepted), _ptr(out_tokens), _ptr(accept_prob), _ptr(logits_out), _ptr(ws),

@@ -17,7 +17,7 @@ CSRC = os.path.join(PKG, "csrc")
 BUILD = os.path.join(PKG, "_build")
 LIB = os.path.join(PKG, "libblockpilot.so")
 TEST_LIB = os.path.join(PKG, "libblockpilot_shortwait.so")  # test-only build (see above)
-SOURCES = ("api.cu", "attention.cu", "accept.cu", "accept_batch.cu", "policy.cu", "verify_epilogue.cu", "tau.cu", "commit.cu")
+SOURCES = ("api.cu", "attention.cu", "accept.cu", "accept_batch.cu", "policy.cu", "verify_epilogue.cu", "verify_stream.cu", "tau.cu", "commit.cu")
 HEADERS = ("common.cuh", "ptx_sm103.cuh", "softmax_math.cuh")
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 FLAGS = ["-O3", "-lineinfo", "-std=c++17", "-Xcompiler", "-fPIC", "-Xcompiler", "-fvisibility=hidden"]

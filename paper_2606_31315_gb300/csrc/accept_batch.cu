@@ -45,13 +45,14 @@ struct BatchParams {
     const int32_t* tokens;
     const int32_t* cu_draft;
     int num_seqs, total_draft, rows_t, vocab, chunks;
+    int nparts;           // statistics per row in part: the chunks, or 1 for rows merged beforehand
     float c2;  // log2(e) / T; 0 at T = 0
     const float* u_accept;
     const float* u_sample;
     int32_t* n_accepted;
     int32_t* out_tokens;
     float* accept_prob;
-    float2* part;      // [rows][chunks] chunk statistics (T = 0: value, index bits)
+    float2* part;      // [rows][nparts] partial statistics (T = 0: value, index bits)
     ulonglong2* ctot;  // [num_seqs][chunks * parts] draw masses of r and p of the chunks' parts (fixed point)
     unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses
     int* tickets;      // [num_seqs], zero between calls
@@ -169,7 +170,7 @@ __device__ __forceinline__ void load_row_parts(const BatchParams& p, int r, int 
     const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
 #pragma unroll
     for (int q = 0; q < kMergeBatch; ++q)
-        x[q] = r >= 0 && c0 + q < p.chunks ? __ldcg(&p.part[(size_t)r * p.chunks + c0 + q]) : ident;
+        x[q] = r >= 0 && c0 + q < p.nparts ? __ldcg(&p.part[(size_t)r * p.nparts + c0 + q]) : ident;
 }
 template <bool GREEDY>
 __device__ __forceinline__ void merge_parts(float2& acc, const float2 (&x)[kMergeBatch]) {
@@ -190,7 +191,7 @@ __device__ __forceinline__ void merge_rows(const BatchParams& p, int r1, int r2,
     const float2 ident = make_float2(-INFINITY, GREEDY ? __int_as_float(INT_MAX) : 0.f);
     a1 = ident;
     a2 = ident;
-    for (int c0 = 0; c0 < p.chunks; c0 += kMergeBatch) {
+    for (int c0 = 0; c0 < p.nparts; c0 += kMergeBatch) {
         float2 x1[kMergeBatch], x2[kMergeBatch];
         load_row_parts<GREEDY>(p, r1, c0, x1);
         load_row_parts<GREEDY>(p, r2, c0, x2);
@@ -574,12 +575,16 @@ __global__ void __launch_bounds__(kBThreads, SPLIT > 1 ? 2 : PH) batch_draw_kern
 
 }  // namespace
 
+size_t accept_draw_scratch_bytes(int num_seqs, int vocab) {
+    const size_t chunks = ((size_t)vocab + kBChunk - 1) / kBChunk;
+    const size_t segm = (size_t)num_seqs * chunks * 2 * 128 * sizeof(unsigned long long);
+    return align_up((size_t)num_seqs * chunks * kMaxDrawSplit * sizeof(ulonglong2), 256) + align_up(segm, 256);
+}
+
 size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
     const size_t chunks = ((size_t)vocab + kBChunk - 1) / kBChunk;
     const size_t rows = 2 * (size_t)total_draft + num_seqs;
-    const size_t segm = (size_t)num_seqs * chunks * 2 * 128 * sizeof(unsigned long long);
-    return align_up(rows * chunks * sizeof(float2), 256) +
-           align_up((size_t)num_seqs * chunks * kMaxDrawSplit * sizeof(ulonglong2), 256) + align_up(segm, 256);
+    return align_up(rows * chunks * sizeof(float2), 256) + accept_draw_scratch_bytes(num_seqs, vocab);
 }
 
 namespace {
@@ -598,11 +603,9 @@ int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_
     return cudaLaunchKernelEx(&cfg, kernel, p) == cudaSuccess ? BP_OK : BP_ERR_CUDA;
 }
 
+// The decisions (and at T > 0 the draw) once p.part holds the rows' statistics.
 template <bool GREEDY, bool VEC>
-int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
-    const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
-    int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
-    if (rc != BP_OK) return rc;
+int run_decisions(const BatchParams& p, int sm_count, cudaStream_t stream) {
     if (GREEDY)
         return launch_pdl(batch_decide_kernel, (unsigned)((p.num_seqs + kBThreads / 32 - 1) / (kBThreads / 32)), p,
                           stream);
@@ -614,9 +617,15 @@ int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     return draw > sm_count ? launch_pdl(batch_draw_kernel<VEC, 2, 1>, (unsigned)draw, p, stream)
                            : launch_pdl(batch_draw_kernel<VEC, 1, 1>, (unsigned)draw, p, stream);
 }
-}  // namespace
 
-int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* scratch, cudaStream_t stream) {
+template <bool GREEDY, bool VEC>
+int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
+    const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
+    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
+    return rc != BP_OK ? rc : run_decisions<GREEDY, VEC>(p, sm_count, stream);
+}
+
+BatchParams batch_params(const AcceptArgs& a, int* tickets, void* draw_scratch) {
     BatchParams p;
     p.target = a.target;
     p.draft = a.draft;
@@ -627,26 +636,46 @@ int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* s
     p.rows_t = a.total_draft + a.num_seqs;
     p.vocab = a.vocab;
     p.chunks = (a.vocab + kBChunk - 1) / kBChunk;
-    const bool greedy = a.temperature == 0.f;
-    p.c2 = greedy ? 0.f : 1.4426950408889634f / a.temperature;
+    p.nparts = p.chunks;
+    p.c2 = a.temperature == 0.f ? 0.f : 1.4426950408889634f / a.temperature;
     p.u_accept = a.u_accept;
     p.u_sample = a.u_sample;
     p.n_accepted = a.n_accepted;
     p.out_tokens = a.out_tokens;
     p.accept_prob = a.accept_prob;
-    const size_t chunks = (size_t)p.chunks, rows = 2 * (size_t)a.total_draft + a.num_seqs;
-    uint8_t* w = static_cast<uint8_t*>(scratch);
-    p.part = reinterpret_cast<float2*>(w);
-    w += align_up(rows * chunks * sizeof(float2), 256);
+    p.part = nullptr;
+    uint8_t* w = static_cast<uint8_t*>(draw_scratch);
     p.ctot = reinterpret_cast<ulonglong2*>(w);
-    w += align_up((size_t)a.num_seqs * chunks * kMaxDrawSplit * sizeof(ulonglong2), 256);
+    w += align_up((size_t)a.num_seqs * p.chunks * kMaxDrawSplit * sizeof(ulonglong2), 256);
     p.segm = reinterpret_cast<unsigned long long*>(w);
     p.tickets = tickets;
     p.err = a.err_word;
-    const bool vec = (a.vocab % 4 == 0) && (reinterpret_cast<uintptr_t>(a.target) % 16 == 0) &&
-                     (greedy || reinterpret_cast<uintptr_t>(a.draft) % 16 == 0);
+    return p;
+}
+bool batch_vec(const AcceptArgs& a, bool greedy) {
+    return (a.vocab % 4 == 0) && (reinterpret_cast<uintptr_t>(a.target) % 16 == 0) &&
+           (greedy || reinterpret_cast<uintptr_t>(a.draft) % 16 == 0);
+}
+}  // namespace
+
+int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* scratch, cudaStream_t stream) {
+    const size_t chunks = ((size_t)a.vocab + kBChunk - 1) / kBChunk, rows = 2 * (size_t)a.total_draft + a.num_seqs;
+    uint8_t* w = static_cast<uint8_t*>(scratch);
+    BatchParams p = batch_params(a, tickets, w + align_up(rows * chunks * sizeof(float2), 256));
+    p.part = reinterpret_cast<float2*>(w);
+    const bool greedy = a.temperature == 0.f, vec = batch_vec(a, greedy);
     if (greedy) return vec ? run_batch<true, true>(p, sm_count, stream) : run_batch<true, false>(p, sm_count, stream);
     return vec ? run_batch<false, true>(p, sm_count, stream) : run_batch<false, false>(p, sm_count, stream);
+}
+
+int launch_accept_rows(const AcceptArgs& a, const float2* row_stats, int sm_count, int* tickets, void* draw_scratch,
+                       cudaStream_t stream) {
+    BatchParams p = batch_params(a, tickets, draw_scratch);
+    p.part = const_cast<float2*>(row_stats);
+    p.nparts = 1;
+    const bool greedy = a.temperature == 0.f, vec = batch_vec(a, greedy);
+    if (greedy) return run_decisions<true, true>(p, sm_count, stream);  // reads no logits
+    return vec ? run_decisions<false, true>(p, sm_count, stream) : run_decisions<false, false>(p, sm_count, stream);
 }
 
 }  // namespace bp

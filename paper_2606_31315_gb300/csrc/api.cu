@@ -1,6 +1,7 @@
 // The C ABI of libblockpilot: argument validation, workspace bookkeeping, device
 // properties and TMA descriptor encoding.  Every entry point only enqueues work on the
 // caller's stream (bp_get_status excepted) and never allocates.
+#include <limits.h>
 #include <math.h>
 #include <mutex>
 
@@ -281,9 +282,9 @@ int bp_spec_accept_noalloc(const float* target_logits, const float* draft_logits
     return rc;
 }
 
-size_t bp_verify_epilogue_workspace_size(int num_seqs, int total_draft) {
-    if (num_seqs < 0 || total_draft < 0) return 0;
-    return sizeof(WorkspaceHeader) + verify_epilogue_scratch_bytes(num_seqs, total_draft);
+size_t bp_verify_epilogue_workspace_size(int num_seqs, int total_draft, int vocab) {
+    if (num_seqs < 0 || total_draft < 0 || vocab < 1) return 0;
+    return sizeof(WorkspaceHeader) + verify_epilogue_scratch_bytes(num_seqs, total_draft, vocab);
 }
 
 int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_draft, int hidden, int vocab,
@@ -302,13 +303,19 @@ int bp_verify_epilogue(const void* lm_head, const void* h_target, const void* h_
     if (!aligned(lm_head, 16) || !aligned(h_target, 16) || (!greedy && h_draft && !aligned(h_draft, 16)))
         return BP_ERR_UNSUPPORTED;
     const long long rows = (long long)total_draft + num_seqs + (greedy ? 0 : total_draft);
-    if (rows > 64) return BP_ERR_UNSUPPORTED;
-    int rc = check_workspace(workspace, workspace_bytes, bp_verify_epilogue_workspace_size(num_seqs, total_draft));
+    if (2LL * total_draft + num_seqs > INT_MAX / 2) return BP_ERR_UNSUPPORTED;
+    int rc = check_workspace(workspace, workspace_bytes,
+                             bp_verify_epilogue_workspace_size(num_seqs, total_draft, vocab));
     if (rc != BP_OK) return rc;
     DeviceInfo dev;
     if ((rc = device_info(&dev)) != BP_OK) return rc;
-    int grid, np, per;
-    if ((rc = verify_epilogue_config((int)rows, vocab, hidden, dev.sm_count, &grid, &np, &per)) != BP_OK) return rc;
+    if (rows > kVerifyResidentRows) {  // streamed: any vocabulary the SMs can be given a slice of
+        if (verify_stream_grid(vocab, dev.sm_count) < 1) return BP_ERR_UNSUPPORTED;
+    } else {
+        int grid, np, per;
+        if ((rc = verify_epilogue_config((int)rows, vocab, hidden, dev.sm_count, &grid, &np, &per)) != BP_OK)
+            return rc;
+    }
     VerifyEpilogueArgs a;
     a.lm_head = lm_head; a.h_target = h_target; a.h_draft = h_draft;
     a.hidden = hidden; a.vocab = vocab; a.num_seqs = num_seqs; a.total_draft = total_draft;

@@ -125,6 +125,12 @@ inline bool accept_may_batch(int num_seqs, int total_draft, int vocab) {
 }
 size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab);
 int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* scratch, cudaStream_t stream);
+// The throughput path's decisions and draw alone, from statistics merged beforehand: row_stats[r] is row
+// r's (scaled max, sum of 2^(l*log2e/T - max)) over the whole vocabulary, at T = 0 its (max, lowest
+// index bits); rows in the stacked order (target rows, then the drafter's).  At T = 0 no logits are read.
+size_t accept_draw_scratch_bytes(int num_seqs, int vocab);
+int launch_accept_rows(const AcceptArgs& a, const float2* row_stats, int sm_count, int* tickets, void* draw_scratch,
+                       cudaStream_t stream);
 // Same kernel, scratch taken from the library's own static device array (no workspace).
 int launch_accept_noalloc(const AcceptArgs& a, const DeviceInfo& dev, cudaStream_t stream);
 
@@ -166,10 +172,24 @@ struct VerifyEpilogueArgs {
     void* scratch;
     unsigned int* err_word;
 };
-size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft);
+// Rows (target + drafter) above which the verify epilogue streams the LM head (verify_stream.cu)
+// instead of keeping every logit in tensor memory (verify_epilogue.cu).
+constexpr int kVerifyResidentRows = 64;
+size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft, int vocab);
 // Grid size, padded row count (MMA N) and tiles per CTA; BP_ERR_UNSUPPORTED outside the limits.
 int verify_epilogue_config(int rows, int vocab, int hidden, int sm_count, int* grid, int* np, int* tiles_per_cta);
 int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, cudaStream_t stream);
+// The streamed path's scratch, carved from the verify epilogue's workspace.
+struct VerifyStreamScratch {
+    float* logits;      // [rows][vocab] fp32: the logits at T > 0 when the caller gives no logits_out
+    float2* part;       // [rows][slices] slice statistics
+    float2* row_stats;  // [rows] merged statistics
+    int* tickets;       // [num_seqs], zero between calls
+    void* draw;         // accept_draw_scratch_bytes(num_seqs, vocab)
+};
+int verify_stream_grid(int vocab, int sm_count);  // slices of the vocabulary (CTAs); < 1: unsupported
+int launch_verify_stream(const VerifyEpilogueArgs& a, const VerifyStreamScratch& s, const DeviceInfo& dev,
+                         cudaStream_t stream);
 
 struct TauArgs {
     const float* gamma;         // [num_reqs][jmax]

@@ -729,8 +729,9 @@ size_t ve_smem_bytes() {
 
 struct VeLayout {
     size_t sync_off, part_off, xg_off, tot_off, total;
+    size_t rowst_off, tickets_off, draw_off, logits_off;  // the streamed path (more than 64 rows at T > 0)
 };
-VeLayout ve_layout(int num_seqs, int total_draft) {
+VeLayout ve_layout(int num_seqs, int total_draft, int vocab) {
     VeLayout l;
     const int rows = 2 * total_draft + num_seqs;
     l.sync_off = 0;
@@ -738,6 +739,14 @@ VeLayout ve_layout(int num_seqs, int total_draft) {
     l.xg_off = l.part_off + align_up((size_t)(rows > 0 ? rows : 1) * kVeMaxGrid * sizeof(float2), 256);
     l.tot_off = l.xg_off + align_up((size_t)(total_draft > 0 ? total_draft : 1) * sizeof(float2), 256);
     l.total = l.tot_off + align_up((size_t)(num_seqs > 0 ? num_seqs : 1) * kVeMaxGrid * sizeof(ulonglong2), 256);
+    l.rowst_off = l.tickets_off = l.draw_off = l.logits_off = 0;
+    if (rows > kVerifyResidentRows) {
+        l.rowst_off = l.total;
+        l.tickets_off = l.rowst_off + align_up((size_t)rows * sizeof(float2), 256);
+        l.draw_off = l.tickets_off + align_up((size_t)num_seqs * sizeof(int), 256);
+        l.logits_off = l.draw_off + align_up(accept_draw_scratch_bytes(num_seqs, vocab), 256);
+        l.total = l.logits_off + align_up((size_t)rows * (size_t)vocab * sizeof(float), 256);
+    }
     return l;
 }
 
@@ -776,15 +785,15 @@ int ve_launch(const CUtensorMap& wmap, const VeParams& p, int grid, const Device
 
 }  // namespace
 
-size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft) {
-    return ve_layout(num_seqs, total_draft).total;
+size_t verify_epilogue_scratch_bytes(int num_seqs, int total_draft, int vocab) {
+    return ve_layout(num_seqs, total_draft, vocab).total;
 }
 
 int verify_epilogue_config(int rows, int vocab, int hidden, int sm_count, int* grid, int* np, int* tiles_per_cta) {
     if (hidden % kVeAtom != 0) return BP_ERR_UNSUPPORTED;
     const int tiles_total = (vocab + kVeM - 1) / kVeM;
     const int g = min(min(sm_count, kVeMaxGrid), tiles_total);
-    if (g < 1 || rows < 1 || rows > 64) return BP_ERR_UNSUPPORTED;
+    if (g < 1 || rows < 1 || rows > kVerifyResidentRows) return BP_ERR_UNSUPPORTED;
     const int NP = rows <= 32 ? 32 : 64;
     const int per = (tiles_total + g - 1) / g;
     if (per > kVeMaxTiles || per * NP > 512) return BP_ERR_UNSUPPORTED;
@@ -798,6 +807,17 @@ int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, c
     const bool greedy = a.temperature == 0.f;
     const int rows_t = a.total_draft + a.num_seqs;
     const int rows = rows_t + (greedy ? 0 : a.total_draft);
+    const VeLayout l = ve_layout(a.num_seqs, a.total_draft, a.vocab);
+    uint8_t* ws = static_cast<uint8_t*>(a.scratch);
+    if (rows > kVerifyResidentRows) {
+        VerifyStreamScratch s;
+        s.logits = reinterpret_cast<float*>(ws + l.logits_off);
+        s.part = reinterpret_cast<float2*>(ws + l.part_off);
+        s.row_stats = reinterpret_cast<float2*>(ws + l.rowst_off);
+        s.tickets = reinterpret_cast<int*>(ws + l.tickets_off);
+        s.draw = ws + l.draw_off;
+        return launch_verify_stream(a, s, dev, stream);
+    }
     int grid = 0, NP = 0, per = 0;
     int rc = verify_epilogue_config(rows, a.vocab, a.hidden, dev.sm_count, &grid, &NP, &per);
     if (rc != BP_OK) return rc;
@@ -813,8 +833,6 @@ int launch_verify_epilogue(const VerifyEpilogueArgs& a, const DeviceInfo& dev, c
                           CU_TENSOR_MAP_SWIZZLE_128B) != BP_OK)
         return BP_ERR_CUDA;
 
-    const VeLayout l = ve_layout(a.num_seqs, a.total_draft);
-    uint8_t* ws = static_cast<uint8_t*>(a.scratch);
     VeParams p;
     p.h_target = static_cast<const __nv_bfloat16*>(a.h_target);
     p.h_draft = static_cast<const __nv_bfloat16*>(greedy ? a.h_target : a.h_draft);

@@ -7,6 +7,9 @@ CASE is one of:
   verify_epilogue_t1  Qwen3-4B LM head (151936 x 2560 bf16) fused with the acceptance, 16 target and
                       15 drafter states, T = 1
   verify_epilogue_t0  the same at T = 0 (16 target states)
+  verify_stream_c5_t1 the long-context batch through the same LM head: 8 sequences x 16 positions,
+                      128 target and 120 drafter states (248 rows, streamed), T = 1
+  verify_stream_c5_t0 the same at T = 0 (128 target states)
   accept_t1           acceptance over 16 x 151936 target and 15 x 151936 draft fp32 logits, T = 1
   accept_batch_t1     acceptance over a batch of 32 sequences of 16 target rows (512 x 151936 target
                       and 480 x 151936 draft fp32 logits), T = 1: the three throughput kernels
@@ -52,7 +55,20 @@ def _verify_epilogue(dev, gen, temperature):
     tok = torch.randint(0, V, (td,), device=dev, generator=gen, dtype=torch.int32)
     cu = torch.tensor([0, td], dtype=torch.int32, device=dev)
     ua, us = torch.rand(td, device=dev, generator=gen), torch.rand(1, device=dev, generator=gen)
-    ws = bp.workspace(bp.verify_epilogue_workspace_size(1, td), dev)
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(1, td, V), dev)
+    return lambda: bp.verify_epilogue(w, h_t, h_d if temperature > 0 else None, tok, cu, temperature, ua, us,
+                                      want_accept_prob=False, ws=ws)
+
+
+def _verify_stream_c5(dev, gen, temperature):
+    S, td = 8, 8 * (B - 1)
+    w = (torch.randn(V, H, device=dev, generator=gen) * (3.0 / H ** 0.5)).to(torch.bfloat16)
+    h_t = torch.randn(td + S, H, device=dev, generator=gen).to(torch.bfloat16)
+    h_d = torch.randn(td, H, device=dev, generator=gen).to(torch.bfloat16)
+    tok = torch.randint(0, V, (td,), device=dev, generator=gen, dtype=torch.int32)
+    cu = torch.arange(0, td + 1, B - 1, dtype=torch.int32, device=dev)
+    ua, us = torch.rand(td, device=dev, generator=gen), torch.rand(S, device=dev, generator=gen)
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(S, td, V), dev)
     return lambda: bp.verify_epilogue(w, h_t, h_d if temperature > 0 else None, tok, cu, temperature, ua, us,
                                       want_accept_prob=False, ws=ws)
 
@@ -156,6 +172,8 @@ def _tau(dev, gen):
 CASES = {
     "verify_epilogue_t1": lambda dev, gen: _verify_epilogue(dev, gen, 1.0),
     "verify_epilogue_t0": lambda dev, gen: _verify_epilogue(dev, gen, 0.0),
+    "verify_stream_c5_t1": lambda dev, gen: _verify_stream_c5(dev, gen, 1.0),
+    "verify_stream_c5_t0": lambda dev, gen: _verify_stream_c5(dev, gen, 0.0),
     "accept_t1": _accept,
     "accept_batch_t1": lambda dev, gen: _accept_batch(dev, gen, 1.0),
     "accept_batch_t0": lambda dev, gen: _accept_batch(dev, gen, 0.0),

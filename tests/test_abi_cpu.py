@@ -144,13 +144,16 @@ def test_verify_epilogue_host_validation_needs_no_gpu(lib):
     def call(hidden=2560, vocab=151936, seqs=1, drafts=15, temp=1.0, h_draft=fake, ws_bytes=1 << 20, w=fake):
         return lib.bp_verify_epilogue(w, fake, h_draft, hidden, vocab, fake, fake, seqs, drafts, f32(temp), fake, fake,
                                       fake, fake, None, None, ws, ws_bytes, None)
-    need = lib.bp_verify_epilogue_workspace_size(1, 15)
+    need = lib.bp_verify_epilogue_workspace_size(1, 15, 151936)
     assert 256 < need < (1 << 20) and need % 256 == 0
     assert call(w=None) == 1                      # no LM head
     assert call(temp=-1.0) == 1                   # negative temperature
     assert call(h_draft=None) == 1                # T > 0 needs the drafter's states
     assert call(hidden=100) == 2                  # hidden not a multiple of 64
-    assert call(drafts=40) == 2                   # 40 + 1 + 40 rows > 64
+    assert call(drafts=40, ws_bytes=need) == 4    # 81 rows: streamed, its workspace holds the logits
+    big = lib.bp_verify_epilogue_workspace_size(1, 40, 151936)
+    assert big >= 81 * 151936 * 4 + need and big % 256 == 0
+    assert lib.bp_verify_epilogue_workspace_size(1, 15, 0) == 0   # no vocabulary
     assert call(w=vp(0x10008)) == 2               # LM head not 16-byte aligned
     assert call(ws_bytes=need - 256) == 4         # workspace too small
     assert call(seqs=0) == 0                      # nothing to do

@@ -47,7 +47,8 @@ def run_gpu(inp: dict, temperature: float, u_accept=None, u_sample=None, want_lo
     rows = d["h_target"].shape[0] + (d["h_draft"].shape[0] if d["h_draft"] is not None else 0)
     logits = torch.full((rows, inp["vocab"]), float("nan"), device=dev()) if want_logits else None
     if ws is None:
-        ws = bp.workspace(bp.verify_epilogue_workspace_size(len(inp["cu_draft"]) - 1, len(inp["draft_tokens"])), dev())
+        ws = bp.workspace(bp.verify_epilogue_workspace_size(len(inp["cu_draft"]) - 1, len(inp["draft_tokens"]),
+                                                      inp["vocab"]), dev())
     n_acc, out, ap = bp.verify_epilogue(d["w"], d["h_target"], d["h_draft"], d["tokens"], d["cu"], temperature, ua, us,
                                         logits_out=logits, ws=ws)
     status = bp.get_status(ws)
@@ -248,7 +249,7 @@ def test_qwen3_4b_full(qwen_weight, temp):
     inp = wl.lm_head_inputs(w, temp, weight=qwen_weight)
     ref = run_oracle(inp, temp)
     d = device_inputs(inp, temp)
-    ws = bp.workspace(bp.verify_epilogue_workspace_size(1, len(inp["draft_tokens"])), dev())
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(1, len(inp["draft_tokens"]), inp["vocab"]), dev())
     compare(inp, temp, run_gpu(inp, temp, want_logits=True, ws=ws, dev_inp=d), ref)
     if temp == 0:
         return
@@ -283,7 +284,7 @@ def test_workspace_reuse_is_deterministic():
     w = wl.custom(seed=24, ctx=(0,) * 2, block=(12, 6), vocab=70000)
     inp = wl.lm_head_inputs(w, 1.0, hidden=128)
     d = device_inputs(inp, 1.0)
-    ws = bp.workspace(bp.verify_epilogue_workspace_size(2, len(inp["draft_tokens"])), dev())
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(2, len(inp["draft_tokens"]), inp["vocab"]), dev())
     first = run_gpu(inp, 1.0, ws=ws, dev_inp=d)
     for _ in range(3):
         again = run_gpu(inp, 1.0, ws=ws, dev_inp=d)
@@ -303,6 +304,97 @@ def test_out_of_range_draft_token_sets_the_device_flag():
 
 def test_host_rejects_unsupported_shapes():
     w = wl.custom(seed=26, ctx=(0,) * 3, block=(16, 16, 16), vocab=1000)
-    inp = wl.lm_head_inputs(w, 1.0, hidden=64)  # 45 drafts: 93 rows > 64
+    inp = wl.lm_head_inputs(w, 1.0, hidden=64)
+    inp["w"] = np.ascontiguousarray(np.concatenate([inp["w"], inp["w"][:, :32]], axis=1))  # hidden 96
+    inp["h_target"] = np.ascontiguousarray(np.concatenate([inp["h_target"], inp["h_target"][:, :32]], axis=1))
+    inp["h_draft"] = np.ascontiguousarray(np.concatenate([inp["h_draft"], inp["h_draft"][:, :32]], axis=1))
     with pytest.raises(bp.BlockPilotError):
         run_gpu(inp, 1.0)
+
+
+# ---- more than 64 rows: the LM head streamed through tensor memory, statistics formed in its epilogue
+STREAM_CASES = [
+    # (seed, blocks, vocab, hidden): rows at T > 0 / T = 0.  Logits leave by TMA stores where a group's
+    # rows are contiguous and rows are 16-byte aligned, else by whole-line stores
+    (31, (16, 16, 16), 1000, 64),              # 93 / 48: one 128-row half; T = 0 resident
+    (32, (16,) * 5, 30011, 128),               # 155 / 80: two halves; odd vocabulary (4-byte stores)
+    (33, (16,) * 10, 20000, 192),              # 310 / 160: two groups of rows at T > 0
+    (34, (16,) * 9 + (5,), 12344, 64),         # 288 / 149: target rows end off an 8-row boundary (16-byte
+                                               # stores in the first group)
+    (35, (1,) * 70, 4096, 64),                 # 70 / 70: blocks of one position (bonus draws only)
+]
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+@pytest.mark.parametrize("case", STREAM_CASES)
+def test_streamed_rows(case, temp):
+    seed, blocks, vocab, hidden = case
+    w = wl.custom(seed=seed, ctx=(0,) * len(blocks), block=blocks, vocab=vocab)
+    inp = wl.lm_head_inputs(w, temp, hidden=hidden)
+    ref = run_oracle(inp, temp)
+    compare(inp, temp, run_gpu(inp, temp, want_logits=True), ref)
+    compare(inp, temp, run_gpu(inp, temp), ref, check_logits=False)  # logits only where the path needs them
+
+
+def test_streamed_workspace_reuse_is_deterministic():
+    """Repeated streamed calls on one workspace give identical results (the draw's tickets return to
+    zero, the slice statistics are merged in a fixed order)."""
+    w = wl.custom(seed=36, ctx=(0,) * 6, block=(16, 12, 16, 3, 16, 9), vocab=50000)
+    inp = wl.lm_head_inputs(w, 1.0, hidden=128)
+    d = device_inputs(inp, 1.0)
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(6, len(inp["draft_tokens"]), inp["vocab"]), dev())
+    first = run_gpu(inp, 1.0, ws=ws, dev_inp=d)
+    for _ in range(3):
+        again = run_gpu(inp, 1.0, ws=ws, dev_inp=d)
+        for a, b in zip(first[:3], again[:3]):
+            np.testing.assert_array_equal(a, b)
+
+
+def test_streamed_out_of_range_draft_token_sets_the_device_flag():
+    w = wl.custom(seed=37, ctx=(0,) * 5, block=(16,) * 5, vocab=4000)
+    inp = wl.lm_head_inputs(w, 1.0, hidden=64)
+    inp["draft_tokens"] = inp["draft_tokens"].copy()
+    inp["draft_tokens"][7] = -3
+    gpu = run_gpu(inp, 1.0)
+    assert gpu[3] == 6  # BP_ERR_DEVICE_FLAG
+
+
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_long_context_batch_full_head(qwen_weight, temp):
+    """The long-context verify batch (8 sequences x 16 positions: 128 target rows and, at T = 1, 120
+    drafter rows -- 248 rows) through the full Qwen3-4B LM head (151936 x 2560), as the benchmark
+    launches it.  At T = 1 also draws with planted uniforms over confident target rows, which must
+    match the oracle exactly."""
+    lc = wl.get("long_context")
+    base = wl.custom(seed=lc.seed, ctx=(0,) * lc.num_seqs, block=lc.block, vocab=lc.vocab, logit_std=lc.logit_std)
+    inp = wl.lm_head_inputs(base, temp, hidden=wl.LM_HIDDEN["long_context"], weight=qwen_weight)
+    ref = run_oracle(inp, temp)
+    d = device_inputs(inp, temp)
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(lc.num_seqs, len(inp["draft_tokens"]), inp["vocab"]), dev())
+    compare(inp, temp, run_gpu(inp, temp, want_logits=True, ws=ws, dev_inp=d), ref)
+    compare(inp, temp, run_gpu(inp, temp, ws=ws, dev_inp=d), ref, check_logits=False)
+    if temp == 0:
+        return
+    exact, ks = 0, set()
+    for seed in range(2):
+        ws_in = wl.custom(seed=200 + seed, ctx=(0,) * lc.num_seqs, block=lc.block, vocab=lc.vocab,
+                          logit_std=lc.logit_std)
+        inp = wl.lm_head_inputs(ws_in, temp, hidden=wl.LM_HIDDEN["long_context"], weight=qwen_weight,
+                                target_peak=22.0)
+        ref = run_oracle(inp, temp)
+        d = device_inputs(inp, temp)
+        rng = np.random.default_rng(seed)
+        for _ in range(2):
+            ua, us, planted = planted_uniforms(inp, ref, temp, rng)
+            trial_inp = dict(inp, u_accept=ua, u_sample=us)
+            tref = dict(ref)
+            tref.update(oracle.spec_accept(ref["target_logits"], ref["draft_logits"], inp["draft_tokens"],
+                                           inp["cu_draft"], temp, ua, us))
+            flagged, _ = compare(trial_inp, temp, run_gpu(trial_inp, temp, ws=ws, dev_inp=d), tref,
+                                 check_logits=False)
+            if planted.all():
+                assert flagged == 0  # every margin is far above the derived tolerance: bit-exact
+            # a planted sequence's margins (>= 0.04) are far above the tolerance: compared bit-exactly
+            exact += int(planted.sum())
+            ks.update(int(k) for k, pl in zip(tref["n_accepted"], planted) if pl)
+    assert exact >= 24 and len(ks) >= 3, (exact, ks)
