@@ -5,8 +5,9 @@ records BP_ERR_TIMEOUT in the workspace error word, waits out its own copies and
 still in flight (a separate drain budget), releases its tensor memory and returns, so the context stays
 usable.  A test-only build of the library (libblockpilot_shortwait.so, compiled with
 BP_TEST_SHORT_WAITS) turns every such wait into a single non-blocking test, which finds the data of a
-copy just issued still in flight: the attention kernel (both key splits) and the cluster acceptance
-kernel (T = 1 and T = 0) then take that path.  Nothing faults and nothing waits on an event that never
+copy just issued still in flight: the attention kernel (both key splits), the cluster acceptance
+kernel (T = 1 and T = 0) and the verify epilogue's streamed LM head (T = 1 and T = 0) then take that
+path.  Nothing faults and nothing waits on an event that never
 comes: the drains wait for copies the kernel itself issued.
 
 The test build runs in a child process, which also checks that its CUDA context still works after
@@ -57,6 +58,15 @@ for temp in (1.0, 0.0):
     bp.spec_accept(t(inp["target_logits"]), t(inp["draft_logits"]) if temp > 0 else None, t(inp["draft_tokens"]),
                    t(inp["cu_draft"]), temp, t(inp["u_accept"]), t(inp["u_sample"]), ws=ws)
     out["accept_t%d" % temp] = bp.get_status(ws)
+# the verify epilogue's streamed path (more than 64 rows): two 128-row halves at T = 1, one at T = 0
+w5 = wl.custom(seed=41, ctx=(0,) * 5, block=(16,) * 5, vocab=30000)
+for temp in (1.0, 0.0):
+    inp = wl.lm_head_inputs(w5, temp, hidden=128)
+    ws = bp.workspace(bp.verify_epilogue_workspace_size(5, len(inp["draft_tokens"]), inp["vocab"]), dev)
+    bp.verify_epilogue(bf(inp["w"]), bf(inp["h_target"]), bf(inp["h_draft"]) if temp > 0 else None,
+                       t(inp["draft_tokens"]), t(inp["cu_draft"]), temp, t(inp["u_accept"]), t(inp["u_sample"]),
+                       ws=ws)
+    out["verify_stream_t%d" % temp] = bp.get_status(ws)
 x = torch.arange(1 << 20, device=dev, dtype=torch.float32)  # the context still runs work
 out["context_ok"] = bool(float(x.sum().item()) == float((1 << 20) * ((1 << 20) - 1) // 2))
 print(json.dumps(out))
@@ -79,7 +89,7 @@ def test_expired_waits_report_timeout_and_leave_the_context_usable():
     got = json.loads([ln for ln in res.stdout.splitlines() if ln.startswith("{")][-1])
     timeout = 5  # BP_ERR_TIMEOUT
     assert got == {"attention_cluster": timeout, "attention_flat": timeout, "accept_t1": timeout, "accept_t0": timeout,
-                   "context_ok": True}, got
+                   "verify_stream_t1": timeout, "verify_stream_t0": timeout, "context_ok": True}, got
 
 
 def test_product_library_after_the_timeouts():
@@ -91,3 +101,9 @@ def test_product_library_after_the_timeouts():
         assert err <= ATTN_TOL and lerr <= LSE_TOL
     for temp in (1.0, 0.0):
         compare_accept(wl.accept_inputs(wl.get("qwen3_4b"), temp), temp)
+    from test_gpu_verify_epilogue import compare, run_gpu, run_oracle
+
+    w5 = wl.custom(seed=41, ctx=(0,) * 5, block=(16,) * 5, vocab=30000)
+    for temp in (1.0, 0.0):
+        inp = wl.lm_head_inputs(w5, temp, hidden=128)
+        compare(inp, temp, run_gpu(inp, temp, want_logits=True), run_oracle(inp, temp))
