@@ -13,10 +13,11 @@
 //      x K=16 tcgen05 MMAs, one per 128-row half of the states.  Tensor-memory lane = state row, so each
 //      epilogue thread owns one row and folds the pass's 256 logits into its row's running (max, sum of
 //      2^(l*log2e/T - max)) -- at T = 0 its (max, lowest index) -- with one exponential per logit and no
-//      exchange between threads.  At T > 0 it also writes the logits once (streaming stores): the draw
-//      at the first rejection needs a whole row pair again, and no on-chip store can hold every row
-//      until the decisions are known.  At T = 0 nothing but the statistics leaves the chip.  Each CTA
-//      writes its slice's statistics of every row.
+//      exchange between threads.  At T > 0 it also writes the logits once (each warp's 32 x 32 chunk
+//      staged in shared memory and sent by one TMA store): the draw at the first rejection needs a
+//      whole row pair again, and no on-chip store can hold every row until the decisions are known.
+//      At T = 0 nothing but the statistics leaves the chip.  Each CTA writes its slice's statistics
+//      of every row.
 //   2. lm_head_row_merge_kernel: one warp per row merges the slices' statistics in a fixed order.
 //   3. The decisions and the draw of accept_batch.cu on those row statistics: only the draw's row pair
 //      per sequence (and the logits at the drafted tokens) is read back.
@@ -50,8 +51,8 @@ constexpr int kVsMaxSlices = 160;        // slices (CTAs) per row in the statist
 
 // MT halves of 128 state rows.  Tensor memory (512 columns) holds two passes' accumulators with one
 // half -- the epilogue of one pass overlaps the MMAs of the next -- or one pass with two.  (Passes of
-// 128 entries would let two halves double-buffer too, but they stream the states from L2 twice as
-// often per entry, and the state stream, not HBM, then bounds the MMAs: measured slower.)  Stages
+// 128 entries would let two halves double-buffer too, but the MMAs' operand reads and the ring's
+// fills then ask more of shared memory per entry than it serves: measured slower.)  Stages
 // of W and states together: 4 x 48 KB with one half, 3 x 64 KB with two; then the store staging.
 __host__ __device__ constexpr int vs_stages(int MT) { return MT == 2 ? 3 : 4; }
 constexpr int kVsStageBytes = 32 * 128;  // per epilogue warp: one chunk of 32 rows x 32 fp32 logits
