@@ -336,6 +336,18 @@ def test_streamed_rows(case, temp):
     compare(inp, temp, run_gpu(inp, temp), ref, check_logits=False)  # logits only where the path needs them
 
 
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+def test_streamed_ragged_batch_rows(temp):
+    """The ragged 32-request batch's blocks (8 to 24 positions: 502 target rows and at T = 1 470
+    drafter rows, 972 rows in four groups of the streamed projection), over a 32000-entry vocabulary."""
+    rg = wl.get("ragged")
+    w = wl.custom(seed=38, ctx=(0,) * rg.num_seqs, block=rg.block, vocab=32000, logit_std=rg.logit_std)
+    inp = wl.lm_head_inputs(w, temp, hidden=256)
+    ref = run_oracle(inp, temp)
+    compare(inp, temp, run_gpu(inp, temp, want_logits=True), ref)
+    compare(inp, temp, run_gpu(inp, temp), ref, check_logits=False)
+
+
 def test_streamed_workspace_reuse_is_deterministic():
     """Repeated streamed calls on one workspace give identical results (the draw's tickets return to
     zero, the slice statistics are merged in a fixed order)."""
