@@ -588,18 +588,22 @@ size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
 }
 
 namespace {
+// pdl: the prologue may overlap the previous kernel's tail (programmatic stream serialization).  The
+// statistics kernel, first of the chain, launches in plain stream order: behind a long kernel its
+// thousands of CTAs were placed early and waiting on every SM, and a step of the ragged batch
+// (attention, then the acceptance) took 220 us instead of 201.
 template <typename Kernel>
-int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_t stream) {
+int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_t stream, bool pdl = true) {
     if (blocks == 0) return BP_OK;
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(blocks);
     cfg.blockDim = dim3(kBThreads);
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
-    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;  // the prologue may overlap the
-    attr[0].val.programmaticStreamSerializationAllowed = 1;            // previous kernel's tail
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
     cfg.attrs = attr;
-    cfg.numAttrs = 1;
+    cfg.numAttrs = pdl ? 1 : 0;
     return cudaLaunchKernelEx(&cfg, kernel, p) == cudaSuccess ? BP_OK : BP_ERR_CUDA;
 }
 
@@ -621,7 +625,7 @@ int run_decisions(const BatchParams& p, int sm_count, cudaStream_t stream) {
 template <bool GREEDY, bool VEC>
 int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
-    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
+    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream, false);
     return rc != BP_OK ? rc : run_decisions<GREEDY, VEC>(p, sm_count, stream);
 }
 
