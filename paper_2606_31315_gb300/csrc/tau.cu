@@ -20,6 +20,7 @@
 #include <mutex>
 
 #include "common.cuh"
+#include "ptx_sm103.cuh"
 
 namespace bp {
 namespace {
@@ -42,9 +43,10 @@ struct TauParams {
     unsigned int* err;
 };
 
-// Per-warp staging area: the warp's 32 gamma rows (ldr floats each), then its 32 tau rows.
+// Per-warp staging area: two buffers of the warp's 32 gamma rows (ldr floats each) -- the next 32
+// requests' rows stream in (cp.async) while the current ones are computed -- then its 32 tau rows.
 __host__ __device__ inline int tau_ldr(int jmax) { return (jmax & 3) == 0 ? jmax + 4 : jmax + 1; }
-__host__ __device__ inline int tau_warp_floats(int jmax, int nc) { return 32 * (tau_ldr(jmax) + nc); }
+__host__ __device__ inline int tau_warp_floats(int jmax, int nc) { return 32 * (2 * tau_ldr(jmax) + nc); }
 
 // tau_c = sum_{i=1}^{b_c} r_c^i P_i is the product of the request's prefix products P with the table
 // R[i][c] = r_c^(i+1) for i < b_c (0 past b_c and for padding candidates), the same for every request.
@@ -63,8 +65,8 @@ __global__ void __launch_bounds__(kTauThreads) tau_kernel(const __grid_constant_
     __shared__ double red_sh[kTauThreads / 32][3];
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int ldr = tau_ldr(p.jmax);
-    float* rows_sh = reinterpret_cast<float*>(dyn4) + warp * tau_warp_floats(p.jmax, p.nc);
-    float* out_sh = rows_sh + 32 * ldr;
+    float* rows_buf = reinterpret_cast<float*>(dyn4) + warp * tau_warp_floats(p.jmax, p.nc);
+    float* out_sh = rows_buf + 2 * 32 * ldr;
     const bool vec = (p.jmax & 3) == 0 && (reinterpret_cast<uintptr_t>(p.gamma) & 15) == 0;
     const int q4 = p.jmax >> 2;
     const unsigned magic = vec ? (unsigned)((0x100000000ull + q4 - 1) / q4) : 0u;  // f / q4 = umulhi(f, magic)
@@ -72,18 +74,29 @@ __global__ void __launch_bounds__(kTauThreads) tau_kernel(const __grid_constant_
     const bool vout = p.tau && (reinterpret_cast<uintptr_t>(p.tau) & 15) == 0;
     float rsum_t = 0.f, lmax_t = 0.f;  // this thread's requests, in order (fp32: the FP64 pipe is slow)
     long long dsum_t = 0;
+    // the warp's 32 rows of requests x0.. are contiguous: coalesced 16-byte asynchronous copies
+    const auto prefetch = [&](long long xp, float* dst) {
+        const int nrows = (int)min(32LL, (long long)p.n - xp);
+        const float4* s4 = reinterpret_cast<const float4*>(p.gamma + (size_t)xp * p.jmax);
+        for (int f = lane; f < nrows * q4; f += 32) {
+            const int r = (int)__umulhi((unsigned)f, magic), q = f - r * q4;
+            cp_async16(dst + r * ldr + 4 * q, s4 + f, true);
+        }
+    };
     // each warp takes 32 consecutive requests; the grid strides over them
-    for (long long x0 = ((long long)blockIdx.x * (kTauThreads / 32) + warp) * 32; x0 < p.n;
-         x0 += (long long)gridDim.x * kTauThreads) {
+    const long long xstride = (long long)gridDim.x * kTauThreads;
+    long long x0 = ((long long)blockIdx.x * (kTauThreads / 32) + warp) * 32;
+    if (vec && x0 < p.n) prefetch(x0, rows_buf);
+    cp_async_commit();
+    for (int buf = 0; x0 < p.n; x0 += xstride, buf ^= (vec ? 1 : 0)) {
         const int rows = (int)min(32LL, (long long)p.n - x0);
-        const float* src = p.gamma + (size_t)x0 * p.jmax;
-        if (vec) {  // the warp's rows are contiguous: coalesced 16-byte copies
-            const float4* s4 = reinterpret_cast<const float4*>(src);
-            for (int f = lane; f < rows * q4; f += 32) {
-                const int r = (int)__umulhi((unsigned)f, magic), q = f - r * q4;
-                *reinterpret_cast<float4*>(rows_sh + r * ldr + 4 * q) = __ldg(s4 + f);
-            }
+        float* rows_sh = rows_buf + buf * 32 * ldr;
+        if (vec) {  // the next 32 requests' rows start streaming; this iteration's have landed
+            if (x0 + xstride < p.n) prefetch(x0 + xstride, rows_buf + (buf ^ 1) * 32 * ldr);
+            cp_async_commit();
+            cp_async_wait_group<1>();
         } else {
+            const float* src = p.gamma + (size_t)x0 * p.jmax;
             for (int f = lane; f < rows * p.jmax; f += 32) rows_sh[(f / p.jmax) * ldr + f % p.jmax] = __ldg(src + f);
         }
         __syncwarp();
