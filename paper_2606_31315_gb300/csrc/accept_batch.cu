@@ -21,8 +21,8 @@
 //      max(0, p_k - q_k) and of p_k in exact 2^-52 fixed point; the last CTA of the sequence (ticket)
 //      finds the part and the 128-entry segment where the inverse CDF crosses u_s * total from the
 //      stored masses, then the entry from that segment's 128 logits, and writes the emitted token.
-// Only the one draw row pair per sequence is read twice.  The kernels chain with programmatic dependent
-// launch.
+// Only the one draw row pair per sequence is read twice.  The decisions and the draw chain behind the
+// statistics with programmatic dependent launch; the statistics kernel launches in plain stream order.
 #include <cuda_runtime.h>
 #include <math.h>
 
