@@ -324,6 +324,14 @@ def run_ours(args):
     value = job_throughput(tokens_per_step, args.steps, elapsed, world)
     ms_per_step = elapsed / args.steps * 1e3
     step_bytes = attention_bytes(hw) + accept_bytes(hw, 1.0)
+    # tokens the steps emit (the accepted drafts and one drawn token per sequence), on the two input copies
+    emitted = []
+    for g in g_steps:
+        with torch.cuda.stream(stream):
+            g.replay()
+        stream.synchronize()
+        emitted.append(int(hstep.n.sum().item()) + hw.num_seqs)
+    emitted_per_step = float(np.mean(emitted))
 
     # the step's kernels timed alone (same alternation, graph replays): the dominant one is the attention
     reps_h = max(20, min(200, args.steps))
@@ -713,6 +721,8 @@ def run_ours(args):
                          "peak": peak, "frac": round(step_bytes / (elapsed / args.steps) / 1e9 / peak, 4),
                          "roofline_tokens_per_s": round(tokens_per_step / (step_bytes / (peak * 1e9)), 1),
                          "requests_per_s": round(job_throughput(hw.num_seqs, args.steps, elapsed, world), 1),
+                         "emitted_tokens_per_s": round(emitted_per_step * args.steps * world / elapsed, 1),
+                         "emitted_per_step": emitted_per_step,
                          "roofline_requests_per_s": round(hw.num_seqs / (step_bytes / (peak * 1e9)), 1)},
         "roofline": roofline,
         "rows": rows,
