@@ -719,34 +719,10 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int per = (m_valid + (int)CS - 1) / (int)CS;
             const int rbeg = (int)crank * per;
             const int nmy = max(0, min(m_valid, rbeg + per) - rbeg);
-            // one round of remote loads for the peers' (m, l) of the owned rows, then the weights
-            float2* ml_st = reinterpret_cast<float2*>(sKV + kM * kD * sizeof(float) + kM * sizeof(float2));
-            float* w_st = reinterpret_cast<float*>(ml_st + kMaxCluster * kM);
-            float* inv_st = w_st + kMaxCluster * kM;
-            for (int idx = tid; idx < (int)CS * nmy; idx += kThreads) {
-                const int pr = idx / nmy, rr = idx % nmy;
-                ml_st[pr * nmy + rr] = *cluster.map_shared_rank(&row_ml[rbeg + rr], pr);
-            }
-            __syncthreads();
-            for (int rr = tid; rr < nmy; rr += kThreads) {
-                float M = -INFINITY;
-                for (uint32_t pr = 0; pr < CS; ++pr) M = fmaxf(M, ml_st[pr * nmy + rr].x);
-                float Lsum = 0.f;
-                for (uint32_t pr = 0; pr < CS; ++pr) {
-                    const float2 ml = ml_st[pr * nmy + rr];
-                    const float w = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - M);
-                    w_st[pr * nmy + rr] = w;
-                    Lsum += w * ml.y;
-                }
-                inv_st[rr] = Lsum > 0.f ? 1.f / Lsum : 0.f;
-                if (p.lse) {
-                    const int lr = row0 + rbeg + rr;
-                    p.lse[(size_t)(one.q0 + lr / G) * p.num_q_heads + one.h * G + lr % G] =
-                        (M + __log2f(Lsum)) * kLn2;
-                }
-            }
-            __syncthreads();
-            // the owned rows: every peer's 16-byte chunk requested at once
+            // one round of remote loads per owned row: a warp takes the row, lane c its 16-byte chunk c of
+            // every peer's partial O and, for c below the cluster size, peer c's (m, l); the weights then
+            // go round the warp by shuffles
+            static_assert(kD / 4 == 32 && kThreads % 32 == 0, "a warp's 32 items are one row");
             for (int item = tid; item < nmy * (kD / 4); item += kThreads) {
                 const int rr = item / (kD / 4);
                 const int c = item % (kD / 4);
@@ -756,24 +732,33 @@ __global__ void __launch_bounds__(kThreads, 1)
 #pragma unroll
                 for (int pr = 0; pr < kMaxCluster; ++pr)
                     if (pr < (int)CS) v[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(src), pr);
+                const float2 ml = c < (int)CS ? *cluster.map_shared_rank(&row_ml[row], c) : make_float2(-INFINITY, 0.f);
+                float M = ml.x;
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
+                const float wl = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - M);
+                float Lsum = wl * ml.y;
+#pragma unroll
+                for (int o = 16; o >= 1; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
                 float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
 #pragma unroll
                 for (int pr = 0; pr < kMaxCluster; ++pr) {
                     if (pr < (int)CS) {
-                        const float w = w_st[pr * nmy + rr];
+                        const float w = __shfl_sync(0xffffffffu, wl, pr);
                         acc.x += w * v[pr].x;
                         acc.y += w * v[pr].y;
                         acc.z += w * v[pr].z;
                         acc.w += w * v[pr].w;
                     }
                 }
-                const float inv = inv_st[rr];
+                const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
                 const int lr = row0 + row;
                 const size_t orow = (size_t)(one.q0 + lr / G) * p.num_q_heads + one.h * G + lr % G;
                 uint2 w2;
                 w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
                 w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
                 *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
+                if (p.lse && c == 0) p.lse[orow] = (M + __log2f(Lsum)) * kLn2;
             }
             cluster.sync();  // no CTA leaves while peers may still read its shared memory
         }
