@@ -86,6 +86,20 @@ def test_blocks_longer_than_a_warp_batch(temp):
     assert n_acc.max() > 32
 
 
+@pytest.mark.parametrize("temp", [1.0, 0.0])
+@pytest.mark.parametrize("num_seqs", [1, 255, 256])
+def test_one_long_or_many_short_sequences(num_seqs, temp):
+    """The throughput kernels on one 48-position block over the full vocabulary (the draw's parts all
+    belong to one sequence) and on hundreds of 1-4 position blocks (one decision warp and one draw per
+    sequence, most of them bonus draws or first-position rejections), against the oracle."""
+    rng = np.random.default_rng(num_seqs)
+    blocks = (48,) if num_seqs == 1 else tuple(int(x) for x in rng.integers(1, 5, num_seqs))
+    vocab = 151936 if num_seqs == 1 else 32000
+    assert accept_uses_batch(blocks, vocab, temp)
+    w = wl.custom(seed=num_seqs + 3, ctx=(0,) * len(blocks), block=blocks, vocab=vocab)
+    compare_accept(wl.accept_inputs(w, temp, planted_match=0.5), temp)
+
+
 @pytest.mark.parametrize("batch", [False, True])
 @pytest.mark.parametrize("vocab", [5, 1001, 4099, 16384, 32000, 50001])
 def test_vocab_sizes_and_scalar_path(vocab, batch):
