@@ -22,7 +22,9 @@
 //      finds the part and the 128-entry segment where the inverse CDF crosses u_s * total from the
 //      stored masses, then the entry from that segment's 128 logits, and writes the emitted token.
 // Only the one draw row pair per sequence is read twice.  The decisions and the draw chain behind the
-// statistics with programmatic dependent launch; the statistics kernel launches in plain stream order.
+// statistics with programmatic dependent launch; the statistics kernel launches in plain stream order,
+// so their decision warps load the inputs that kernel does not write (offsets, drafted tokens, uniforms,
+// the drafted tokens' logits) before their grid-dependency wait.
 #include <cuda_runtime.h>
 #include <math.h>
 
@@ -56,6 +58,7 @@ struct BatchParams {
     ulonglong2* ctot;  // [num_seqs][chunks * parts] draw masses of r and p of the chunks' parts (fixed point)
     unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses
     int* tickets;      // [num_seqs], zero between calls
+    int inputs_early;  // every input was written before the chain's first kernel started (see DecideIn)
     unsigned int* err;
 };
 
@@ -200,16 +203,44 @@ __device__ __forceinline__ void merge_rows(const BatchParams& p, int r1, int r2,
     }
 }
 
+// A decision warp's inputs for block positions 0..31 of sequence s: the sequence's offsets, lane i's
+// drafted token, its acceptance uniform and (T > 0) that token's target and drafter logits.  None of
+// them is written by the statistics kernel, so when the chain's first kernel started in plain stream
+// order (every earlier kernel complete, `inputs_early`) the warp loads them before its grid-dependency
+// wait, while the statistics still stream; otherwise (a chain behind kernels that may still be writing
+// the logits) right after it.  That takes two dependent round trips (offsets -> tokens -> logits) off
+// the path behind the statistics.
+struct DecideIn {
+    int d0, g, x;
+    float u, tx, dx;
+};
+template <bool GREEDY>
+__device__ __forceinline__ DecideIn decide_inputs(const BatchParams& p, int s, int lane) {
+    DecideIn q;
+    q.d0 = p.cu_draft[s];
+    q.g = p.cu_draft[s + 1] - q.d0;
+    const bool draft = lane < q.g;
+    q.x = draft ? p.tokens[q.d0 + lane] : -1;
+    q.u = !GREEDY && draft ? p.u_accept[q.d0 + lane] : 1.f;
+    q.tx = -INFINITY;
+    q.dx = -INFINITY;
+    if (!GREEDY && draft && q.x >= 0 && q.x < p.vocab) {
+        q.tx = p.target[(size_t)(q.d0 + s + lane) * p.vocab + q.x];
+        q.dx = p.draft[(size_t)(q.d0 + lane) * p.vocab + q.x];
+    }
+    return q;
+}
+
 // Greedy decisions (T = 0) of sequence s by one warp, one lane per block position (32 at a time): lane
 // i <= gamma merges target row i's (max, lowest index) from its chunks' and compares drafted token i
 // with it; the first mismatch k by ballot; the emitted token is row k's argmax (the bonus row's when
 // every draft matches).
-__device__ __forceinline__ void decide_greedy(const BatchParams& p, int s, int lane) {
-    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
+__device__ __forceinline__ void decide_greedy(const BatchParams& p, int s, int lane, const DecideIn& in) {
+    const int d0 = in.d0, g = in.g, t0 = d0 + s;
     int k = g, emitted = 0, bonus = 0;
     for (int i0 = 0; i0 <= g; i0 += 32) {
         const int i = i0 + lane;
-        const int x = i < g ? p.tokens[d0 + i] : -1;
+        const int x = i0 == 0 ? in.x : (i < g ? p.tokens[d0 + i] : -1);
         float2 st, none;
         merge_rows<true>(p, i <= g ? t0 + i : -1, -1, st, none);
         int am = __float_as_int(st.y);
@@ -245,23 +276,27 @@ __device__ __forceinline__ void decide_greedy(const BatchParams& p, int s, int l
 // writer CTA also writes n_accepted, accept_prob and the out_tokens slots other than the emitted
 // token's, and reports draft tokens outside the vocabulary; the others stop at the first block of 32
 // positions that holds a rejection.
-__device__ __forceinline__ void decide_draw(const BatchParams& p, int s, int lane, bool writer, DrawPair* d) {
-    const int d0 = p.cu_draft[s], g = p.cu_draft[s + 1] - d0, t0 = d0 + s;
+__device__ __forceinline__ void decide_draw(const BatchParams& p, int s, int lane, bool writer, DrawPair* d,
+                                            const DecideIn& in) {
+    const int d0 = in.d0, g = in.g, t0 = d0 + s;
     int k = g;
     float2 stk = make_float2(-INFINITY, 0.f), sdk = stk, bonus = stk;
     for (int i0 = 0; i0 <= g; i0 += 32) {
         const int i = i0 + lane;
         const bool draft = i < g;
         // every load at once: the tokens (their logits follow), the uniforms, both rows' chunk statistics
-        const int x = draft ? p.tokens[d0 + i] : -1;
-        const float u = draft ? p.u_accept[d0 + i] : 1.f;
+        const int x = i0 == 0 ? in.x : (draft ? p.tokens[d0 + i] : -1);
+        const float u = i0 == 0 ? in.u : (draft ? p.u_accept[d0 + i] : 1.f);
         float2 st, sd;
         merge_rows<false>(p, i <= g ? t0 + i : -1, draft ? p.rows_t + d0 + i : -1, st, sd);
         bool rej = false;
         if (draft) {
             const bool valid = x >= 0 && x < p.vocab;
             float tx = -INFINITY, dx = -INFINITY;
-            if (valid) {
+            if (i0 == 0) {
+                tx = in.tx;
+                dx = in.dx;
+            } else if (valid) {
                 tx = p.target[(size_t)(t0 + i) * p.vocab + x];
                 dx = p.draft[(size_t)(d0 + i) * p.vocab + x];
             }
@@ -313,9 +348,13 @@ __device__ __forceinline__ void decide_draw(const BatchParams& p, int s, int lan
 // ---- 2. greedy decisions (T = 0): one warp per sequence.  (At T > 0 the draw kernel decides.)
 __global__ void __launch_bounds__(kBThreads) batch_decide_kernel(const BatchParams p) {
     griddep_launch_dependents();
-    griddep_wait();
     const int s = blockIdx.x * (kBThreads / 32) + (threadIdx.x >> 5);
-    if (s < p.num_seqs) decide_greedy(p, s, threadIdx.x & 31);
+    DecideIn in = {};
+    if (p.inputs_early && s < p.num_seqs) in = decide_inputs<true>(p, s, threadIdx.x & 31);
+    griddep_wait();
+    if (s >= p.num_seqs) return;
+    if (!p.inputs_early) in = decide_inputs<true>(p, s, threadIdx.x & 31);
+    decide_greedy(p, s, threadIdx.x & 31, in);
 }
 
 // Weights of four entries: (r = max(0, p - q), p) with p = 2^(l*c2 - Mt) / Zt (r = 0 without a draft row).
@@ -395,12 +434,17 @@ __global__ void __launch_bounds__(kBThreads, SPLIT > 1 ? 2 : PH) batch_draw_kern
     __shared__ unsigned long long off_sh, base_sh;
     __shared__ DrawPair d_sh;
     griddep_launch_dependents();
-    griddep_wait();
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int units = p.chunks * SPLIT;  // parts of the sequence's draw, in entry order
     const int s = blockIdx.x / units, unit = blockIdx.x - s * units;
     const int chunk = unit / SPLIT, sub = unit - chunk * SPLIT;
-    if (warp == 0) decide_draw(p, s, lane, unit == 0, &d_sh);
+    DecideIn in = {};
+    if (p.inputs_early && warp == 0) in = decide_inputs<false>(p, s, lane);
+    griddep_wait();
+    if (warp == 0) {
+        if (!p.inputs_early) in = decide_inputs<false>(p, s, lane);
+        decide_draw(p, s, lane, unit == 0, &d_sh, in);
+    }
     __syncthreads();
     const DrawPair d = d_sh;
     constexpr int kSeg = kBThreads / 32 * kBSegs;  // 128 segments per chunk
@@ -653,6 +697,7 @@ BatchParams batch_params(const AcceptArgs& a, int* tickets, void* draw_scratch) 
     w += align_up((size_t)a.num_seqs * p.chunks * kMaxDrawSplit * sizeof(ulonglong2), 256);
     p.segm = reinterpret_cast<unsigned long long*>(w);
     p.tickets = tickets;
+    p.inputs_early = 0;
     p.err = a.err_word;
     return p;
 }
@@ -667,6 +712,7 @@ int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* s
     uint8_t* w = static_cast<uint8_t*>(scratch);
     BatchParams p = batch_params(a, tickets, w + align_up(rows * chunks * sizeof(float2), 256));
     p.part = reinterpret_cast<float2*>(w);
+    p.inputs_early = 1;  // the statistics kernel starts in plain stream order
     const bool greedy = a.temperature == 0.f, vec = batch_vec(a, greedy);
     if (greedy) return vec ? run_batch<true, true>(p, sm_count, stream) : run_batch<true, false>(p, sm_count, stream);
     return vec ? run_batch<false, true>(p, sm_count, stream) : run_batch<false, false>(p, sm_count, stream);
