@@ -27,9 +27,14 @@
  *     they return before the GPU has run it and never synchronize, except bp_get_status.
  *   - `workspace` is caller-owned device scratch of at least the size the matching
  *     *_workspace_size function returns, 256-byte aligned, ZERO-FILLED BEFORE ITS FIRST
- *     USE.  Every call leaves it in a state the next call can use (counters back at zero);
- *     its first 16 bytes hold a sticky device error word read by bp_get_status.  Two calls
- *     that may run concurrently need distinct workspaces.
+ *     USE.  Every call puts its own counters back at zero, so the next call of the same
+ *     entry point with the same *_workspace_size arguments can follow on it directly.  Its
+ *     other scratch keeps data, and the counters of a call with other size arguments (or of
+ *     another entry point) may lie where that data is: zero-fill the workspace again before
+ *     such a call (spec_accept's per-sequence tickets come first, in 256-byte units of 64
+ *     sequences, so there only a call with more of those units than an earlier one needs
+ *     this).  Its first 16 bytes hold a sticky device error word read by bp_get_status.  Two
+ *     calls that may run concurrently need distinct workspaces.
  *   - Host-checkable problems (NULL pointers, unsupported shapes, a workspace that is too
  *     small) return an error code immediately and enqueue nothing.  Problems only the GPU
  *     sees (a draft token id outside [0, V), a bounded wait that timed out) set the
