@@ -30,6 +30,7 @@
 
 #include <algorithm>
 #include <mutex>
+#include <type_traits>
 
 #include "common.cuh"
 #include "ptx_sm103.cuh"
@@ -721,44 +722,84 @@ __global__ void __launch_bounds__(kThreads, 1)
             const int nmy = max(0, min(m_valid, rbeg + per) - rbeg);
             // one round of remote loads per owned row: a warp takes the row, lane c its 16-byte chunk c of
             // every peer's partial O and, for c below the cluster size, peer c's (m, l); the weights then
-            // go round the warp by shuffles
+            // go round the warp by shuffles.  With more owned rows than warps a warp takes two rows per pass
+            // (rows w and w + 6 of warp w), so up to twelve owned rows take one pass
             static_assert(kD / 4 == 32 && kThreads % 32 == 0, "a warp's 32 items are one row");
-            for (int item = tid; item < nmy * (kD / 4); item += kThreads) {
-                const int rr = item / (kD / 4);
+            const int nitems = nmy * (kD / 4);
+            // one pass: the row of `item` and (PAIR, when present) the row six further, their loads in flight
+            // together and their shuffle chains interleaved
+            auto merge_pass = [&](auto pair_tag, int item) {
+                constexpr bool PAIR = decltype(pair_tag)::value;
+                const bool two = PAIR && item + kThreads < nitems;  // warp-uniform
                 const int c = item % (kD / 4);
-                const int row = rbeg + rr;
-                const float* src = opart + row * kD + ((c ^ (row & 31)) * 4);
-                float4 v[kMaxCluster];
+                const int rowa = rbeg + item / (kD / 4), rowb = rowa + kThreads / 32;
+                float4 va[kMaxCluster], vb[kMaxCluster];
+                const float* srca = opart + rowa * kD + ((c ^ (rowa & 31)) * 4);
+                const float* srcb = opart + rowb * kD + ((c ^ (rowb & 31)) * 4);
 #pragma unroll
-                for (int pr = 0; pr < kMaxCluster; ++pr)
-                    if (pr < (int)CS) v[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(src), pr);
-                const float2 ml = c < (int)CS ? *cluster.map_shared_rank(&row_ml[row], c) : make_float2(-INFINITY, 0.f);
-                float M = ml.x;
+                for (int pr = 0; pr < kMaxCluster; ++pr) {
+                    if (pr < (int)CS) va[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(srca), pr);
+                    if constexpr (PAIR) {
+                        if (pr < (int)CS && two)
+                            vb[pr] = *cluster.map_shared_rank(reinterpret_cast<const float4*>(srcb), pr);
+                        else
+                            vb[pr] = make_float4(0.f, 0.f, 0.f, 0.f);
+                    }
+                }
+                const float2 mla = c < (int)CS ? *cluster.map_shared_rank(&row_ml[rowa], c) : make_float2(-INFINITY, 0.f);
+                float2 mlb = make_float2(-INFINITY, 0.f);
+                if constexpr (PAIR) {
+                    if (c < (int)CS && two) mlb = *cluster.map_shared_rank(&row_ml[rowb], c);
+                }
+                float Ma = mla.x, Mb = mlb.x;
 #pragma unroll
-                for (int o = 16; o >= 1; o >>= 1) M = fmaxf(M, __shfl_xor_sync(0xffffffffu, M, o));
-                const float wl = ml.x == -INFINITY ? 0.f : fast_exp2(ml.x - M);
-                float Lsum = wl * ml.y;
+                for (int o = 16; o >= 1; o >>= 1) {
+                    Ma = fmaxf(Ma, __shfl_xor_sync(0xffffffffu, Ma, o));
+                    if constexpr (PAIR) Mb = fmaxf(Mb, __shfl_xor_sync(0xffffffffu, Mb, o));
+                }
+                const float wla = mla.x == -INFINITY ? 0.f : fast_exp2(mla.x - Ma);
+                const float wlb = mlb.x == -INFINITY ? 0.f : fast_exp2(mlb.x - Mb);
+                float La = wla * mla.y, Lb = wlb * mlb.y;
 #pragma unroll
-                for (int o = 16; o >= 1; o >>= 1) Lsum += __shfl_xor_sync(0xffffffffu, Lsum, o);
-                float4 acc = make_float4(0.f, 0.f, 0.f, 0.f);
+                for (int o = 16; o >= 1; o >>= 1) {
+                    La += __shfl_xor_sync(0xffffffffu, La, o);
+                    if constexpr (PAIR) Lb += __shfl_xor_sync(0xffffffffu, Lb, o);
+                }
+                float4 acca = make_float4(0.f, 0.f, 0.f, 0.f), accb = acca;
 #pragma unroll
                 for (int pr = 0; pr < kMaxCluster; ++pr) {
                     if (pr < (int)CS) {
-                        const float w = __shfl_sync(0xffffffffu, wl, pr);
-                        acc.x += w * v[pr].x;
-                        acc.y += w * v[pr].y;
-                        acc.z += w * v[pr].z;
-                        acc.w += w * v[pr].w;
+                        const float wa = __shfl_sync(0xffffffffu, wla, pr);
+                        acca.x += wa * va[pr].x;
+                        acca.y += wa * va[pr].y;
+                        acca.z += wa * va[pr].z;
+                        acca.w += wa * va[pr].w;
+                        if constexpr (PAIR) {
+                            const float wb = __shfl_sync(0xffffffffu, wlb, pr);
+                            accb.x += wb * vb[pr].x;
+                            accb.y += wb * vb[pr].y;
+                            accb.z += wb * vb[pr].z;
+                            accb.w += wb * vb[pr].w;
+                        }
                     }
                 }
-                const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
-                const int lr = row0 + row;
-                const size_t orow = (size_t)(one.q0 + lr / G) * p.num_q_heads + one.h * G + lr % G;
-                uint2 w2;
-                w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
-                w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
-                *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
-                if (p.lse && c == 0) p.lse[orow] = (M + __log2f(Lsum)) * kLn2;
+                auto store = [&](int row, float4 acc, float M, float Lsum) {
+                    const float inv = Lsum > 0.f ? 1.f / Lsum : 0.f;
+                    const int lr = row0 + row;
+                    const size_t orow = (size_t)(one.q0 + lr / G) * p.num_q_heads + one.h * G + lr % G;
+                    uint2 w2;
+                    w2.x = pack_bf16x2(acc.x * inv, acc.y * inv);
+                    w2.y = pack_bf16x2(acc.z * inv, acc.w * inv);
+                    *reinterpret_cast<uint2*>(p.o + orow * kD + c * 4) = w2;
+                    if (p.lse && c == 0) p.lse[orow] = (M + __log2f(Lsum)) * kLn2;
+                };
+                store(rowa, acca, Ma, La);
+                if (two) store(rowb, accb, Mb, Lb);
+            };
+            if (nmy > kThreads / 32) {  // more owned rows than warps: two rows per warp and pass
+                for (int item = tid; item < nitems; item += 2 * kThreads) merge_pass(std::true_type{}, item);
+            } else {
+                for (int item = tid; item < nitems; item += kThreads) merge_pass(std::false_type{}, item);
             }
             cluster.sync();  // no CTA leaves while peers may still read its shared memory
         }
@@ -1061,18 +1102,26 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     attr[1].id = cudaLaunchAttributeProgrammaticStreamSerialization;
     attr[1].val.programmaticStreamSerializationAllowed = 1;
 
-    // cluster split: the largest split of each unit's keys for which every unit's cluster is resident in
-    // the same wave (a unit left for a second wave would double the time); the tiles of the longest unit
-    // per CTA set the time: minimise them, then prefer the smallest cluster, whose merge is cheapest
-    int cs = 1, best = max_tiles;
+    // cluster split: a split of each unit's keys for which every unit's cluster is resident in the same
+    // wave (a unit left for a second wave would double the time).  The tiles of the longest unit per CTA
+    // set the time: minimise them; among equal counts take the smallest cluster whose merge needs the
+    // fewest passes (a pass merges up to 12 owned rows per CTA).  A cluster's barriers and merge cost
+    // about three tiles of one CTA's chain (batch 1, Qwen3-4B heads: 2 tiles 5.3 us alone against
+    // 7.3-9.9 us in clusters; 4 tiles 7.6 us alone, 7.4 us in clusters of 6), so a split that saves
+    // fewer than three tiles stays whole
+    const int m_rows = std::min(kM, a.max_q_len * G);
+    int cs = 1, best = max_tiles, best_pass = 0;
     for (int c = 2; c <= kMaxCluster; ++c) {
         if (c > max_tiles || units > max_active[c] || units * c > dev.sm_count) continue;
         const int per = (max_tiles + c - 1) / c;
-        if (per < best) {
+        const int passes = ((m_rows + c - 1) / c + 11) / 12;
+        if (per < best || (per == best && cs > 1 && passes < best_pass)) {
             best = per;
             cs = c;
+            best_pass = passes;
         }
     }
+    if (cs > 1 && max_tiles - best < 3) cs = 1;
 
     // flat split: the tiles of every sequence's query tiles cut evenly over groups of CTAs, one CTA per KV
     // head and per SM (at most kAttnFlatMaxGrid in all, and no more groups than one head has tiles); units
@@ -1082,7 +1131,8 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     // run (8 x 32K keys: 170 vs 175 us), and where the cluster split needs three or more waves (64 x 528
     // keys: 46 vs 50 us); elsewhere the second kernel and the stretch boundaries cost more than the idle
     // SMs (1 x 2K keys: 13.8 vs 9.3 us; 16 x 4K: 60 vs 52 us; the ragged 32: 109 vs 100 us).
-    // BP_ATTENTION_SPLIT=flat or =cluster overrides the choice (for tests and measurements).
+    // BP_ATTENTION_SPLIT=flat or =cluster overrides the choice, =cluster:N also the cluster size (for tests
+    // and measurements).
     const long long tiles_bound = (long long)a.num_seqs * m_tiles * max_tiles;
     const int ngroups = (int)std::min<long long>(std::min(dev.sm_count, kAttnFlatMaxGrid) / a.num_kv_heads,
                                                  tiles_bound);
@@ -1093,8 +1143,14 @@ int launch_attention_bf16(const AttentionArgs& a, const DeviceInfo& dev, cudaStr
     bool flat = flat_ok && ((cluster_ctas * 10 <= 9LL * dev.sm_count && tiles_bound >= 64LL * ngroups) ||
                             cluster_ctas >= 3LL * dev.sm_count);
     if (const char* force = getenv("BP_ATTENTION_SPLIT")) {
-        if (strcmp(force, "flat") == 0) flat = flat_ok;
-        else if (strcmp(force, "cluster") == 0) flat = false;
+        if (strcmp(force, "flat") == 0) {
+            flat = flat_ok;
+        } else if (strncmp(force, "cluster", 7) == 0) {
+            flat = false;
+            // cluster:N forces clusters of N CTAs when every unit's cluster is then resident in one wave
+            const int c = force[7] == ':' ? atoi(force + 8) : 0;
+            if (c >= 2 && c <= kMaxCluster && units <= max_active[c] && units * c <= dev.sm_count) cs = c;
+        }
     }
     cudaError_t e;
     if (flat) {

@@ -40,10 +40,13 @@ def attention_ws(a: dict, split: str = "auto"):
 @contextlib.contextmanager
 def forced_split(split: str):
     """The library's choice between the flat and the cluster split of the keys ("auto"), or one of them
-    forced through BP_ATTENTION_SPLIT, which the library reads at every call."""
+    forced through BP_ATTENTION_SPLIT, which the library reads at every call ("cluster3": the cluster
+    split in clusters of 3, so that short contexts too take the distributed-shared-memory merge)."""
     old = os.environ.get("BP_ATTENTION_SPLIT")
     if split in ("flat", "cluster"):
         os.environ["BP_ATTENTION_SPLIT"] = split
+    elif split == "cluster3":
+        os.environ["BP_ATTENTION_SPLIT"] = "cluster:3"
     else:
         os.environ.pop("BP_ATTENTION_SPLIT", None)
     try:
@@ -57,7 +60,7 @@ def forced_split(split: str):
 
 def run_attention(a: dict, mask: int, split: str = "auto"):
     """CUDA path on the whole workload; returns (o fp32 numpy, lse numpy).  split: "auto" (the library
-    chooses), "flat" or "cluster" (forced)."""
+    chooses), "flat", "cluster" or "cluster3" (forced)."""
     q, k, v = to_dev(a["q"], a["dtype"]), to_dev(a["k"], a["dtype"]), to_dev(a["v"], a["dtype"])
     cu_q, cu_kv = to_dev(a["cu_q"]), to_dev(a["cu_kv"])
     lse = torch.empty(q.shape[0], q.shape[1], dtype=torch.float32, device=dev())

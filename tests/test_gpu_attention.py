@@ -2,7 +2,9 @@
 
 Tolerance: max |O - O_ref| / max |O_ref| <= 2e-2 per (sequence, query head) slice (bf16 inputs,
 fp32 accumulation); log-sum-exp within 2e-3.  Small ragged cases are compared in full, on both
-splits of the keys (the flat split and the cluster split, each forced); the full-size workloads run
+splits of the keys (the flat split and the cluster split, each forced, the cluster split also in
+clusters of 3: contexts this short stay in one CTA per unit when the library chooses, so the forced
+clusters keep the distributed-shared-memory merge covered at every group size); the full-size workloads run
 exactly as the benchmark launches them (the library's own choice of split) and are compared on
 sampled sequences (and KV heads for the 32K-context case).
 """
@@ -44,14 +46,14 @@ def _check(a, mask, seqs=None, kv_head=None, split="auto"):
     ((2048,), (16,)),                                # Qwen3-4B verify shape, one sequence
     ((4000, 10, 255, 256, 257), (16, 16, 16, 16, 16)),
 ])
-@pytest.mark.parametrize("split", ["flat", "cluster"])
+@pytest.mark.parametrize("split", ["flat", "cluster", "cluster3"])
 def test_ragged_small(ctx, block, mask, split):
     w = wl.custom(seed=sum(ctx) + len(block), ctx=ctx, block=block, num_q_heads=32, num_kv_heads=8)
     _check(wl.attention_inputs(w), mask, split=split)
 
 
 @pytest.mark.parametrize("hq,hkv", [(8, 8), (64, 8), (16, 2), (4, 1), (24, 8)])
-@pytest.mark.parametrize("split", ["flat", "cluster"])
+@pytest.mark.parametrize("split", ["flat", "cluster", "cluster3"])
 def test_group_sizes(hq, hkv, split):
     # (24, 8): a group of 3 does not divide the 128-row tile, so Q is gathered without TMA (cluster split)
     w = wl.custom(seed=hq * 10 + hkv, ctx=(300, 77), block=(12, 31), num_q_heads=hq, num_kv_heads=hkv)
