@@ -21,10 +21,11 @@
 //      max(0, p_k - q_k) and of p_k in exact 2^-52 fixed point; the last CTA of the sequence (ticket)
 //      finds the part and the 128-entry segment where the inverse CDF crosses u_s * total from the
 //      stored masses, then the entry from that segment's 128 logits, and writes the emitted token.
-// Only the one draw row pair per sequence is read twice.  The decisions and the draw chain behind the
-// statistics with programmatic dependent launch; the statistics kernel launches in plain stream order,
-// so their decision warps load the inputs that kernel does not write (offsets, drafted tokens, uniforms,
-// the drafted tokens' logits) before their grid-dependency wait.
+// Only the one draw row pair per sequence is read twice.  Every kernel of the chain launches with
+// programmatic dependent launch.  The statistics kernel releases the decisions (or the draw) only once
+// its own grid-dependency wait has returned, i.e. once every kernel before the chain is complete, so
+// their decision warps load the inputs that the statistics kernel does not write (offsets, drafted
+// tokens, uniforms, the drafted tokens' logits) before their own wait.
 #include <cuda_runtime.h>
 #include <math.h>
 
@@ -58,7 +59,7 @@ struct BatchParams {
     ulonglong2* ctot;  // [num_seqs][chunks * parts] draw masses of r and p of the chunks' parts (fixed point)
     unsigned long long* segm;  // [num_seqs][chunks][2][128] their segment masses
     int* tickets;      // [num_seqs], zero between calls
-    int inputs_early;  // every input was written before the chain's first kernel started (see DecideIn)
+    int inputs_early;  // every input was complete when the statistics kernel released this one (DecideIn)
     unsigned int* err;
 };
 
@@ -102,8 +103,8 @@ struct DrawPair {
 template <bool GREEDY, bool VEC>
 __global__ void __launch_bounds__(kBThreads) batch_stats_kernel(const BatchParams p) {
     __shared__ float2 red[kBThreads / 32];
-    griddep_launch_dependents();
     griddep_wait();
+    griddep_launch_dependents();  // after the wait: the decisions kernel may read inputs early (DecideIn)
     const int tid = threadIdx.x, lane = tid & 31, warp = tid >> 5;
     const int row = blockIdx.x / p.chunks, chunk = blockIdx.x - row * p.chunks;
     const int v0 = chunk * kBChunk, n = min(kBChunk, p.vocab - v0);
@@ -205,11 +206,11 @@ __device__ __forceinline__ void merge_rows(const BatchParams& p, int r1, int r2,
 
 // A decision warp's inputs for block positions 0..31 of sequence s: the sequence's offsets, lane i's
 // drafted token, its acceptance uniform and (T > 0) that token's target and drafter logits.  None of
-// them is written by the statistics kernel, so when the chain's first kernel started in plain stream
-// order (every earlier kernel complete, `inputs_early`) the warp loads them before its grid-dependency
-// wait, while the statistics still stream; otherwise (a chain behind kernels that may still be writing
-// the logits) right after it.  That takes two dependent round trips (offsets -> tokens -> logits) off
-// the path behind the statistics.
+// them is written by the statistics kernel, and the statistics kernel releases its dependents only
+// after its own grid-dependency wait (every earlier kernel complete), so behind it (`inputs_early`)
+// the warp loads them before its grid-dependency wait, while the statistics still stream; behind the
+// streamed LM head, which writes the logits, right after it.  That takes two dependent round trips
+// (offsets -> tokens -> logits) off the path behind the statistics.
 struct DecideIn {
     int d0, g, x;
     float u, tx, dx;
@@ -633,9 +634,11 @@ size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
 
 namespace {
 // pdl: the prologue may overlap the previous kernel's tail (programmatic stream serialization).  The
-// statistics kernel, first of the chain, launches in plain stream order: behind a long kernel its
-// thousands of CTAs were placed early and waiting on every SM, and a step of the ragged batch
-// (attention, then the acceptance) took 220 us instead of 201.
+// statistics kernel too: its CTAs wait for the previous kernel at their start.  Behind a kernel that
+// releases its dependents before its last wave has started, its thousands of CTAs would take the SMs
+// that wave needs (the attention kernels release theirs at their end: released at their start, a step
+// of the ragged batch ran 720-820 us instead of 195).  Behind the flat-split attention's merge the
+// chained launch takes 1.8 us off the long-context step (200.3 against 202.1 us).
 template <typename Kernel>
 int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_t stream, bool pdl = true) {
     if (blocks == 0) return BP_OK;
@@ -669,7 +672,7 @@ int run_decisions(const BatchParams& p, int sm_count, cudaStream_t stream) {
 template <bool GREEDY, bool VEC>
 int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
-    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream, false);
+    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
     return rc != BP_OK ? rc : run_decisions<GREEDY, VEC>(p, sm_count, stream);
 }
 
@@ -712,7 +715,7 @@ int launch_accept_batch(const AcceptArgs& a, int sm_count, int* tickets, void* s
     uint8_t* w = static_cast<uint8_t*>(scratch);
     BatchParams p = batch_params(a, tickets, w + align_up(rows * chunks * sizeof(float2), 256));
     p.part = reinterpret_cast<float2*>(w);
-    p.inputs_early = 1;  // the statistics kernel starts in plain stream order
+    p.inputs_early = 1;  // the statistics kernel releases the decisions after its own wait
     const bool greedy = a.temperature == 0.f, vec = batch_vec(a, greedy);
     if (greedy) return vec ? run_batch<true, true>(p, sm_count, stream) : run_batch<true, false>(p, sm_count, stream);
     return vec ? run_batch<false, true>(p, sm_count, stream) : run_batch<false, false>(p, sm_count, stream);
