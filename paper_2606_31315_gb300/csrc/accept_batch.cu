@@ -637,8 +637,7 @@ namespace {
 // statistics kernel too: its CTAs wait for the previous kernel at their start.  Behind a kernel that
 // releases its dependents before its last wave has started, its thousands of CTAs would take the SMs
 // that wave needs (the attention kernels release theirs at their end: released at their start, a step
-// of the ragged batch ran 720-820 us instead of 195).  Behind the flat-split attention's merge the
-// chained launch takes 1.8 us off the long-context step (200.3 against 202.1 us).
+// of the ragged batch ran 720-820 us instead of 195).
 template <typename Kernel>
 int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_t stream, bool pdl = true) {
     if (blocks == 0) return BP_OK;
@@ -672,7 +671,9 @@ int run_decisions(const BatchParams& p, int sm_count, cudaStream_t stream) {
 template <bool GREEDY, bool VEC>
 int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
-    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream);
+    // chained at T > 0 (long-context step 200.3 against 202.0 us in plain order); at T = 0, where the
+    // statistics CTAs are small enough to sit eight to an SM, plain order (184.5 against 187.1 us)
+    const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream, !GREEDY);
     return rc != BP_OK ? rc : run_decisions<GREEDY, VEC>(p, sm_count, stream);
 }
 
