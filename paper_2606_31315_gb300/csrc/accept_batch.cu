@@ -634,10 +634,10 @@ size_t accept_batch_scratch_bytes(int num_seqs, int total_draft, int vocab) {
 
 namespace {
 // pdl: the prologue may overlap the previous kernel's tail (programmatic stream serialization).  The
-// statistics kernel too: its CTAs wait for the previous kernel at their start.  Behind a kernel that
-// releases its dependents before its last wave has started, its thousands of CTAs would take the SMs
-// that wave needs (the attention kernels release theirs at their end: released at their start, a step
-// of the ragged batch ran 720-820 us instead of 195).
+// statistics kernel too (at T > 0): its CTAs wait for the previous kernel at their start.  Behind a
+// kernel of several waves that releases its dependents early, its thousands of CTAs would take the SMs
+// those waves need; the attention kernels release theirs early only when they run in one wave
+// (released early from two waves, a step of the ragged batch ran 720-820 us instead of 195).
 template <typename Kernel>
 int launch_pdl(Kernel kernel, unsigned blocks, const BatchParams& p, cudaStream_t stream, bool pdl = true) {
     if (blocks == 0) return BP_OK;
@@ -671,8 +671,9 @@ int run_decisions(const BatchParams& p, int sm_count, cudaStream_t stream) {
 template <bool GREEDY, bool VEC>
 int run_batch(const BatchParams& p, int sm_count, cudaStream_t stream) {
     const int rows = p.rows_t + (GREEDY ? 0 : p.total_draft);
-    // chained at T > 0 (long-context step 200.3 against 202.0 us in plain order); at T = 0, where the
-    // statistics CTAs are small enough to sit eight to an SM, plain order (184.5 against 187.1 us)
+    // chained at T > 0 (long-context step 200.3 against 202.0 us in plain order, graphs of 32 steps); at
+    // T = 0, where the statistics CTAs are small enough to sit eight to an SM, plain order (184.5 against
+    // 187.1 us chained)
     const int rc = launch_pdl(batch_stats_kernel<GREEDY, VEC>, (unsigned)(rows * p.chunks), p, stream, !GREEDY);
     return rc != BP_OK ? rc : run_decisions<GREEDY, VEC>(p, sm_count, stream);
 }
